@@ -1,0 +1,148 @@
+"""Oracle pins for the flow transformer on an active subset (Sec. 4.2,
+Supp. Sec. F) and for the whole sampler (Algorithm 1)."""
+import numpy as np
+import pytest
+
+from paper_2511_22533_gb300 import synth
+
+TINY = synth.SHAPES["tiny"]
+
+
+@pytest.fixture(scope="module")
+def tiny(orc):
+    blob = synth.weights_blob(TINY, 0)
+    m = orc.Model(TINY, blob)
+    cond = synth.cond_tokens(TINY, 2, 0)
+    S = synth.latents(TINY, 2, 0)
+    kv = m.cond_kv(cond[0])
+    return dict(model=m, blob=blob, cond=cond, S=S, kv=kv)
+
+
+def test_forward_shapes_and_finite(tiny):
+    m, S, kv = tiny["model"], tiny["S"][0], tiny["kv"]
+    v = m.forward(S, np.arange(TINY.tokens), 0.8, kv)
+    assert v.shape == (TINY.tokens, TINY.channels) and np.isfinite(v).all()
+    assert 0.05 < v.std() < 20
+
+
+def test_forward_permutation_equivariant(tiny):
+    # attention is permutation-equivariant over the active set: reordering the
+    # active list reorders the outputs and changes nothing else
+    m, S, kv = tiny["model"], tiny["S"][0], tiny["kv"]
+    rng = np.random.default_rng(0)
+    idx = np.sort(rng.choice(TINY.tokens, 200, replace=False)).astype(np.int32)
+    p = rng.permutation(200)
+    v = m.forward(S, idx, 0.7, kv)
+    vp = m.forward(S, idx[p], 0.7, kv)
+    np.testing.assert_allclose(vp, v[p], rtol=1e-5, atol=1e-5)
+
+
+def test_forward_ignores_cached_tokens(tiny):
+    # self-attention runs among the active tokens only (Sec. 4.2): the latent
+    # of a token outside I_active cannot influence any active output
+    m, S, kv = tiny["model"], tiny["S"][0].copy(), tiny["kv"]
+    idx = np.arange(0, TINY.tokens, 3, dtype=np.int32)
+    v = m.forward(S, idx, 0.6, kv)
+    S[1] += 100.0
+    S[TINY.tokens - 1] -= 50.0
+    v2 = m.forward(S, idx, 0.6, kv)
+    np.testing.assert_array_equal(v, v2)
+
+
+def test_forward_depends_on_active_neighbours(tiny):
+    m, S, kv = tiny["model"], tiny["S"][0].copy(), tiny["kv"]
+    idx = np.arange(0, 64, dtype=np.int32)
+    v = m.forward(S, idx, 0.6, kv)
+    S[5] += 1.0
+    v2 = m.forward(S, idx, 0.6, kv)
+    assert np.abs(v2 - v)[np.arange(64) != 5].max() > 0  # coupling through attention
+
+
+def test_zeroed_branches_make_block_identity(orc):
+    # with every modulation of a block zero (gates 0) and its cross-attention
+    # output projection zero, the block passes the residual stream through:
+    # an L=2 model with block 1 zeroed equals the L=1 model sharing block 0.
+    s2 = synth.ModelShape(4, 8, 48, 2, 2, 4, 5, 48, 4, 8)
+    s1 = synth.ModelShape(4, 8, 48, 1, 2, 4, 5, 48, 4, 8)
+    b2 = synth.weights_blob(s2, 3)
+    for name in ("mod_w", "mod_b", "co_w", "co_b"):
+        synth.set_weight(b2, s2, name, 1, 0.0)
+    b1 = synth.weights_blob(s1, 3)
+    offs2, _ = synth.weight_offsets(s2)
+    offs1, _ = synth.weight_offsets(s1)
+    for (name, blk), (off1, dims) in offs1.items():
+        off2, _ = offs2[(name, blk)]
+        n = int(np.prod(dims))
+        b1[off1:off1 + n] = b2[off2:off2 + n]
+    m1, m2 = orc.Model(s1, b1), orc.Model(s2, b2)
+    rng = np.random.default_rng(1)
+    S = rng.standard_normal((64, 8)).astype(np.float32)
+    cond = synth.cond_tokens(s2, 1, 2)[0]
+    idx = np.arange(64, dtype=np.int32)
+    v1 = m1.forward(S, idx, 0.5, m1.cond_kv(cond))
+    v2 = m2.forward(S, idx, 0.5, m2.cond_kv(cond))
+    np.testing.assert_allclose(v2, v1, rtol=1e-6, atol=1e-6)
+    # and a nonzero gate does change the output
+    b3 = b2.copy()
+    synth.set_weight(b3, s2, "mod_b", 1, 0.5)
+    m3 = orc.Model(s2, b3)
+    v3 = m3.forward(S, idx, 0.5, m3.cond_kv(cond))
+    assert np.abs(v3 - v2).max() > 1e-3
+
+
+def test_sample_quota_zero_is_plain_euler(tiny, orc):
+    # quota 0 at every step must reproduce the uncached sampler exactly
+    m, S, cond = tiny["model"], tiny["S"][:1], tiny["cond"][:1]
+    T = 4
+    out = m.sample(S, cond, T=T, quota_schedule=np.zeros((T, 1), np.int32), tau=0)
+    t = orc.time_schedule(T, 3.0)
+    x = S[0].copy()
+    kv = m.cond_kv(cond[0])
+    vc = np.zeros((TINY.tokens, 8), np.uint16)
+    for k in range(T):
+        v = m.forward(x, np.arange(TINY.tokens), float(t[k]), kv)
+        x, vc = orc.merge_euler(x, np.arange(TINY.tokens, dtype=np.int32), v, vc, float(t[k] - t[k + 1]))
+    np.testing.assert_array_equal(out["S"][0], x)
+    assert np.all(out["n_active"] == TINY.tokens)
+
+
+def test_sample_cached_tokens_carry_velocity(tiny, orc):
+    # a token cached at step k keeps v_t = v_(t-1) bit for bit, so its
+    # acceleration A_i is exactly 0 at step k+1
+    m, S, cond = tiny["model"], tiny["S"][:1], tiny["cond"][:1]
+    T = 4
+    q = np.array([[0], [0], [0], [300]], np.int32)
+    out = m.sample(S, cond, T=T, quota_schedule=q, tau=0)
+    vcache, vprev = out["v_hist"][0, 0], out["v_hist"][1, 0]
+    same = np.all(vcache == vprev, axis=1)
+    assert same.sum() == 300
+    assert out["n_active"][3, 0] == TINY.tokens - 300
+
+
+def test_sample_batch_members_independent(tiny):
+    m, S, cond = tiny["model"], tiny["S"], tiny["cond"]
+    q = np.tile(np.array([[0], [0], [0], [256], [256]], np.int32), (1, 2))
+    both = m.sample(S, cond, T=5, quota_schedule=q, tau=0)
+    one = m.sample(S[1:], cond[1:], T=5, quota_schedule=q[:, 1:], tau=0)
+    np.testing.assert_array_equal(both["S"][1], one["S"][0])
+
+
+def test_sample_pcsc_anchor_and_log(tiny, orc):
+    # Algorithm 1 with PCSC: sigma is measured at the anchor step k_a (Eq. 1)
+    # and the forecast uses it; sigma_override replaces it in the forecast
+    m, S, cond = tiny["model"], tiny["S"][:1], tiny["cond"][:1]
+    T = 8
+    out = m.sample(S, cond, T=T, tau=3)
+    ka = orc.ceil_steps(T, 0.2)
+    assert np.all(out["quota"][:ka] == 0)
+    assert out["sigma"][0] >= 0
+    gate = orc.TauGate(3, 0)
+    for k in range(1, T + 1):
+        c, _ = orc.phase_quota(TINY.tokens, T, 0.2, 0.75, -0.07, 0.7, 3, TINY.gamma_up,
+                               float(out["sigma"][0]), k)
+        assert out["quota"][k - 1, 0] == gate(c)
+    assert np.all(out["n_active"] == TINY.tokens - out["quota"])
+    ov = m.sample(S, cond, T=T, tau=3, sigma_override=np.array([64.0 * 100]))
+    assert ov["sigma"][0] == out["sigma"][0]
+    c6, _ = orc.phase_quota(TINY.tokens, T, 0.2, 0.75, -0.07, 0.7, 3, TINY.gamma_up, 6400.0, ka + 1)
+    assert ov["quota"][ka, 0] == c6
