@@ -1,0 +1,865 @@
+// api.cu -- the C-ABI of libf3dc (include/f3dc.h): handle life cycle,
+// host-side schedule logic (Supp. Sec. D time shift; Sec. 4.2 PCSC;
+// Algorithm 1 phases and tau refresh), the cached step (Algorithm 1 steps
+// 2-3) and the sampler (Algorithm 1), plus kernel-level diagnostic calls.
+#include <cmath>
+#include <cstdio>
+#include <cstring>
+#include <string>
+#include <vector>
+
+#include "../../include/f3dc.h"
+#include "kernels.h"
+
+using namespace f3dc;
+
+namespace {
+
+thread_local std::string g_last_error;
+
+struct BlockOffsets {
+    size_t mod_w, mod_b, qkv_w, qkv_b, qn_g, kn_g, o_w, o_b, ln2_g, ln2_b;
+    size_t cq_w, cq_b, ckv_w, ckv_b, co_w, co_b, fc1_w, fc1_b, fc2_w, fc2_b;
+};
+
+struct Layout {
+    size_t in_w, in_b, t_w1, t_b1, t_w2, t_b2, fmod_w, fmod_b, out_w, out_b, dec_w;
+    std::vector<BlockOffsets> blk;
+    size_t total;
+};
+
+// Walks the layout-v1 tensor order; each tensor starts on a 64-element
+// boundary.
+Layout weight_layout(const f3dc_config &c)
+{
+    Layout L;
+    size_t pos = 0;
+    const size_t W = c.width, C = c.channels, Dc = c.cond_dim, G = c.gamma_up, Wm = (size_t)c.mlp_ratio * W;
+    auto take = [&](size_t n) {
+        size_t o = pos;
+        pos += (n + 63) / 64 * 64;
+        return o;
+    };
+    L.in_w = take(W * C);
+    L.in_b = take(W);
+    L.t_w1 = take(W * 256);
+    L.t_b1 = take(W);
+    L.t_w2 = take(W * W);
+    L.t_b2 = take(W);
+    for (int l = 0; l < c.blocks; ++l) {
+        BlockOffsets b;
+        b.mod_w = take(6 * W * W);
+        b.mod_b = take(6 * W);
+        b.qkv_w = take(3 * W * W);
+        b.qkv_b = take(3 * W);
+        b.qn_g = take(W);
+        b.kn_g = take(W);
+        b.o_w = take(W * W);
+        b.o_b = take(W);
+        b.ln2_g = take(W);
+        b.ln2_b = take(W);
+        b.cq_w = take(W * W);
+        b.cq_b = take(W);
+        b.ckv_w = take(2 * W * Dc);
+        b.ckv_b = take(2 * W);
+        b.co_w = take(W * W);
+        b.co_b = take(W);
+        b.fc1_w = take(Wm * W);
+        b.fc1_b = take(Wm);
+        b.fc2_w = take(W * Wm);
+        b.fc2_b = take(W);
+        L.blk.push_back(b);
+    }
+    L.fmod_w = take(2 * W * W);
+    L.fmod_b = take(2 * W);
+    L.out_w = take(C * W);
+    L.out_b = take(C);
+    L.dec_w = take(C * G);
+    L.total = pos;
+    return L;
+}
+
+bool config_valid(const f3dc_config *c, std::string &why)
+{
+    if (!c) {
+        why = "null config";
+        return false;
+    }
+    const long long N = (long long)c->grid * c->grid * c->grid;
+    if (c->grid < 1 || N % 32 != 0) why = "grid^3 must be a positive multiple of 32";
+    else if (N > ssc_select_max_tokens()) why = "too many tokens for the selection kernel";
+    else if (c->channels != kChannels) why = "channels must be 8";
+    else if (c->width < 128 || c->width % 128 != 0 || c->width > 2048) why = "width must be a multiple of 128 in [128, 2048]";
+    else if (c->heads < 1 || c->width % c->heads != 0) why = "width must be divisible by heads";
+    else if (c->width / c->heads != 32 && c->width / c->heads != 64) why = "head dim must be 32 or 64";
+    else if (c->mlp_ratio != 4) why = "mlp_ratio must be 4";
+    else if (c->blocks < 1) why = "blocks must be >= 1";
+    else if (c->cond_tokens < 1 || c->cond_dim < 64 || c->cond_dim % 64 != 0 || c->cond_dim > 4096)
+        why = "cond_tokens >= 1 and cond_dim a multiple of 64 up to 4096";
+    else if (c->steps < 1) why = "steps must be >= 1";
+    else if (c->max_batch < 1 || c->max_batch > kMaxBatch) why = "max_batch must be in [1, 64]";
+    else if (c->gamma_up < 1 || c->gamma_up > 512) why = "gamma_up must be in [1, 512]";
+    else if (c->refresh_mode != F3DC_REFRESH_PERIOD && c->refresh_mode != F3DC_REFRESH_LITERAL)
+        why = "unknown refresh_mode";
+    else if (!(c->eta > 0.0) || !std::isfinite(c->mu) || !(c->omega >= 0.0 && c->omega <= 1.0) ||
+             !(c->xi >= 0.0 && c->xi <= 1.0) || !(c->rho_a >= 0.0) || !(c->rho_cfg_off >= 0.0))
+        why = "hyperparameter out of range";
+    else
+        return true;
+    return false;
+}
+
+int ceil_steps(int T, double rho) { return (int)std::ceil((double)T * rho); }
+
+// Three-phase budget (Algorithm 1 step 1) with the PCSC forecast (Sec. 4.2).
+int phase_quota(const f3dc_config &c, double sigma, int k, int *phase)
+{
+    const int N = c.grid * c.grid * c.grid;
+    const int ka = ceil_steps(c.steps, c.rho_a), koff = ceil_steps(c.steps, c.rho_cfg_off);
+    double q;
+    if (k <= ka) {
+        *phase = 1;
+        return 0;
+    }
+    if (k < koff) {
+        *phase = 2;
+        const double forecast = sigma * std::exp(c.mu * (double)(k - ka));  // dS_hat_k
+        q = std::floor((double)N - forecast / (double)c.gamma_up);
+    } else {
+        *phase = 3;
+        const int kr = k - koff;
+        if (c.f_corr > 0 && (kr + 1) % c.f_corr == 0) return 0;
+        q = std::floor((double)N * c.xi);
+    }
+    if (!(q > 0.0)) return 0;
+    if (q > (double)N) return N;
+    return (int)q;
+}
+
+// Error-accumulation elimination (Sec. 4.3 Phase 2; Algorithm 1 SSC).
+int tau_gate(const f3dc_config &c, int quota, int32_t *consec)
+{
+    if (quota > 0 && c.tau > 0) {
+        const int limit = c.refresh_mode == F3DC_REFRESH_PERIOD ? c.tau - 1 : c.tau;
+        if (*consec >= limit) quota = 0;
+    }
+    if (quota > 0) *consec += 1;
+    else *consec = 0;
+    return quota;
+}
+
+void time_schedule(const f3dc_config &c, float *t)
+{
+    for (int k = 1; k <= c.steps + 1; ++k) {
+        const double tl = 1.0 - (double)(k - 1) / (double)c.steps;
+        t[k - 1] = (float)(c.eta * tl / (1.0 + (c.eta - 1.0) * tl));
+    }
+}
+
+// Fixed 3-D sin-cos position embedding of every token (host, fp64, once):
+// per axis (d, h, w) F = W / 6 frequencies 10000^(-f/F), [sin | cos] blocks,
+// the remaining W - 6F entries zero.
+std::vector<float> position_table(int grid, int W)
+{
+    const int N = grid * grid * grid, F = W / 6;
+    std::vector<float> pos((size_t)N * W, 0.0f);
+    for (int i = 0; i < N; ++i) {
+        const int coord[3] = {i / (grid * grid), (i / grid) % grid, i % grid};
+        float *row = pos.data() + (size_t)i * W;
+        for (int a = 0; a < 3; ++a)
+            for (int f = 0; f < F; ++f) {
+                const double w = std::pow(10000.0, -(double)f / (double)F);
+                row[a * 2 * F + f] = (float)std::sin(coord[a] * w);
+                row[a * 2 * F + F + f] = (float)std::cos(coord[a] * w);
+            }
+    }
+    return pos;
+}
+
+}  // namespace
+
+struct f3dc_handle {
+    f3dc_config cfg;
+    int N = 0, W = 0, Wm = 0, H = 0, dh = 0, L = 0, Nc = 0, Dc = 0, G = 0, T = 0;
+    int max_rows = 0, max_tiles = 0, num_sms = 0, device = 0;
+    size_t ckv_rows = 0;  // rows per layer of the condition K/V cache
+    std::string err;
+    Layout lay;
+
+    bf16 *wblob = nullptr, *mod_w = nullptr, *mod_b = nullptr;
+    int mod_rows = 0;
+    float *pos = nullptr;
+
+    float *x = nullptr, *v_active = nullptr, *freq = nullptr, *h1 = nullptr, *temb = nullptr, *mod = nullptr;
+    bf16 *h = nullptr, *qkv = nullptr, *att = nullptr, *qc = nullptr, *u = nullptr, *ckv = nullptr;
+    uint16_t *ring = nullptr;
+    Plan *plan = nullptr;
+    int32_t *tile_sample = nullptr, *active_idx = nullptr, *row_of_token = nullptr, *n_active = nullptr;
+    uint8_t *mask = nullptr;
+    int32_t *quota_dev = nullptr;
+    int64_t *dyn = nullptr;
+    uint32_t *dev_err = nullptr;
+    cudaStream_t last_stream = nullptr;
+    int cond_B = 0;
+    // pinned per-step quota slots, two generations so one sampler call can
+    // be enqueued while the previous one still copies from its slots
+    int32_t *h_quota = nullptr;
+    cudaEvent_t quota_done[2] = {nullptr, nullptr};
+    unsigned calls = 0;
+
+    CUtensorMap tm_h, tm_att, tm_u, tm_cond, tm_q_self, tm_q_cross;
+    std::vector<CUtensorMap> tm_qkv_w, tm_o_w, tm_cq_w, tm_co_w, tm_fc1_w, tm_fc2_w, tm_ckv_w, tm_kv_cross;
+    int bn_qkv = 128, bn_w = 128, bn_fc1 = 128, bn_ckv = 128;
+
+    const bf16 *wt(size_t off) const { return wblob + off; }
+};
+
+namespace {
+
+f3dc_status fail(f3dc_handle *h, f3dc_status st, const std::string &msg)
+{
+    if (h) h->err = msg;
+    g_last_error = msg;
+    return st;
+}
+
+#define CK(expr)                                                                                   \
+    do {                                                                                           \
+        cudaError_t e_ = (expr);                                                                   \
+        if (e_ != cudaSuccess)                                                                     \
+            return fail(h, F3DC_ERR_CUDA, std::string(#expr) + ": " + cudaGetErrorString(e_));     \
+    } while (0)
+
+template <typename T>
+cudaError_t dalloc(T **p, size_t count)
+{
+    return cudaMalloc(reinterpret_cast<void **>(p), count * sizeof(T) + 256);
+}
+
+int pick_bn(int N)
+{
+    if (N % 256 == 0 && N >= 2048) return 256;
+    if (N % 128 == 0) return 128;
+    return 64;
+}
+
+cudaError_t run_gemm(f3dc_handle *h, const CUtensorMap &ta, const CUtensorMap &tb, int N, int K, int bn, int epi,
+                     void *out, int ldo, const bf16 *bias, const float *gate, const bf16 *qn, const bf16 *kn,
+                     cudaStream_t s)
+{
+    GemmParams p;
+    memset(&p, 0, sizeof(p));
+    p.M = h->max_rows;
+    p.N = N;
+    p.K = K;
+    p.m_tiles_dev = &h->plan->n_tiles;
+    p.out = out;
+    p.ldo = ldo;
+    p.bias = bias;
+    p.gate = gate;
+    p.qn_g = qn;
+    p.kn_g = kn;
+    p.width = h->W;
+    p.dh = h->dh;
+    p.err = h->dev_err;
+    int tiles = h->max_tiles * (N / bn);
+    int grid = tiles < h->num_sms ? tiles : h->num_sms;
+    return launch_gemm(&ta, &tb, p, epi, bn, grid, s);
+}
+
+cudaError_t run_attention(f3dc_handle *h, int mode, const CUtensorMap &tq, const CUtensorMap &tkv, int q_col0,
+                          int k_col0, int v_col0, cudaStream_t s)
+{
+    AttnParams p;
+    memset(&p, 0, sizeof(p));
+    p.heads = h->H;
+    p.dh = h->dh;
+    p.q_col0 = q_col0;
+    p.k_col0 = k_col0;
+    p.v_col0 = v_col0;
+    p.mode = mode;
+    p.n_tiles_dev = &h->plan->n_tiles;
+    p.tile_sample = h->tile_sample;
+    p.plan = h->plan;
+    p.nk_fixed = h->Nc;
+    p.out = h->att;
+    p.ldo = h->W;
+    p.scale_log2 = (float)(1.4426950408889634 / std::sqrt((double)h->dh));
+    p.err = h->dev_err;
+    int items = h->max_tiles * h->H;
+    int grid = items < h->num_sms ? items : h->num_sms;
+    return launch_attention(&tq, &tkv, &tkv, p, grid, s);
+}
+
+// The flow transformer on the packed active rows described by h->plan,
+// h->tile_sample and h->active_idx (Sec. 4.2; Supp. Sec. F).
+f3dc_status run_dit(f3dc_handle *h, float t, const float *S, cudaStream_t s)
+{
+    const int W = h->W, L = h->L;
+    const Layout &ly = h->lay;
+    // timestep embedding and every block's modulation (adaLN)
+    CK(launch_time_freq(t, h->freq, s));
+    CK(launch_gemv(h->freq, 256, h->wt(ly.t_w1), h->wt(ly.t_b1), h->h1, W, 0, 1, h->num_sms, s));
+    CK(launch_gemv(h->h1, W, h->wt(ly.t_w2), h->wt(ly.t_b2), h->temb, W, 0, 0, h->num_sms, s));
+    CK(launch_gemv(h->temb, W, h->mod_w, h->mod_b, h->mod, h->mod_rows, 1, 0, h->num_sms, s));
+    // gather + embed the active tokens
+    CK(launch_gather_embed(S, h->N, W, h->active_idx, h->plan, h->tile_sample, h->wt(ly.in_w), h->wt(ly.in_b),
+                           h->pos, h->x, h->max_rows, h->num_sms, h->dev_err, s));
+    for (int l = 0; l < L; ++l) {
+        const BlockOffsets &b = ly.blk[l];
+        const float *m = h->mod + (size_t)l * 6 * W;
+        // self-attention among the active tokens
+        CK(launch_layernorm(h->x, W, h->plan, 0, m, m + W, nullptr, nullptr, h->h, h->max_rows, h->num_sms, s));
+        CK(run_gemm(h, h->tm_h, h->tm_qkv_w[l], 3 * W, W, h->bn_qkv, kEpiQKNorm, h->qkv, 3 * W, h->wt(b.qkv_b),
+                    nullptr, h->wt(b.qn_g), h->wt(b.kn_g), s));
+        CK(run_attention(h, 0, h->tm_q_self, h->tm_q_self, 0, W, 2 * W, s));
+        CK(run_gemm(h, h->tm_att, h->tm_o_w[l], W, W, h->bn_w, kEpiResid, h->x, W, h->wt(b.o_b), m + 2 * W,
+                    nullptr, nullptr, s));
+        // cross-attention to the condition
+        CK(launch_layernorm(h->x, W, h->plan, 1, nullptr, nullptr, h->wt(b.ln2_g), h->wt(b.ln2_b), h->h,
+                            h->max_rows, h->num_sms, s));
+        CK(run_gemm(h, h->tm_h, h->tm_cq_w[l], W, W, h->bn_w, kEpiBias, h->qc, W, h->wt(b.cq_b), nullptr,
+                    nullptr, nullptr, s));
+        CK(run_attention(h, 1, h->tm_q_cross, h->tm_kv_cross[l], 0, 0, W, s));
+        CK(run_gemm(h, h->tm_att, h->tm_co_w[l], W, W, h->bn_w, kEpiResid, h->x, W, h->wt(b.co_b), nullptr,
+                    nullptr, nullptr, s));
+        // MLP
+        CK(launch_layernorm(h->x, W, h->plan, 0, m + 3 * W, m + 4 * W, nullptr, nullptr, h->h, h->max_rows,
+                            h->num_sms, s));
+        CK(run_gemm(h, h->tm_h, h->tm_fc1_w[l], h->Wm, W, h->bn_fc1, kEpiGelu, h->u, h->Wm, h->wt(b.fc1_b),
+                    nullptr, nullptr, nullptr, s));
+        CK(run_gemm(h, h->tm_u, h->tm_fc2_w[l], W, h->Wm, h->bn_w, kEpiResid, h->x, W, h->wt(b.fc2_b), m + 5 * W,
+                    nullptr, nullptr, s));
+    }
+    const float *fm = h->mod + (size_t)L * 6 * W;
+    CK(launch_final_layer(h->x, W, h->plan, fm, fm + W, h->wt(ly.out_w), h->wt(ly.out_b), h->v_active,
+                          h->max_rows, h->num_sms, s));
+    return F3DC_OK;
+}
+
+bool build_maps(f3dc_handle *h)
+{
+    const int W = h->W, Wm = h->Wm, dh = h->dh;
+    const uint64_t R = (uint64_t)h->max_rows;
+    bool ok = make_tmap_bf16(&h->tm_h, h->h, R, W, W, 128, 64) && make_tmap_bf16(&h->tm_att, h->att, R, W, W, 128, 64) &&
+              make_tmap_bf16(&h->tm_u, h->u, R, Wm, Wm, 128, 64) &&
+              make_tmap_bf16(&h->tm_q_self, h->qkv, R, 3 * W, 3 * W, 128, dh) &&
+              make_tmap_bf16(&h->tm_q_cross, h->qc, R, W, W, 128, dh);
+    if (!ok) return false;
+    const int L = h->L;
+    h->tm_qkv_w.resize(L);
+    h->tm_o_w.resize(L);
+    h->tm_cq_w.resize(L);
+    h->tm_co_w.resize(L);
+    h->tm_fc1_w.resize(L);
+    h->tm_fc2_w.resize(L);
+    h->tm_ckv_w.resize(L);
+    h->tm_kv_cross.resize(L);
+    for (int l = 0; l < L; ++l) {
+        const BlockOffsets &b = h->lay.blk[l];
+        ok = ok && make_tmap_bf16(&h->tm_qkv_w[l], h->wt(b.qkv_w), 3 * W, W, W, h->bn_qkv, 64);
+        ok = ok && make_tmap_bf16(&h->tm_o_w[l], h->wt(b.o_w), W, W, W, h->bn_w, 64);
+        ok = ok && make_tmap_bf16(&h->tm_cq_w[l], h->wt(b.cq_w), W, W, W, h->bn_w, 64);
+        ok = ok && make_tmap_bf16(&h->tm_co_w[l], h->wt(b.co_w), W, W, W, h->bn_w, 64);
+        ok = ok && make_tmap_bf16(&h->tm_fc1_w[l], h->wt(b.fc1_w), Wm, W, W, h->bn_fc1, 64);
+        ok = ok && make_tmap_bf16(&h->tm_fc2_w[l], h->wt(b.fc2_w), W, Wm, Wm, h->bn_w, 64);
+        ok = ok && make_tmap_bf16(&h->tm_ckv_w[l], h->wt(b.ckv_w), 2 * W, h->Dc, h->Dc, h->bn_ckv, 64);
+        ok = ok && make_tmap_bf16(&h->tm_kv_cross[l], h->ckv + (size_t)l * h->ckv_rows * 2 * W, h->ckv_rows, 2 * W,
+                                  2 * W, 128, dh);
+    }
+    return ok;
+}
+
+void free_handle(f3dc_handle *h)
+{
+    void *ptrs[] = {h->wblob, h->mod_w, h->mod_b, h->pos, h->x, h->v_active, h->freq, h->h1, h->temb, h->mod,
+                    h->h, h->qkv, h->att, h->qc, h->u, h->ckv, h->ring, h->plan, h->tile_sample, h->active_idx,
+                    h->row_of_token, h->n_active, h->mask, h->quota_dev, h->dyn, h->dev_err};
+    for (void *p : ptrs)
+        if (p) cudaFree(p);
+    if (h->h_quota) cudaFreeHost(h->h_quota);
+    for (cudaEvent_t ev : h->quota_done)
+        if (ev) cudaEventDestroy(ev);
+    delete h;
+}
+
+}  // namespace
+
+// ============================================================================
+// C-ABI
+// ============================================================================
+extern "C" {
+
+f3dc_status f3dc_config_default(f3dc_config *cfg)
+{
+    if (!cfg) return fail(nullptr, F3DC_ERR_INVALID_ARG, "null config");
+    memset(cfg, 0, sizeof(*cfg));
+    cfg->grid = 16;
+    cfg->channels = 8;
+    cfg->width = 1024;
+    cfg->blocks = 24;
+    cfg->heads = 16;
+    cfg->mlp_ratio = 4;
+    cfg->cond_tokens = 1374;
+    cfg->cond_dim = 1024;
+    cfg->steps = 25;
+    cfg->max_batch = 1;
+    cfg->gamma_up = 64;
+    cfg->tau = 3;
+    cfg->f_corr = 3;
+    cfg->refresh_mode = F3DC_REFRESH_PERIOD;
+    cfg->eta = 3.0;
+    cfg->rho_a = 0.2;
+    cfg->mu = -0.07;
+    cfg->omega = 0.7;
+    cfg->xi = 0.7;
+    cfg->rho_cfg_off = 0.75;
+    return F3DC_OK;
+}
+
+size_t f3dc_weights_elems(const f3dc_config *cfg)
+{
+    std::string why;
+    if (!config_valid(cfg, why)) return 0;
+    return weight_layout(*cfg).total;
+}
+
+f3dc_status f3dc_time_schedule(const f3dc_config *cfg, float *t_out)
+{
+    std::string why;
+    if (!config_valid(cfg, why)) return fail(nullptr, F3DC_ERR_INVALID_ARG, why);
+    if (!t_out) return fail(nullptr, F3DC_ERR_INVALID_ARG, "null t_out");
+    time_schedule(*cfg, t_out);
+    return F3DC_OK;
+}
+
+f3dc_status f3dc_pcsc_quota(const f3dc_config *cfg, double sigma, int32_t k, int32_t *consec_inout,
+                            int32_t *quota_out, int32_t *phase_out)
+{
+    std::string why;
+    if (!config_valid(cfg, why)) return fail(nullptr, F3DC_ERR_INVALID_ARG, why);
+    if (!quota_out) return fail(nullptr, F3DC_ERR_INVALID_ARG, "null quota_out");
+    if (k < 1 || k > cfg->steps) return fail(nullptr, F3DC_ERR_INVALID_ARG, "step k outside [1, T]");
+    if (std::isnan(sigma) || sigma < 0.0) return fail(nullptr, F3DC_ERR_NONFINITE, "sigma must be a non-negative number");
+    int phase = 0;
+    int q = phase_quota(*cfg, sigma, k, &phase);
+    if (consec_inout) q = tau_gate(*cfg, q, consec_inout);
+    *quota_out = q;
+    if (phase_out) *phase_out = phase;
+    return F3DC_OK;
+}
+
+f3dc_status f3dc_create(const f3dc_config *cfg, const f3dc_weights *w, void *stream, f3dc_handle **out)
+{
+    f3dc_handle *h = nullptr;
+    std::string why;
+    if (!out) return fail(nullptr, F3DC_ERR_INVALID_ARG, "null out");
+    *out = nullptr;
+    if (!config_valid(cfg, why)) return fail(nullptr, F3DC_ERR_INVALID_ARG, why);
+    if (!w || w->layout_version != 1 || !w->blob) return fail(nullptr, F3DC_ERR_INVALID_ARG, "weights: need layout_version 1 and a blob");
+    const Layout lay = weight_layout(*cfg);
+    if (w->blob_elems != lay.total)
+        return fail(nullptr, F3DC_ERR_INVALID_ARG,
+                    "weights: blob_elems " + std::to_string(w->blob_elems) + " != " + std::to_string(lay.total));
+    cudaStream_t s = (cudaStream_t)stream;
+
+    h = new f3dc_handle();
+    h->cfg = *cfg;
+    h->lay = lay;
+    h->N = cfg->grid * cfg->grid * cfg->grid;
+    h->W = cfg->width;
+    h->Wm = cfg->mlp_ratio * cfg->width;
+    h->H = cfg->heads;
+    h->dh = cfg->width / cfg->heads;
+    h->L = cfg->blocks;
+    h->Nc = cfg->cond_tokens;
+    h->Dc = cfg->cond_dim;
+    h->G = cfg->gamma_up;
+    h->T = cfg->steps;
+    const int B = cfg->max_batch;
+    h->max_tiles = B * ((h->N + kTileRows - 1) / kTileRows);
+    h->max_rows = h->max_tiles * kTileRows;
+    h->ckv_rows = ((size_t)B * h->Nc + 2 * kTileRows - 1) / kTileRows * kTileRows;
+    h->bn_qkv = pick_bn(3 * h->W);
+    h->bn_w = pick_bn(h->W);
+    h->bn_fc1 = pick_bn(h->Wm);
+    h->bn_ckv = pick_bn(2 * h->W);
+    h->mod_rows = h->L * 6 * h->W + 2 * h->W;
+
+    cudaError_t e;
+#define CKC(expr)                                                                                  \
+    do {                                                                                           \
+        e = (expr);                                                                                \
+        if (e != cudaSuccess) {                                                                    \
+            std::string m_ = std::string(#expr) + ": " + cudaGetErrorString(e);                  \
+            free_handle(h);                                                                        \
+            return fail(nullptr, e == cudaErrorMemoryAllocation ? F3DC_ERR_OOM : F3DC_ERR_CUDA, m_); \
+        }                                                                                          \
+    } while (0)
+    CKC(cudaGetDevice(&h->device));
+    CKC(cudaDeviceGetAttribute(&h->num_sms, cudaDevAttrMultiProcessorCount, h->device));
+    int cc_major = 0, cc_minor = 0;
+    CKC(cudaDeviceGetAttribute(&cc_major, cudaDevAttrComputeCapabilityMajor, h->device));
+    CKC(cudaDeviceGetAttribute(&cc_minor, cudaDevAttrComputeCapabilityMinor, h->device));
+    if (cc_major != 10 || cc_minor != 3) {
+        free_handle(h);
+        return fail(nullptr, F3DC_ERR_UNSUPPORTED, "libf3dc is built for sm_103a (GB300) only");
+    }
+
+    const size_t R = h->max_rows, W = h->W, N = h->N;
+    CKC(dalloc(&h->wblob, lay.total));
+    CKC(cudaMemcpyAsync(h->wblob, w->blob, lay.total * sizeof(bf16), cudaMemcpyDeviceToDevice, s));
+    // modulation weights of every block and of the final layer, repacked into
+    // one [L*6W + 2W, W] matrix for a single streaming GEMV per step
+    CKC(dalloc(&h->mod_w, (size_t)h->mod_rows * W));
+    CKC(dalloc(&h->mod_b, (size_t)h->mod_rows));
+    const bf16 *src = reinterpret_cast<const bf16 *>(w->blob);
+    for (int l = 0; l < h->L; ++l) {
+        CKC(cudaMemcpyAsync(h->mod_w + (size_t)l * 6 * W * W, src + lay.blk[l].mod_w, 6 * W * W * sizeof(bf16),
+                            cudaMemcpyDeviceToDevice, s));
+        CKC(cudaMemcpyAsync(h->mod_b + (size_t)l * 6 * W, src + lay.blk[l].mod_b, 6 * W * sizeof(bf16),
+                            cudaMemcpyDeviceToDevice, s));
+    }
+    CKC(cudaMemcpyAsync(h->mod_w + (size_t)h->L * 6 * W * W, src + lay.fmod_w, 2 * W * W * sizeof(bf16),
+                        cudaMemcpyDeviceToDevice, s));
+    CKC(cudaMemcpyAsync(h->mod_b + (size_t)h->L * 6 * W, src + lay.fmod_b, 2 * W * sizeof(bf16),
+                        cudaMemcpyDeviceToDevice, s));
+    {
+        std::vector<float> pos = position_table(cfg->grid, h->W);
+        CKC(dalloc(&h->pos, pos.size()));
+        CKC(cudaMemcpyAsync(h->pos, pos.data(), pos.size() * sizeof(float), cudaMemcpyHostToDevice, s));
+        CKC(cudaStreamSynchronize(s));
+    }
+    CKC(dalloc(&h->x, R * W));
+    CKC(dalloc(&h->h, R * W));
+    CKC(dalloc(&h->qkv, R * 3 * W));
+    CKC(dalloc(&h->att, R * W));
+    CKC(dalloc(&h->qc, R * W));
+    CKC(dalloc(&h->u, R * h->Wm));
+    CKC(dalloc(&h->v_active, R * kChannels));
+    CKC(dalloc(&h->ckv, (size_t)h->L * h->ckv_rows * 2 * W));
+    CKC(cudaMemsetAsync(h->ckv, 0, (size_t)h->L * h->ckv_rows * 2 * W * sizeof(bf16), s));
+    CKC(cudaMemsetAsync(h->x, 0, R * W * sizeof(float), s));
+    CKC(cudaMemsetAsync(h->qkv, 0, R * 3 * W * sizeof(bf16), s));
+    CKC(cudaMemsetAsync(h->qc, 0, R * W * sizeof(bf16), s));
+    CKC(dalloc(&h->freq, 256));
+    CKC(dalloc(&h->h1, W));
+    CKC(dalloc(&h->temb, W));
+    CKC(dalloc(&h->mod, (size_t)h->mod_rows));
+    CKC(dalloc(&h->ring, (size_t)3 * B * N * kChannels));
+    CKC(dalloc(&h->plan, 1));
+    CKC(cudaMemsetAsync(h->plan, 0, sizeof(Plan), s));
+    CKC(dalloc(&h->tile_sample, (size_t)h->max_tiles));
+    CKC(dalloc(&h->active_idx, (size_t)B * N));
+    CKC(dalloc(&h->row_of_token, (size_t)B * N));
+    CKC(dalloc(&h->n_active, (size_t)B));
+    CKC(dalloc(&h->mask, (size_t)B * N));
+    CKC(dalloc(&h->quota_dev, (size_t)(h->T + 1) * B));
+    CKC(dalloc(&h->dyn, (size_t)B));
+    CKC(dalloc(&h->dev_err, 1));
+    CKC(cudaMemsetAsync(h->dev_err, 0, sizeof(uint32_t), s));
+    CKC(cudaMallocHost(reinterpret_cast<void **>(&h->h_quota), (size_t)2 * (h->T + 1) * B * sizeof(int32_t)));
+    CKC(cudaEventCreateWithFlags(&h->quota_done[0], cudaEventDisableTiming));
+    CKC(cudaEventCreateWithFlags(&h->quota_done[1], cudaEventDisableTiming));
+#undef CKC
+    if (!build_maps(h)) {
+        free_handle(h);
+        return fail(nullptr, F3DC_ERR_CUDA, "cuTensorMapEncodeTiled failed");
+    }
+    e = cudaStreamSynchronize(s);
+    if (e != cudaSuccess) {
+        std::string m = std::string("create: ") + cudaGetErrorString(e);
+        free_handle(h);
+        return fail(nullptr, F3DC_ERR_CUDA, m);
+    }
+    h->last_stream = s;
+    *out = h;
+    return F3DC_OK;
+}
+
+f3dc_status f3dc_destroy(f3dc_handle *h)
+{
+    if (!h) return F3DC_OK;
+    cudaDeviceSynchronize();
+    free_handle(h);
+    return F3DC_OK;
+}
+
+const char *f3dc_last_error(const f3dc_handle *h)
+{
+    if (h) return h->err.c_str();
+    return g_last_error.c_str();
+}
+
+f3dc_status f3dc_device_status(f3dc_handle *h, uint32_t *status_out)
+{
+    if (!h || !status_out) return fail(h, F3DC_ERR_INVALID_ARG, "null argument");
+    CK(cudaStreamSynchronize(h->last_stream));
+    uint32_t v = 0;
+    CK(cudaMemcpy(&v, h->dev_err, sizeof(v), cudaMemcpyDeviceToHost));
+    CK(cudaMemset(h->dev_err, 0, sizeof(uint32_t)));
+    *status_out = v;
+    return F3DC_OK;
+}
+
+f3dc_status f3dc_ssc_select(f3dc_handle *h, const void *v_prev1, const void *v_prev2, int32_t B,
+                            const int32_t *quota_dev, int32_t *active_idx_out, int32_t *n_active_out,
+                            uint8_t *cached_mask_out, void *stream)
+{
+    if (!h) return fail(nullptr, F3DC_ERR_INVALID_ARG, "null handle");
+    if (!v_prev1 || !v_prev2 || !quota_dev || !active_idx_out) return fail(h, F3DC_ERR_INVALID_ARG, "null pointer");
+    if (B < 1 || B > h->cfg.max_batch) return fail(h, F3DC_ERR_INVALID_ARG, "B outside [1, max_batch]");
+    cudaStream_t s = (cudaStream_t)stream;
+    h->last_stream = s;
+    SelectArgs a;
+    memset(&a, 0, sizeof(a));
+    a.v1 = reinterpret_cast<const uint16_t *>(v_prev1);
+    a.v2 = reinterpret_cast<const uint16_t *>(v_prev2);
+    a.quota = quota_dev;
+    a.B = B;
+    a.N = h->N;
+    a.wa = (float)h->cfg.omega;
+    a.wv = 1.0f - a.wa;
+    a.active_idx = active_idx_out;
+    a.n_active = n_active_out;
+    a.mask = cached_mask_out;
+    a.err = h->dev_err;
+    CK(launch_ssc_select(a, s));
+    return F3DC_OK;
+}
+
+f3dc_status f3dc_set_cond(f3dc_handle *h, const void *cond, int32_t B, void *stream)
+{
+    if (!h) return fail(nullptr, F3DC_ERR_INVALID_ARG, "null handle");
+    if (!cond) return fail(h, F3DC_ERR_INVALID_ARG, "null cond");
+    if (B < 1 || B > h->cfg.max_batch) return fail(h, F3DC_ERR_INVALID_ARG, "B outside [1, max_batch]");
+    if (((uintptr_t)cond & 15) != 0) return fail(h, F3DC_ERR_INVALID_ARG, "cond must be 16-byte aligned");
+    cudaStream_t s = (cudaStream_t)stream;
+    h->last_stream = s;
+    const int rows = B * h->Nc;
+    if (!make_tmap_bf16(&h->tm_cond, cond, rows, h->Dc, h->Dc, 128, 64))
+        return fail(h, F3DC_ERR_CUDA, "cuTensorMapEncodeTiled failed for cond");
+    for (int l = 0; l < h->L; ++l) {
+        GemmParams p;
+        memset(&p, 0, sizeof(p));
+        p.M = rows;
+        p.N = 2 * h->W;
+        p.K = h->Dc;
+        p.m_tiles = (rows + kTileRows - 1) / kTileRows;
+        p.out = h->ckv + (size_t)l * h->ckv_rows * 2 * h->W;
+        p.ldo = 2 * h->W;
+        p.bias = h->wt(h->lay.blk[l].ckv_b);
+        p.err = h->dev_err;
+        const int tiles = p.m_tiles * (p.N / h->bn_ckv);
+        CK(launch_gemm(&h->tm_cond, &h->tm_ckv_w[l], p, kEpiBias, h->bn_ckv, tiles < h->num_sms ? tiles : h->num_sms,
+                       s));
+    }
+    h->cond_B = B;
+    return F3DC_OK;
+}
+
+f3dc_status f3dc_step(f3dc_handle *h, int32_t k, int32_t B, float *S_inout, void *v_ring,
+                      const int32_t *quota_dev, int64_t *dyn_voxels_dev, void *stream)
+{
+    if (!h) return fail(nullptr, F3DC_ERR_INVALID_ARG, "null handle");
+    if (!S_inout || !v_ring || !quota_dev) return fail(h, F3DC_ERR_INVALID_ARG, "null pointer");
+    if (k < 1 || k > h->T) return fail(h, F3DC_ERR_INVALID_ARG, "step k outside [1, T]");
+    if (B < 1 || B > h->cfg.max_batch) return fail(h, F3DC_ERR_INVALID_ARG, "B outside [1, max_batch]");
+    if (B > h->cond_B) return fail(h, F3DC_ERR_INVALID_ARG, "f3dc_set_cond was not called for this batch");
+    cudaStream_t s = (cudaStream_t)stream;
+    h->last_stream = s;
+    const size_t slot = (size_t)B * h->N * kChannels;
+    uint16_t *ring = reinterpret_cast<uint16_t *>(v_ring);
+    uint16_t *v_new = ring + (size_t)(k % 3) * slot;
+    const uint16_t *v1 = ring + (size_t)((k - 1) % 3) * slot;
+    const uint16_t *v2 = ring + (size_t)(((k - 2) % 3 + 3) % 3) * slot;
+
+    // SSC selection + row plan (Algorithm 1 step 2, first line)
+    SelectArgs a;
+    memset(&a, 0, sizeof(a));
+    a.v1 = v1;
+    a.v2 = v2;
+    a.quota = quota_dev;
+    a.B = B;
+    a.N = h->N;
+    a.wa = (float)h->cfg.omega;
+    a.wv = 1.0f - a.wa;
+    a.active_idx = h->active_idx;
+    a.n_active = h->n_active;
+    a.mask = h->mask;
+    a.row_of_token = h->row_of_token;
+    a.plan = h->plan;
+    a.tile_sample = h->tile_sample;
+    a.err = h->dev_err;
+    CK(launch_ssc_select(a, s));
+
+    // FlowTransformer on the active tokens at t_k
+    std::vector<float> t(h->T + 1);
+    time_schedule(h->cfg, t.data());
+    f3dc_status st = run_dit(h, t[k - 1], S_inout, s);
+    if (st != F3DC_OK) return st;
+
+    // merge + Euler + history (Algorithm 1 step 3)
+    MergeArgs m;
+    memset(&m, 0, sizeof(m));
+    m.S = S_inout;
+    m.v_active = h->v_active;
+    m.row_of_token = h->row_of_token;
+    m.v_prev1 = v1;
+    m.v_out = v_new;
+    m.B = B;
+    m.N = h->N;
+    m.dt = t[k - 1] - t[k];
+    m.dec_w = reinterpret_cast<const uint16_t *>(h->wt(h->lay.dec_w));
+    m.G = h->G;
+    m.dyn = dyn_voxels_dev;
+    m.max_rows = h->max_rows;
+    m.err = h->dev_err;
+    CK(launch_merge_euler(m, s));
+    return F3DC_OK;
+}
+
+f3dc_status f3dc_sample(f3dc_handle *h, float *S_inout, const void *cond, int32_t B, const double *sigma_override,
+                        const int32_t *quota_schedule, int32_t *quota_log, double *sigma_out, void *stream)
+{
+    if (!h) return fail(nullptr, F3DC_ERR_INVALID_ARG, "null handle");
+    if (!S_inout || !cond) return fail(h, F3DC_ERR_INVALID_ARG, "null pointer");
+    if (B < 1 || B > h->cfg.max_batch) return fail(h, F3DC_ERR_INVALID_ARG, "B outside [1, max_batch]");
+    if (sigma_override)
+        for (int b = 0; b < B; ++b)
+            if (std::isnan(sigma_override[b]) || sigma_override[b] < 0.0)
+                return fail(h, F3DC_ERR_NONFINITE, "sigma_override must be non-negative numbers");
+    cudaStream_t s = (cudaStream_t)stream;
+    const int T = h->T, N = h->N;
+    const int ka = ceil_steps(T, h->cfg.rho_a);
+    f3dc_status st = f3dc_set_cond(h, cond, B, stream);
+    if (st != F3DC_OK) return st;
+    CK(cudaMemsetAsync(h->ring, 0, (size_t)3 * B * N * kChannels * sizeof(uint16_t), s));
+    CK(cudaMemsetAsync(h->dyn, 0, (size_t)B * sizeof(int64_t), s));
+
+    const unsigned gen = h->calls++ & 1u;
+    CK(cudaEventSynchronize(h->quota_done[gen]));  // slots of the call before last are free
+    int32_t *hq = h->h_quota + (size_t)gen * (T + 1) * B;
+    std::vector<double> sigma(B, 0.0), measured(B, 0.0);
+    if (sigma_override)
+        for (int b = 0; b < B; ++b) sigma[b] = sigma_override[b];
+    std::vector<int32_t> consec(B, 0);
+    const bool need_measure = !quota_schedule && !sigma_override;
+    bool have_measured = false;
+    for (int k = 1; k <= T; ++k) {
+        for (int b = 0; b < B; ++b) {
+            int phase = 0;
+            int c = quota_schedule ? quota_schedule[(size_t)(k - 1) * B + b] : phase_quota(h->cfg, sigma[b], k, &phase);
+            if (c < 0) c = 0;
+            if (c > N) c = N;
+            hq[(size_t)k * B + b] = tau_gate(h->cfg, c, &consec[b]);
+            if (quota_log) quota_log[(size_t)(k - 1) * B + b] = hq[(size_t)k * B + b];
+        }
+        int32_t *qd = h->quota_dev + (size_t)k * B;
+        CK(cudaMemcpyAsync(qd, hq + (size_t)k * B, (size_t)B * sizeof(int32_t), cudaMemcpyHostToDevice, s));
+        st = f3dc_step(h, k, B, S_inout, h->ring, qd, k == ka ? h->dyn : nullptr, stream);
+        if (st != F3DC_OK) return st;
+        if (k == ka && need_measure) {
+            std::vector<int64_t> d(B);
+            CK(cudaMemcpyAsync(d.data(), h->dyn, (size_t)B * sizeof(int64_t), cudaMemcpyDeviceToHost, s));
+            CK(cudaStreamSynchronize(s));
+            for (int b = 0; b < B; ++b) sigma[b] = measured[b] = (double)d[b];
+            have_measured = true;
+        }
+    }
+    if (sigma_out) {
+        if (!have_measured && ka >= 1 && ka <= T) {
+            std::vector<int64_t> d(B);
+            CK(cudaMemcpyAsync(d.data(), h->dyn, (size_t)B * sizeof(int64_t), cudaMemcpyDeviceToHost, s));
+            CK(cudaStreamSynchronize(s));
+            for (int b = 0; b < B; ++b) measured[b] = (double)d[b];
+        }
+        for (int b = 0; b < B; ++b) sigma_out[b] = measured[b];
+    }
+    CK(cudaEventRecord(h->quota_done[gen], s));
+    if (quota_log) CK(cudaStreamSynchronize(s));
+    return F3DC_OK;
+}
+
+f3dc_status f3dc_forward(f3dc_handle *h, float t, int32_t B, const float *S, const int32_t *active_idx,
+                         const int32_t *n_active, float *v_out, void *stream)
+{
+    if (!h) return fail(nullptr, F3DC_ERR_INVALID_ARG, "null handle");
+    if (!S || !active_idx || !n_active || !v_out) return fail(h, F3DC_ERR_INVALID_ARG, "null pointer");
+    if (B < 1 || B > h->cfg.max_batch) return fail(h, F3DC_ERR_INVALID_ARG, "B outside [1, max_batch]");
+    if (B > h->cond_B) return fail(h, F3DC_ERR_INVALID_ARG, "f3dc_set_cond was not called for this batch");
+    cudaStream_t s = (cudaStream_t)stream;
+    h->last_stream = s;
+    CK(cudaMemcpyAsync(h->active_idx, active_idx, (size_t)B * h->N * sizeof(int32_t), cudaMemcpyDeviceToDevice, s));
+    CK(launch_plan_from_counts(n_active, h->active_idx, B, h->N, h->plan, h->tile_sample, nullptr, h->dev_err, s));
+    f3dc_status st = run_dit(h, t, S, s);
+    if (st != F3DC_OK) return st;
+    CK(launch_scatter_rows(h->v_active, h->plan, B, h->N, v_out, s));
+    return F3DC_OK;
+}
+
+f3dc_status f3dc_gemm(const void *A, const void *B, const void *bias, const float *gate, void *out, int32_t M,
+                      int32_t N, int32_t K, int32_t epilogue, void *stream)
+{
+    f3dc_handle *h = nullptr;
+    if (!A || !B || !out) return fail(nullptr, F3DC_ERR_INVALID_ARG, "null pointer");
+    if (M < 1 || N < 64 || N % 64 != 0 || K < 64 || K % 64 != 0)
+        return fail(nullptr, F3DC_ERR_INVALID_ARG, "need M >= 1, N and K positive multiples of 64");
+    if (epilogue < F3DC_EPI_BIAS || epilogue > F3DC_EPI_RESID) return fail(nullptr, F3DC_ERR_INVALID_ARG, "bad epilogue");
+    if (((uintptr_t)out & 15) || (bias && ((uintptr_t)bias & 15)) || (gate && ((uintptr_t)gate & 15)))
+        return fail(nullptr, F3DC_ERR_INVALID_ARG, "pointers must be 16-byte aligned");
+    const int bn = N % 256 == 0 ? 256 : (N % 128 == 0 ? 128 : 64);
+    CUtensorMap ta, tb;
+    if (!make_tmap_bf16(&ta, A, M, K, K, 128, 64) || !make_tmap_bf16(&tb, B, N, K, K, bn, 64))
+        return fail(nullptr, F3DC_ERR_INVALID_ARG, "cuTensorMapEncodeTiled rejected A or B (alignment?)");
+    GemmParams p;
+    memset(&p, 0, sizeof(p));
+    p.M = M;
+    p.N = N;
+    p.K = K;
+    p.m_tiles = (M + kTileRows - 1) / kTileRows;
+    p.out = out;
+    p.ldo = N;
+    p.bias = reinterpret_cast<const bf16 *>(bias);
+    p.gate = gate;
+    int dev = 0, sms = 0;
+    CK(cudaGetDevice(&dev));
+    CK(cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev));
+    const int tiles = p.m_tiles * (N / bn);
+    const int epi = epilogue == F3DC_EPI_BIAS ? kEpiBias : (epilogue == F3DC_EPI_GELU ? kEpiGelu : kEpiResid);
+    CK(launch_gemm(&ta, &tb, p, epi, bn, tiles < sms ? tiles : sms, (cudaStream_t)stream));
+    return F3DC_OK;
+}
+
+f3dc_status f3dc_attention(const void *q, int32_t ldq, const void *k, const void *v, int32_t ldkv, void *out,
+                           int32_t nq, int32_t nk, int32_t heads, int32_t dh, void *stream)
+{
+    f3dc_handle *h = nullptr;
+    if (!q || !k || !v || !out) return fail(nullptr, F3DC_ERR_INVALID_ARG, "null pointer");
+    if (nq < 1 || nk < 1 || heads < 1 || (dh != 32 && dh != 64) || ldq % 8 || ldkv % 8 || ldq < heads * dh ||
+        ldkv < heads * dh)
+        return fail(nullptr, F3DC_ERR_INVALID_ARG, "bad attention shape");
+    CUtensorMap tq, tk, tv;
+    if (!make_tmap_bf16(&tq, q, nq, ldq, ldq, 128, dh) || !make_tmap_bf16(&tk, k, nk, ldkv, ldkv, 128, dh) ||
+        !make_tmap_bf16(&tv, v, nk, ldkv, ldkv, 128, dh))
+        return fail(nullptr, F3DC_ERR_INVALID_ARG, "cuTensorMapEncodeTiled rejected q / k / v (alignment?)");
+    AttnParams p;
+    memset(&p, 0, sizeof(p));
+    p.heads = heads;
+    p.dh = dh;
+    p.mode = 2;
+    p.n_tiles = (nq + 127) / 128;
+    p.nk_fixed = nk;
+    p.q_rows = nq;
+    p.out = reinterpret_cast<bf16 *>(out);
+    p.ldo = heads * dh;
+    p.scale_log2 = (float)(1.4426950408889634 / std::sqrt((double)dh));
+    int dev = 0, sms = 0;
+    CK(cudaGetDevice(&dev));
+    CK(cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev));
+    const int items = p.n_tiles * heads;
+    CK(launch_attention(&tq, &tk, &tv, p, items < sms ? items : sms, (cudaStream_t)stream));
+    return F3DC_OK;
+}
+
+}  // extern "C"

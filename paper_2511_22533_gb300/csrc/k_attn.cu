@@ -1,0 +1,396 @@
+// k_attn.cu -- K5 / K6: multi-head attention softmax(Q K^T / sqrt(dh)) V on
+// 5th-generation tensor cores, flash style (online softmax), for
+//   mode 0  self-attention of every sample among its ACTIVE tokens only
+//           (Sec. 4.2: attention runs on the compacted active subset)
+//   mode 1  cross-attention of the active tokens to the sample's condition
+//           tokens (Supp. Sec. F cross-attention)
+//   mode 2  one sequence (diagnostic entry point)
+//
+// Persistent kernel, one CTA per SM (192 threads), work item = (128-query
+// tile, head):
+//   warp 0     TMA producer: Q tile once per item, K / V tiles of 128 keys
+//              into a 3-deep ring
+//   warp 1     TMEM allocator + tcgen05.mma issuer:
+//                S_j = Q K_j^T   (M=128, N=128, K=dh)      -> TMEM S[j%2]
+//                O_j = P_j V_j   (M=128, N=dh,  K=128 keys) -> TMEM O[j%2]
+//              issued as S_j, then O_(j-1), so the tensor core computes the
+//              next scores and the previous P V while the softmax runs
+//   warps 2-5  softmax, one thread per query row (TMEM lane = row):
+//              running max / sum, P_j = exp2(S_j scale - m) written as bf16
+//              to 128B-swizzled shared memory (the K-major A operand of the
+//              P V MMA), O accumulated in registers with the lazy rescale
+//              O <- (O + O_(j-1)) * exp2(m_(j-1) - m_j)
+// V is the MN-major B operand of the P V MMA straight from its row-major
+// TMA tile.  Keys beyond a sample's count are masked to -inf before the
+// exponent; padding rows are finite by construction, so 0 * pad = 0.
+#include "common.cuh"
+#include "kernels.h"
+
+namespace f3dc {
+
+namespace {
+
+constexpr int kAttnThreads = 192;
+constexpr int kKVStages = 3;
+
+template <int DH>
+struct AttnCfg {
+    static constexpr int kRowBytes = DH * 2;            // 128 (DH 64) or 64 (DH 32)
+    static constexpr int kTileBytes = 128 * kRowBytes;  // Q, K or V tile
+    static constexpr uint32_t kAtom = 8 * kRowBytes;    // 8-row swizzle atom
+    static constexpr uint32_t kSwz = DH == 64 ? kSwizzle128 : kSwizzle64;
+    static constexpr int kPPanel = 128 * 128;           // 64 keys x 128 rows x 2 B
+    static constexpr int kPBytes = 2 * kPPanel;
+    static constexpr size_t kSmem = 1024 + kTileBytes * (1 + 2 * kKVStages) + 2 * kPBytes + 512;
+    static constexpr uint32_t kTmemCols = 512;          // S0 S1 | O0 O1
+};
+
+struct Item {
+    int q_row0, kv_row0, nk, h, store_end;
+};
+
+F3DC_DEV Item decode_item(const AttnParams &p, int w)
+{
+    Item it;
+    const int t = w / p.heads;
+    it.h = w - t * p.heads;
+    it.q_row0 = t * 128;
+    it.store_end = 0x7FFFFFFF;
+    if (p.mode == 0) {
+        const int b = p.tile_sample[t];
+        it.kv_row0 = p.plan->row_off[b];
+        it.nk = p.plan->n_active[b];
+    } else if (p.mode == 1) {
+        const int b = p.tile_sample[t];
+        it.kv_row0 = b * p.nk_fixed;
+        it.nk = p.nk_fixed;
+    } else {
+        it.kv_row0 = 0;
+        it.nk = p.nk_fixed;
+        it.store_end = p.q_rows;
+    }
+    return it;
+}
+
+F3DC_DEV bool wait_bounded(uint64_t *bar, uint32_t parity, uint64_t ns)
+{
+    const uint64_t t0 = globaltimer();
+    while (!mbar_try_wait(bar, parity))
+        if (globaltimer() - t0 > ns) return false;
+    return true;
+}
+
+template <int DH>
+__global__ void __launch_bounds__(kAttnThreads, 1)
+    k_attn(const __grid_constant__ CUtensorMap tmq, const __grid_constant__ CUtensorMap tmk,
+           const __grid_constant__ CUtensorMap tmv, const AttnParams p)
+{
+    using Cfg = AttnCfg<DH>;
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+    uint8_t *sQ = smem;
+    uint8_t *sK = sQ + Cfg::kTileBytes;
+    uint8_t *sV = sK + kKVStages * Cfg::kTileBytes;
+    uint8_t *sP = sV + kKVStages * Cfg::kTileBytes;
+    uint64_t *bars = reinterpret_cast<uint64_t *>(sP + 2 * Cfg::kPBytes);
+    uint64_t *q_full = bars, *q_empty = bars + 1;
+    uint64_t *kv_full = bars + 2, *kv_empty = kv_full + kKVStages;
+    uint64_t *s_full = kv_empty + kKVStages, *s_empty = s_full + 2;
+    uint64_t *p_full = s_empty + 2, *p_empty = p_full + 2;
+    uint64_t *o_full = p_empty + 2, *o_empty = o_full + 2;
+    uint64_t *drain = o_empty + 2;
+    uint32_t *tmem_holder = reinterpret_cast<uint32_t *>(drain + 1);
+    volatile int *abort_flag = reinterpret_cast<volatile int *>(tmem_holder + 1);
+
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int n_tiles = p.n_tiles_dev ? *p.n_tiles_dev : p.n_tiles;
+    const int total = n_tiles * p.heads;
+
+    if (threadIdx.x == 0) {
+        mbar_init(q_full, 1);
+        mbar_init(q_empty, 1);
+        for (int s = 0; s < kKVStages; ++s) {
+            mbar_init(&kv_full[s], 1);
+            mbar_init(&kv_empty[s], 1);
+        }
+        for (int s = 0; s < 2; ++s) {
+            mbar_init(&s_full[s], 1);
+            mbar_init(&s_empty[s], 128);
+            mbar_init(&p_full[s], 128);
+            mbar_init(&p_empty[s], 1);
+            mbar_init(&o_full[s], 1);
+            mbar_init(&o_empty[s], 128);
+        }
+        mbar_init(drain, 1);
+        *abort_flag = 0;
+        fence_mbar_init();
+    }
+    if (warp == 1) {
+        tmem_alloc(tmem_holder, Cfg::kTmemCols);
+        tmem_relinquish();
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = *tmem_holder;
+
+    if (warp == 0) {
+        // ------------------------------------------------ TMA producer
+        if (lane == 0) {
+            tma_prefetch(&tmq);
+            tma_prefetch(&tmk);
+            tma_prefetch(&tmv);
+            uint32_t kv_it = 0, item_it = 0;
+            bool ok = true;
+            for (int w = blockIdx.x; w < total && ok; w += gridDim.x, ++item_it) {
+                const Item it = decode_item(p, w);
+                if (!mbar_wait(q_empty, (item_it & 1) ^ 1, abort_flag, p.err)) break;
+                mbar_arrive_expect_tx(q_full, Cfg::kTileBytes);
+                tma_load_2d(sQ, &tmq, p.q_col0 + it.h * DH, it.q_row0, q_full);
+                const int nkt = (it.nk + 127) / 128;
+                for (int j = 0; j < nkt; ++j, ++kv_it) {
+                    const int s = kv_it % kKVStages;
+                    const uint32_t ph = (kv_it / kKVStages) & 1;
+                    if (!mbar_wait(&kv_empty[s], ph ^ 1, abort_flag, p.err)) {
+                        ok = false;
+                        break;
+                    }
+                    mbar_arrive_expect_tx(&kv_full[s], 2 * Cfg::kTileBytes);
+                    tma_load_2d(sK + s * Cfg::kTileBytes, &tmk, p.k_col0 + it.h * DH, it.kv_row0 + j * 128,
+                                &kv_full[s]);
+                    tma_load_2d(sV + s * Cfg::kTileBytes, &tmv, p.v_col0 + it.h * DH, it.kv_row0 + j * 128,
+                                &kv_full[s]);
+                }
+            }
+        }
+    } else if (warp == 1) {
+        // ------------------------------------------------ MMA issuer
+        if (lane == 0) {
+            constexpr uint32_t idesc_s = make_idesc_bf16(128, 128, 0, 0);
+            constexpr uint32_t idesc_o = make_idesc_bf16(128, DH, 0, 1);
+            const uint32_t q_addr = smem_u32(sQ);
+            uint32_t kv_it = 0, g = 0, item_it = 0;
+            bool ok = true;
+            auto issue_pv = [&](uint32_t gp, uint32_t kvp) -> bool {
+                const uint32_t pb = gp & 1, pph = (gp >> 1) & 1;
+                if (!mbar_wait(&p_full[pb], pph, abort_flag, p.err)) return false;
+                if (!mbar_wait(&o_empty[pb], pph ^ 1, abort_flag, p.err)) return false;
+                tc_fence_after();
+                const int s = kvp % kKVStages;
+                const uint32_t p_addr = smem_u32(sP + pb * Cfg::kPBytes);
+                const uint32_t v_addr = smem_u32(sV + s * Cfg::kTileBytes);
+#pragma unroll
+                for (int kk = 0; kk < 8; ++kk) {
+                    const uint64_t ad = make_sdesc(p_addr + (kk >> 2) * Cfg::kPPanel + (kk & 3) * 32, 16, 1024,
+                                                   kSwizzle128);
+                    const uint64_t bd = make_sdesc(v_addr + kk * 16 * Cfg::kRowBytes, Cfg::kAtom, Cfg::kAtom, Cfg::kSwz);
+                    mma_bf16(tmem + 256 + pb * DH, ad, bd, idesc_o, kk > 0);
+                }
+                mma_commit(&o_full[pb]);
+                mma_commit(&kv_empty[s]);
+                mma_commit(&p_empty[pb]);
+                return true;
+            };
+            for (int w = blockIdx.x; w < total && ok; w += gridDim.x, ++item_it) {
+                const Item it = decode_item(p, w);
+                if (!mbar_wait(q_full, item_it & 1, abort_flag, p.err)) break;
+                tc_fence_after();
+                const int nkt = (it.nk + 127) / 128;
+                for (int j = 0; j < nkt; ++j, ++kv_it, ++g) {
+                    const int s = kv_it % kKVStages;
+                    if (!mbar_wait(&kv_full[s], (kv_it / kKVStages) & 1, abort_flag, p.err)) {
+                        ok = false;
+                        break;
+                    }
+                    const uint32_t sb = g & 1;
+                    if (!mbar_wait(&s_empty[sb], ((g >> 1) & 1) ^ 1, abort_flag, p.err)) {
+                        ok = false;
+                        break;
+                    }
+                    tc_fence_after();
+                    const uint32_t k_addr = smem_u32(sK + s * Cfg::kTileBytes);
+#pragma unroll
+                    for (int kk = 0; kk < DH / 16; ++kk)
+                        mma_bf16(tmem + sb * 128, make_sdesc(q_addr + kk * 32, 16, Cfg::kAtom, Cfg::kSwz),
+                                 make_sdesc(k_addr + kk * 32, 16, Cfg::kAtom, Cfg::kSwz), idesc_s, kk > 0);
+                    mma_commit(&s_full[sb]);
+                    if (j == nkt - 1) mma_commit(q_empty);
+                    if (j >= 1 && !issue_pv(g - 1, kv_it - 1)) {
+                        ok = false;
+                        break;
+                    }
+                }
+                if (ok && !issue_pv(g - 1, kv_it - 1)) ok = false;
+            }
+        }
+    } else {
+        // ------------------------------------------------ softmax warps
+        const int q = warp & 3;
+        const int row = q * 32 + lane;
+        const uint32_t tl = (uint32_t)(q * 32) << 16;
+        uint32_t g = 0;
+        for (int w = blockIdx.x; w < total; w += gridDim.x) {
+            const Item it = decode_item(p, w);
+            const int nkt = (it.nk + 127) / 128;
+            float m_run = -INFINITY, l_run = 0.f;
+            float acc[DH];
+#pragma unroll
+            for (int d = 0; d < DH; ++d) acc[d] = 0.f;
+            bool ok = true;
+            for (int j = 0; j < nkt; ++j, ++g) {
+                const uint32_t sb = g & 1, sph = (g >> 1) & 1;
+                if (!mbar_wait(&s_full[sb], sph, abort_flag, p.err)) {
+                    ok = false;
+                    break;
+                }
+                tc_fence_after();
+                const int valid = min(128, it.nk - j * 128);
+                const uint32_t s_addr = tmem + tl + sb * 128;
+                // pass 1: row max of the scaled, masked scores
+                float mx = -INFINITY;
+#pragma unroll 1
+                for (int c0 = 0; c0 < 128; c0 += 32) {
+                    uint32_t r[32];
+                    tmem_ld32(s_addr + c0, r);
+                    tmem_wait_ld();
+#pragma unroll
+                    for (int c = 0; c < 32; ++c)
+                        if (c0 + c < valid) mx = fmaxf(mx, __uint_as_float(r[c]) * p.scale_log2);
+                }
+                const float m_new = fmaxf(m_run, mx);
+                const float alpha = exp2_fast(m_run - m_new);
+                // P[sb] may still be read by the P V MMA of tile g-2
+                if (!mbar_wait(&p_empty[sb], sph ^ 1, abort_flag, p.err)) {
+                    ok = false;
+                    break;
+                }
+                // pass 2: P = exp2(s - m_new) -> bf16, 128B-swizzled K-major rows
+                float sum = 0.f;
+                uint8_t *prow = sP + sb * Cfg::kPBytes + row * 128;
+#pragma unroll 1
+                for (int c0 = 0; c0 < 128; c0 += 32) {
+                    uint32_t r[32];
+                    tmem_ld32(s_addr + c0, r);
+                    tmem_wait_ld();
+                    float pv[32];
+#pragma unroll
+                    for (int c = 0; c < 32; ++c) {
+                        const float x = (c0 + c < valid) ? __uint_as_float(r[c]) * p.scale_log2 - m_new : -INFINITY;
+                        pv[c] = exp2_fast(x);
+                        sum += pv[c];
+                    }
+                    uint8_t *panel = prow + (c0 >> 6) * Cfg::kPPanel;
+#pragma unroll
+                    for (int ch = 0; ch < 4; ++ch) {
+                        const int chunk = ((c0 & 63) >> 3) + ch;  // 16-byte chunk within the 128-byte row
+                        uint4 u;
+                        u.x = pack_bf16x2(pv[ch * 8 + 0], pv[ch * 8 + 1]);
+                        u.y = pack_bf16x2(pv[ch * 8 + 2], pv[ch * 8 + 3]);
+                        u.z = pack_bf16x2(pv[ch * 8 + 4], pv[ch * 8 + 5]);
+                        u.w = pack_bf16x2(pv[ch * 8 + 6], pv[ch * 8 + 7]);
+                        *reinterpret_cast<uint4 *>(panel + ((chunk ^ (row & 7)) << 4)) = u;
+                    }
+                }
+                tc_fence_before();
+                mbar_arrive(&s_empty[sb]);
+                fence_proxy_async_smem();
+                mbar_arrive(&p_full[sb]);
+                l_run = l_run * alpha + sum;
+                m_run = m_new;
+                if (j >= 1) {  // fold O_(j-1), then rescale to the new max
+                    const uint32_t pb = (g - 1) & 1, pph = ((g - 1) >> 1) & 1;
+                    if (!mbar_wait(&o_full[pb], pph, abort_flag, p.err)) {
+                        ok = false;
+                        break;
+                    }
+                    tc_fence_after();
+#pragma unroll
+                    for (int d0 = 0; d0 < DH; d0 += 32) {
+                        uint32_t r[32];
+                        tmem_ld32(tmem + tl + 256 + pb * DH + d0, r);
+                        tmem_wait_ld();
+#pragma unroll
+                        for (int d = 0; d < 32; ++d) acc[d0 + d] += __uint_as_float(r[d]);
+                    }
+                    tc_fence_before();
+                    mbar_arrive(&o_empty[pb]);
+                }
+#pragma unroll
+                for (int d = 0; d < DH; ++d) acc[d] *= alpha;
+            }
+            if (!ok) break;
+            {  // fold the last O
+                const uint32_t pb = (g - 1) & 1, pph = ((g - 1) >> 1) & 1;
+                if (!mbar_wait(&o_full[pb], pph, abort_flag, p.err)) break;
+                tc_fence_after();
+#pragma unroll
+                for (int d0 = 0; d0 < DH; d0 += 32) {
+                    uint32_t r[32];
+                    tmem_ld32(tmem + tl + 256 + pb * DH + d0, r);
+                    tmem_wait_ld();
+#pragma unroll
+                    for (int d = 0; d < 32; ++d) acc[d0 + d] += __uint_as_float(r[d]);
+                }
+                tc_fence_before();
+                mbar_arrive(&o_empty[pb]);
+            }
+            const int orow = it.q_row0 + row;
+            if (orow < it.store_end) {
+                const float inv = 1.0f / l_run;
+                uint4 *dst = reinterpret_cast<uint4 *>(p.out + (size_t)orow * p.ldo + it.h * DH);
+#pragma unroll
+                for (int d = 0; d < DH; d += 8) {
+                    uint4 u;
+                    u.x = pack_bf16x2(acc[d + 0] * inv, acc[d + 1] * inv);
+                    u.y = pack_bf16x2(acc[d + 2] * inv, acc[d + 3] * inv);
+                    u.z = pack_bf16x2(acc[d + 4] * inv, acc[d + 5] * inv);
+                    u.w = pack_bf16x2(acc[d + 6] * inv, acc[d + 7] * inv);
+                    dst[d / 8] = u;
+                }
+            }
+        }
+    }
+    __syncthreads();
+    if (*abort_flag) {
+        if (warp == 1 && lane == 0) {
+            mma_commit(drain);
+            wait_bounded(drain, 0, 100000000ull);
+        }
+        if (threadIdx.x == 0) spin_ns(200000);
+        __syncthreads();
+    }
+    if (warp == 1) {
+        tc_fence_after();
+        tmem_dealloc(tmem, Cfg::kTmemCols);
+    }
+}
+
+template <int DH>
+cudaError_t launch_dh(const CUtensorMap *tq, const CUtensorMap *tk, const CUtensorMap *tv, const AttnParams &p,
+                      int grid, cudaStream_t s)
+{
+    static bool attr_set = false;
+    const size_t smem = AttnCfg<DH>::kSmem;
+    if (!attr_set) {
+        cudaError_t e = cudaFuncSetAttribute(k_attn<DH>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+        if (e != cudaSuccess) return e;
+        attr_set = true;
+    }
+    k_attn<DH><<<grid, kAttnThreads, smem, s>>>(*tq, *tk, *tv, p);
+    return cudaGetLastError();
+}
+
+}  // namespace
+
+size_t attn_smem_bytes(int dh) { return dh == 64 ? AttnCfg<64>::kSmem : AttnCfg<32>::kSmem; }
+
+cudaError_t launch_attention(const CUtensorMap *tq, const CUtensorMap *tk, const CUtensorMap *tv,
+                             const AttnParams &p, int grid, cudaStream_t s)
+{
+    if (grid < 1) return cudaErrorInvalidValue;
+    if (p.dh == 64) return launch_dh<64>(tq, tk, tv, p, grid, s);
+    if (p.dh == 32) return launch_dh<32>(tq, tk, tv, p, grid, s);
+    return cudaErrorInvalidValue;
+}
+
+}  // namespace f3dc

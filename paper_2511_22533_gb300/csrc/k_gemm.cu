@@ -1,0 +1,388 @@
+// k_gemm.cu -- K4: the dense projections of the flow transformer (QKV,
+// attention output, cross-attention Q / output, MLP fc1 / fc2, condition
+// K / V; Supp. Sec. F) on 5th-generation tensor cores.
+//
+// out[m, n] = epilogue( sum_k A[m, k] B[n, k] ),  A = activations [M, K]
+// bf16, B = weights [N, K] bf16 (nn.Linear layout), fp32 accumulation.
+//
+// Persistent warp-specialised kernel, one CTA per SM (192 threads):
+//   warp 0     TMA producer: 128x64 A and BNx64 B tiles, 128B-swizzled, into
+//              a STAGES-deep shared-memory ring (mbarrier full / empty)
+//   warp 1     TMEM allocator + single-thread tcgen05.mma issuer
+//              (M=128, N=BN, K=16 per instruction), accumulating in TMEM;
+//              two accumulator buffers so the epilogue of tile i overlaps
+//              the MMAs of tile i+1
+//   warps 2-5  epilogue: tcgen05.ld (thread = row), fused bias / GELU /
+//              per-head RMSNorm / gated fp32 residual, global stores
+// Tiles are walked m-fastest so the CTAs in flight share weight tiles in L2.
+// The tile count can come from device memory (the step's row plan), so the
+// same launch serves any number of active tokens.
+#include <stdio.h>
+
+#include <cudaTypedefs.h>
+
+#include "common.cuh"
+#include "kernels.h"
+
+namespace f3dc {
+
+namespace {
+
+constexpr int kGemmThreads = 192;
+constexpr int kBK = 64;
+constexpr int kAStage = 128 * kBK * 2;
+
+template <int BN>
+struct GemmCfg {
+    static constexpr int kBStage = BN * kBK * 2;
+    static constexpr int kStages = BN == 256 ? 4 : (BN == 128 ? 6 : 8);
+    static constexpr uint32_t kTmemCols = 2 * BN;
+    static constexpr size_t kBarBytes = 256;
+    static constexpr size_t kSmem = 1024 + (size_t)kStages * (kAStage + kBStage) + kBarBytes;
+};
+
+F3DC_DEV bool mbar_wait_bounded(uint64_t *bar, uint32_t parity, uint64_t ns)
+{
+    const uint64_t t0 = globaltimer();
+    while (!mbar_try_wait(bar, parity))
+        if (globaltimer() - t0 > ns) return false;
+    return true;
+}
+
+F3DC_DEV void load_bias32(const bf16 *bias, int col, float (&b)[32])
+{
+    if (!bias) {
+#pragma unroll
+        for (int j = 0; j < 32; ++j) b[j] = 0.f;
+        return;
+    }
+    const uint4 *p = reinterpret_cast<const uint4 *>(bias + col);
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+        const uint4 u = __ldg(p + q);
+        const uint32_t w[4] = {u.x, u.y, u.z, u.w};
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+            b[q * 8 + 2 * j] = bf16_bits_to_f32(w[j] & 0xFFFFu);
+            b[q * 8 + 2 * j + 1] = bf16_bits_to_f32(w[j] >> 16);
+        }
+    }
+}
+
+F3DC_DEV void store_bf16x32(bf16 *dst, const float (&v)[32])
+{
+    uint4 *p = reinterpret_cast<uint4 *>(dst);
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+        uint4 u;
+        u.x = pack_bf16x2(v[q * 8 + 0], v[q * 8 + 1]);
+        u.y = pack_bf16x2(v[q * 8 + 2], v[q * 8 + 3]);
+        u.z = pack_bf16x2(v[q * 8 + 4], v[q * 8 + 5]);
+        u.w = pack_bf16x2(v[q * 8 + 6], v[q * 8 + 7]);
+        p[q] = u;
+    }
+}
+
+// RMSNorm over groups of `dh` columns of a 32-column chunk pair.
+F3DC_DEV void rms_scale(float *v, int n, const bf16 *g, int gcol)
+{
+    float ss = 0.f;
+    for (int j = 0; j < n; ++j) ss += v[j] * v[j];
+    const float rs = rsqrtf(ss / (float)n + 1e-6f);
+    for (int j = 0; j < n; ++j)
+        v[j] = v[j] * rs * bf16_bits_to_f32(reinterpret_cast<const uint16_t *>(g)[gcol + j]);
+}
+
+template <int BN, int EPI>
+F3DC_DEV void epilogue_tile(const GemmParams &p, uint32_t tbase, int grow, int n0)
+{
+    const bool row_ok = grow < p.M;
+    if constexpr (EPI == kEpiQKNorm) {
+#pragma unroll 1
+        for (int c0 = 0; c0 < BN; c0 += 64) {
+            uint32_t r0[32], r1[32];
+            tmem_ld32(tbase + c0, r0);
+            tmem_ld32(tbase + c0 + 32, r1);
+            tmem_wait_ld();
+            const int col = n0 + c0;
+            float b0[32], b1[32];
+            load_bias32(p.bias, col, b0);
+            load_bias32(p.bias, col + 32, b1);
+            float v[64];
+#pragma unroll
+            for (int j = 0; j < 32; ++j) {
+                v[j] = __uint_as_float(r0[j]) + b0[j];
+                v[32 + j] = __uint_as_float(r1[j]) + b1[j];
+            }
+            if (col < 2 * p.width) {
+                const bf16 *g = col < p.width ? p.qn_g : p.kn_g;
+                const int gc = col < p.width ? col : col - p.width;
+                if (p.dh == 64) {
+                    rms_scale(v, 64, g, gc);
+                } else {
+                    rms_scale(v, 32, g, gc);
+                    rms_scale(v + 32, 32, g, gc + 32);
+                }
+            }
+            if (row_ok) {
+                bf16 *dst = reinterpret_cast<bf16 *>(p.out) + (size_t)grow * p.ldo + col;
+                float lo[32], hi[32];
+#pragma unroll
+                for (int j = 0; j < 32; ++j) {
+                    lo[j] = v[j];
+                    hi[j] = v[32 + j];
+                }
+                store_bf16x32(dst, lo);
+                store_bf16x32(dst + 32, hi);
+            }
+        }
+    } else {
+#pragma unroll 1
+        for (int c0 = 0; c0 < BN; c0 += 32) {
+            uint32_t r[32];
+            tmem_ld32(tbase + c0, r);
+            tmem_wait_ld();
+            const int col = n0 + c0;
+            float b[32], v[32];
+            load_bias32(p.bias, col, b);
+#pragma unroll
+            for (int j = 0; j < 32; ++j) v[j] = __uint_as_float(r[j]) + b[j];
+            if constexpr (EPI == kEpiGelu) {
+#pragma unroll
+                for (int j = 0; j < 32; ++j) v[j] = gelu_tanh(v[j]);
+            }
+            if (!row_ok) continue;
+            if constexpr (EPI == kEpiResid) {
+                float *dst = reinterpret_cast<float *>(p.out) + (size_t)grow * p.ldo + col;
+#pragma unroll
+                for (int q = 0; q < 8; ++q) {
+                    float4 x = reinterpret_cast<float4 *>(dst)[q];
+                    float4 g = p.gate ? __ldg(reinterpret_cast<const float4 *>(p.gate + col) + q)
+                                      : make_float4(1.f, 1.f, 1.f, 1.f);
+                    x.x += g.x * v[4 * q + 0];
+                    x.y += g.y * v[4 * q + 1];
+                    x.z += g.z * v[4 * q + 2];
+                    x.w += g.w * v[4 * q + 3];
+                    reinterpret_cast<float4 *>(dst)[q] = x;
+                }
+            } else {
+                store_bf16x32(reinterpret_cast<bf16 *>(p.out) + (size_t)grow * p.ldo + col, v);
+            }
+        }
+    }
+}
+
+template <int BN, int EPI>
+__global__ void __launch_bounds__(kGemmThreads, 1)
+    k_gemm(const __grid_constant__ CUtensorMap tma, const __grid_constant__ CUtensorMap tmb, const GemmParams p)
+{
+    using Cfg = GemmCfg<BN>;
+    constexpr int S = Cfg::kStages;
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+    uint8_t *sa = smem;
+    uint8_t *sb = smem + S * kAStage;
+    uint64_t *bars = reinterpret_cast<uint64_t *>(sb + S * Cfg::kBStage);
+    uint64_t *full = bars, *empty = bars + S, *accf = bars + 2 * S, *acce = accf + 2, *drain = acce + 2;
+    uint32_t *tmem_holder = reinterpret_cast<uint32_t *>(drain + 1);
+    volatile int *abort_flag = reinterpret_cast<volatile int *>(tmem_holder + 1);
+
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int m_tiles = p.m_tiles_dev ? *p.m_tiles_dev : p.m_tiles;
+    const int n_tiles = p.N / BN;
+    const int total = m_tiles * n_tiles;
+    const int kb_n = p.K / kBK;
+
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < S; ++s) {
+            mbar_init(&full[s], 1);
+            mbar_init(&empty[s], 1);
+        }
+        mbar_init(&accf[0], 1);
+        mbar_init(&accf[1], 1);
+        mbar_init(&acce[0], 128);
+        mbar_init(&acce[1], 128);
+        mbar_init(drain, 1);
+        *abort_flag = 0;
+        fence_mbar_init();
+    }
+    if (warp == 1) {
+        tmem_alloc(tmem_holder, Cfg::kTmemCols);
+        tmem_relinquish();
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = *tmem_holder;
+
+    if (warp == 0) {
+        if (lane == 0) {
+            tma_prefetch(&tma);
+            tma_prefetch(&tmb);
+            int s = 0;
+            uint32_t ph = 0;
+            bool ok = true;
+            for (int t = blockIdx.x; t < total && ok; t += gridDim.x) {
+                const int m0 = (t % m_tiles) * 128, n0 = (t / m_tiles) * BN;
+                for (int kb = 0; kb < kb_n; ++kb) {
+                    if (!mbar_wait(&empty[s], ph ^ 1, abort_flag, p.err)) {
+                        ok = false;
+                        break;
+                    }
+                    mbar_arrive_expect_tx(&full[s], kAStage + Cfg::kBStage);
+                    tma_load_2d(sa + s * kAStage, &tma, kb * kBK, m0, &full[s]);
+                    tma_load_2d(sb + s * Cfg::kBStage, &tmb, kb * kBK, n0, &full[s]);
+                    if (++s == S) {
+                        s = 0;
+                        ph ^= 1;
+                    }
+                }
+            }
+        }
+    } else if (warp == 1) {
+        if (lane == 0) {
+            constexpr uint32_t idesc = make_idesc_bf16(128, BN, 0, 0);
+            int s = 0, it = 0;
+            uint32_t ph = 0;
+            bool ok = true;
+            for (int t = blockIdx.x; t < total && ok; t += gridDim.x, ++it) {
+                const int buf = it & 1;
+                const uint32_t aph = (it >> 1) & 1;
+                if (!mbar_wait(&acce[buf], aph ^ 1, abort_flag, p.err)) break;
+                tc_fence_after();
+                const uint32_t d = tmem + buf * BN;
+                for (int kb = 0; kb < kb_n; ++kb) {
+                    if (!mbar_wait(&full[s], ph, abort_flag, p.err)) {
+                        ok = false;
+                        break;
+                    }
+                    tc_fence_after();
+                    const uint32_t a0 = smem_u32(sa + s * kAStage), b0 = smem_u32(sb + s * Cfg::kBStage);
+#pragma unroll
+                    for (int k = 0; k < kBK / 16; ++k)
+                        mma_bf16(d, make_sdesc(a0 + k * 32, 16, 1024, kSwizzle128),
+                                 make_sdesc(b0 + k * 32, 16, 1024, kSwizzle128), idesc, (kb | k) != 0);
+                    mma_commit(&empty[s]);
+                    if (++s == S) {
+                        s = 0;
+                        ph ^= 1;
+                    }
+                }
+                if (ok) mma_commit(&accf[buf]);
+            }
+        }
+    } else {
+        const int q = warp & 3;
+        const int row = q * 32 + lane;
+        int it = 0;
+        for (int t = blockIdx.x; t < total; t += gridDim.x, ++it) {
+            const int buf = it & 1;
+            const uint32_t aph = (it >> 1) & 1;
+            if (!mbar_wait(&accf[buf], aph, abort_flag, p.err)) break;
+            tc_fence_after();
+            const int m0 = (t % m_tiles) * 128, n0 = (t / m_tiles) * BN;
+            const uint32_t tbase = tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(buf * BN);
+            epilogue_tile<BN, EPI>(p, tbase, m0 + row, n0);
+            tc_fence_before();
+            mbar_arrive(&acce[buf]);
+        }
+    }
+    __syncthreads();
+    if (*abort_flag) {
+        // drain: wait (bounded) for this CTA's outstanding MMAs and copies
+        if (warp == 1 && lane == 0) {
+            mma_commit(drain);
+            mbar_wait_bounded(drain, 0, 100000000ull);
+        }
+        if (threadIdx.x == 0) spin_ns(200000);
+        __syncthreads();
+    }
+    if (warp == 1) {
+        tc_fence_after();
+        tmem_dealloc(tmem, Cfg::kTmemCols);
+    }
+}
+
+template <int BN, int EPI>
+cudaError_t launch_one(const CUtensorMap *ta, const CUtensorMap *tb, const GemmParams &p, int grid, cudaStream_t s)
+{
+    static bool attr_set = false;
+    const size_t smem = GemmCfg<BN>::kSmem;
+    if (!attr_set) {
+        cudaError_t e = cudaFuncSetAttribute(k_gemm<BN, EPI>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+        if (e != cudaSuccess) return e;
+        attr_set = true;
+    }
+    k_gemm<BN, EPI><<<grid, kGemmThreads, smem, s>>>(*ta, *tb, p);
+    return cudaGetLastError();
+}
+
+template <int BN>
+cudaError_t launch_bn(const CUtensorMap *ta, const CUtensorMap *tb, const GemmParams &p, int epi, int grid,
+                      cudaStream_t s)
+{
+    switch (epi) {
+    case kEpiBias: return launch_one<BN, kEpiBias>(ta, tb, p, grid, s);
+    case kEpiGelu: return launch_one<BN, kEpiGelu>(ta, tb, p, grid, s);
+    case kEpiResid: return launch_one<BN, kEpiResid>(ta, tb, p, grid, s);
+    case kEpiQKNorm: return launch_one<BN, kEpiQKNorm>(ta, tb, p, grid, s);
+    default: return cudaErrorInvalidValue;
+    }
+}
+
+}  // namespace
+
+size_t gemm_smem_bytes(int bn)
+{
+    switch (bn) {
+    case 64: return GemmCfg<64>::kSmem;
+    case 128: return GemmCfg<128>::kSmem;
+    case 256: return GemmCfg<256>::kSmem;
+    default: return 0;
+    }
+}
+
+cudaError_t launch_gemm(const CUtensorMap *ta, const CUtensorMap *tb, const GemmParams &p, int epi, int bn,
+                        int grid, cudaStream_t s)
+{
+    if (p.K % kBK != 0 || p.N % bn != 0 || grid < 1) return cudaErrorInvalidValue;
+    switch (bn) {
+    case 64: return launch_bn<64>(ta, tb, p, epi, grid, s);
+    case 128: return launch_bn<128>(ta, tb, p, epi, grid, s);
+    case 256: return launch_bn<256>(ta, tb, p, epi, grid, s);
+    default: return cudaErrorInvalidValue;
+    }
+}
+
+bool make_tmap_bf16(CUtensorMap *map, const void *base, uint64_t rows, uint64_t cols, uint64_t ld,
+                    uint32_t box_rows, uint32_t box_cols)
+{
+    static PFN_cuTensorMapEncodeTiled_v12000 encode = nullptr;
+    if (!encode) {
+        cudaDriverEntryPointQueryResult q;
+        void *fn = nullptr;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000, cudaEnableDefault, &q) !=
+                cudaSuccess ||
+            q != cudaDriverEntryPointSuccess || !fn)
+            return false;
+        encode = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(fn);
+    }
+    if (((uintptr_t)base & 15) != 0 || (ld * 2) % 16 != 0) return false;
+    CUtensorMapSwizzle swz;
+    switch (box_cols * 2) {
+    case 128: swz = CU_TENSOR_MAP_SWIZZLE_128B; break;
+    case 64: swz = CU_TENSOR_MAP_SWIZZLE_64B; break;
+    case 32: swz = CU_TENSOR_MAP_SWIZZLE_32B; break;
+    default: return false;
+    }
+    cuuint64_t dims[2] = {cols, rows};
+    cuuint64_t strides[1] = {ld * 2};
+    cuuint32_t box[2] = {box_cols, box_rows};
+    cuuint32_t estr[2] = {1, 1};
+    CUresult r = encode(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void *>(base), dims, strides, box, estr,
+                        CU_TENSOR_MAP_INTERLEAVE_NONE, swz, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                        CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    return r == CUDA_SUCCESS;
+}
+
+}  // namespace f3dc

@@ -1,0 +1,411 @@
+// k_rows.cu -- bandwidth-bound row kernels of the cached step:
+//   K2 gather + input embedding of the active tokens (Sec. 4.2 compaction)
+//   K7 LayerNorm with adaLN modulation or affine parameters (Supp. Sec. F)
+//   final layer (LN + adaLN + Linear W -> C)
+//   K3 cache merge + Euler update + history write (Algorithm 1 step 3) with
+//      the optional dynamic-voxel count of the stand-in decoder (Eq. 1)
+//   K9 timestep embedding and the modulation GEMV of every block
+// All row kernels are persistent grid-stride loops over rows of the packed
+// active matrix whose row count is read from the device plan, so a step can
+// be launched without the host knowing the active counts.
+#include "common.cuh"
+#include "kernels.h"
+
+namespace f3dc {
+
+namespace {
+
+constexpr int kRowThreads = 256;  // 8 warps, one row per warp
+
+F3DC_DEV float4 ld_f4(const float *p) { return *reinterpret_cast<const float4 *>(p); }
+F3DC_DEV void st_f4(float *p, float4 v) { *reinterpret_cast<float4 *>(p) = v; }
+
+F3DC_DEV void bf16x8_to_f32(uint4 u, float (&f)[8])
+{
+    const uint32_t w[4] = {u.x, u.y, u.z, u.w};
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+        f[2 * j] = bf16_bits_to_f32(w[j] & 0xFFFFu);
+        f[2 * j + 1] = bf16_bits_to_f32(w[j] >> 16);
+    }
+}
+
+F3DC_DEV float bf16_at(const bf16 *p, size_t i)
+{
+    return bf16_bits_to_f32(reinterpret_cast<const uint16_t *>(p)[i]);
+}
+
+// ------------------------------------------------------------------ K2
+__global__ void __launch_bounds__(kRowThreads) k_gather_embed(const float *S, int N, int W,
+                                                              const int32_t *active_idx, const Plan *plan,
+                                                              const int32_t *tile_sample, const bf16 *in_w,
+                                                              const bf16 *in_b, const float *pos, float *x,
+                                                              uint32_t *err)
+{
+    const int m_rows = plan->m_rows;
+    const int lane = threadIdx.x & 31, wpb = blockDim.x >> 5;
+    for (int r = blockIdx.x * wpb + (threadIdx.x >> 5); r < m_rows; r += gridDim.x * wpb) {
+        const int b = tile_sample[r / kTileRows];
+        const int j = r - plan->row_off[b];
+        float *xr = x + (size_t)r * W;
+        int i = -1;
+        if (j < plan->n_active[b]) {
+            i = active_idx[(size_t)b * N + j];
+            if ((unsigned)i >= (unsigned)N) {
+                raise_error(err, kDevBadIndex);
+                i = -1;
+            }
+        }
+        if (i < 0) {  // padding row: zeros keep every downstream value finite
+            for (int q = lane; q < W / 4; q += 32) st_f4(xr + 4 * q, make_float4(0.f, 0.f, 0.f, 0.f));
+            continue;
+        }
+        const float *Si = S + ((size_t)b * N + i) * kChannels;
+        float s[8];
+        const float4 s0 = ld_f4(Si), s1 = ld_f4(Si + 4);
+        s[0] = s0.x; s[1] = s0.y; s[2] = s0.z; s[3] = s0.w;
+        s[4] = s1.x; s[5] = s1.y; s[6] = s1.z; s[7] = s1.w;
+        const float *pi = pos + (size_t)i * W;
+        for (int q = lane; q < W / 4; q += 32) {
+            const float4 pe = ld_f4(pi + 4 * q);
+            float o[4] = {pe.x, pe.y, pe.z, pe.w};
+#pragma unroll
+            for (int u = 0; u < 4; ++u) {
+                const int n = 4 * q + u;
+                float wv[8];
+                bf16x8_to_f32(__ldg(reinterpret_cast<const uint4 *>(in_w) + n), wv);
+                float acc = bf16_at(in_b, n);
+#pragma unroll
+                for (int c = 0; c < 8; ++c) acc = fmaf(s[c], wv[c], acc);
+                o[u] += acc;
+            }
+            st_f4(xr + 4 * q, make_float4(o[0], o[1], o[2], o[3]));
+        }
+    }
+}
+
+// ------------------------------------------------------------------ K7
+template <int NV>
+F3DC_DEV void row_stats(const float4 (&v)[NV], int W, float &mean, float &rstd)
+{
+    float s = 0.f;
+#pragma unroll
+    for (int q = 0; q < NV; ++q) s += (v[q].x + v[q].y) + (v[q].z + v[q].w);
+    mean = warp_sum(s) / (float)W;
+    float ss = 0.f;
+#pragma unroll
+    for (int q = 0; q < NV; ++q) {
+        const float a = v[q].x - mean, b = v[q].y - mean, c = v[q].z - mean, d = v[q].w - mean;
+        ss += (a * a + b * b) + (c * c + d * d);
+    }
+    const float var = warp_sum(ss) / (float)W;
+    rstd = rsqrtf(var + 1e-6f);
+}
+
+template <int NV>
+__global__ void __launch_bounds__(kRowThreads) k_layernorm(const float *x, int W, const Plan *plan, int mode,
+                                                           const float *shift, const float *scale, const bf16 *g,
+                                                           const bf16 *bb, bf16 *out)
+{
+    const int m_rows = plan->m_rows;
+    const int lane = threadIdx.x & 31, wpb = blockDim.x >> 5;
+    for (int r = blockIdx.x * wpb + (threadIdx.x >> 5); r < m_rows; r += gridDim.x * wpb) {
+        const float *xr = x + (size_t)r * W;
+        float4 v[NV];
+#pragma unroll
+        for (int q = 0; q < NV; ++q) v[q] = ld_f4(xr + 4 * (q * 32 + lane));
+        float mean, rstd;
+        row_stats<NV>(v, W, mean, rstd);
+        uint16_t *orow = reinterpret_cast<uint16_t *>(out) + (size_t)r * W;
+#pragma unroll
+        for (int q = 0; q < NV; ++q) {
+            const int n0 = 4 * (q * 32 + lane);
+            float y[4] = {(v[q].x - mean) * rstd, (v[q].y - mean) * rstd, (v[q].z - mean) * rstd,
+                          (v[q].w - mean) * rstd};
+            if (mode == 0) {
+                const float4 sc = ld_f4(scale + n0), sh = ld_f4(shift + n0);
+                y[0] = y[0] * (1.f + sc.x) + sh.x;
+                y[1] = y[1] * (1.f + sc.y) + sh.y;
+                y[2] = y[2] * (1.f + sc.z) + sh.z;
+                y[3] = y[3] * (1.f + sc.w) + sh.w;
+            } else {
+#pragma unroll
+                for (int u = 0; u < 4; ++u) y[u] = y[u] * bf16_at(g, n0 + u) + bf16_at(bb, n0 + u);
+            }
+            uint2 pk;
+            pk.x = pack_bf16x2(y[0], y[1]);
+            pk.y = pack_bf16x2(y[2], y[3]);
+            *reinterpret_cast<uint2 *>(orow + n0) = pk;
+        }
+    }
+}
+
+template <int NV>
+__global__ void __launch_bounds__(kRowThreads) k_final_layer(const float *x, int W, const Plan *plan,
+                                                             const float *shift, const float *scale,
+                                                             const bf16 *out_w, const bf16 *out_b, float *v_active)
+{
+    const int m_rows = plan->m_rows;
+    const int lane = threadIdx.x & 31, wpb = blockDim.x >> 5;
+    for (int r = blockIdx.x * wpb + (threadIdx.x >> 5); r < m_rows; r += gridDim.x * wpb) {
+        const float *xr = x + (size_t)r * W;
+        float4 v[NV];
+#pragma unroll
+        for (int q = 0; q < NV; ++q) v[q] = ld_f4(xr + 4 * (q * 32 + lane));
+        float mean, rstd;
+        row_stats<NV>(v, W, mean, rstd);
+        float acc[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+        for (int q = 0; q < NV; ++q) {
+            const int n0 = 4 * (q * 32 + lane);
+            const float4 sc = ld_f4(scale + n0), sh = ld_f4(shift + n0);
+            const float y[4] = {(v[q].x - mean) * rstd * (1.f + sc.x) + sh.x,
+                                (v[q].y - mean) * rstd * (1.f + sc.y) + sh.y,
+                                (v[q].z - mean) * rstd * (1.f + sc.z) + sh.z,
+                                (v[q].w - mean) * rstd * (1.f + sc.w) + sh.w};
+#pragma unroll
+            for (int c = 0; c < 8; ++c) {
+                const uint2 wp = __ldg(reinterpret_cast<const uint2 *>(
+                    reinterpret_cast<const uint16_t *>(out_w) + (size_t)c * W + n0));
+                acc[c] += y[0] * bf16_bits_to_f32(wp.x & 0xFFFFu) + y[1] * bf16_bits_to_f32(wp.x >> 16) +
+                          y[2] * bf16_bits_to_f32(wp.y & 0xFFFFu) + y[3] * bf16_bits_to_f32(wp.y >> 16);
+            }
+        }
+#pragma unroll
+        for (int c = 0; c < 8; ++c) acc[c] = warp_sum(acc[c]);
+        if (lane == 0) {
+            float o[8];
+#pragma unroll
+            for (int c = 0; c < 8; ++c) o[c] = acc[c] + bf16_at(out_b, c);
+            st_f4(v_active + (size_t)r * 8, make_float4(o[0], o[1], o[2], o[3]));
+            st_f4(v_active + (size_t)r * 8 + 4, make_float4(o[4], o[5], o[6], o[7]));
+        }
+    }
+}
+
+// ------------------------------------------------------------------ K3
+constexpr int kMergeThreads = 256;
+constexpr int kMaxG = 512;
+
+__global__ void __launch_bounds__(kMergeThreads) k_merge_euler(const MergeArgs a)
+{
+    __shared__ float dec[8 * kMaxG];
+    const bool count = a.dyn != nullptr;
+    if (count) {
+        for (int q = threadIdx.x; q < 8 * a.G; q += blockDim.x)
+            dec[q] = bf16_bits_to_f32(a.dec_w[q]);
+        __syncthreads();
+    }
+    const size_t total = (size_t)a.B * a.N;
+    const size_t tok = (size_t)blockIdx.x * blockDim.x + threadIdx.x;
+    const bool valid = tok < total;
+    int flips = 0;
+    int b = 0;
+    if (valid) {
+        b = (int)(tok / a.N);
+        float *Sp = a.S + tok * 8;
+        const float4 s0 = ld_f4(Sp), s1 = ld_f4(Sp + 4);
+        const float so[8] = {s0.x, s0.y, s0.z, s0.w, s1.x, s1.y, s1.z, s1.w};
+        const int row = a.row_of_token[tok];
+        uint32_t vb[8];
+        if (row >= 0) {
+            if (row >= a.max_rows) {
+                raise_error(a.err, kDevBadIndex);
+                for (int c = 0; c < 8; ++c) vb[c] = 0;
+            } else {
+                const float4 v0 = ld_f4(a.v_active + (size_t)row * 8), v1 = ld_f4(a.v_active + (size_t)row * 8 + 4);
+                const float va[8] = {v0.x, v0.y, v0.z, v0.w, v1.x, v1.y, v1.z, v1.w};
+#pragma unroll
+                for (int c = 0; c < 8; ++c) vb[c] = f32_to_bf16_bits(va[c]);
+            }
+        } else {  // cached token: reuse the stored velocity bit for bit
+            const uint4 p = *reinterpret_cast<const uint4 *>(a.v_prev1 + tok * 8);
+            const uint32_t pw[4] = {p.x, p.y, p.z, p.w};
+#pragma unroll
+            for (int c = 0; c < 8; ++c) vb[c] = (pw[c >> 1] >> ((c & 1) * 16)) & 0xFFFFu;
+        }
+        float sn[8];
+#pragma unroll
+        for (int c = 0; c < 8; ++c) sn[c] = __fsub_rn(so[c], __fmul_rn(a.dt, bf16_bits_to_f32(vb[c])));
+        st_f4(Sp, make_float4(sn[0], sn[1], sn[2], sn[3]));
+        st_f4(Sp + 4, make_float4(sn[4], sn[5], sn[6], sn[7]));
+        uint4 vo;
+        vo.x = vb[0] | (vb[1] << 16);
+        vo.y = vb[2] | (vb[3] << 16);
+        vo.z = vb[4] | (vb[5] << 16);
+        vo.w = vb[6] | (vb[7] << 16);
+        *reinterpret_cast<uint4 *>(a.v_out + tok * 8) = vo;
+        if (count) {
+            for (int j = 0; j < a.G; ++j) {
+                float lo = 0.0f, ln = 0.0f;
+#pragma unroll
+                for (int c = 0; c < 8; ++c) {
+                    lo = __fadd_rn(lo, __fmul_rn(so[c], dec[c * a.G + j]));
+                    ln = __fadd_rn(ln, __fmul_rn(sn[c], dec[c * a.G + j]));
+                }
+                flips += (lo > 0.0f) != (ln > 0.0f);
+            }
+        }
+    }
+    if (count) {
+        // N % 32 == 0 is enforced at create, so a warp never spans two samples
+        int f = flips;
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) f += __shfl_xor_sync(0xffffffffu, f, o);
+        if ((threadIdx.x & 31) == 0 && valid && f)
+            atomicAdd(reinterpret_cast<unsigned long long *>(a.dyn + b), (unsigned long long)f);
+    }
+}
+
+__global__ void k_scatter_rows(const float *v_active, const Plan *plan, int N, float *v_out)
+{
+    const int b = blockIdx.y;
+    const int na = plan->n_active[b], off = plan->row_off[b];
+    for (int j = blockIdx.x * blockDim.x + threadIdx.x; j < na; j += gridDim.x * blockDim.x) {
+        const float *src = v_active + (size_t)(off + j) * 8;
+        float *dst = v_out + ((size_t)b * N + j) * 8;
+        st_f4(dst, ld_f4(src));
+        st_f4(dst + 4, ld_f4(src + 4));
+    }
+}
+
+// ------------------------------------------------------------------ K9
+__global__ void k_time_freq(float t, float *freq)
+{
+    const int f = threadIdx.x;  // 128 threads
+    const float w = expf(-9.210340371976184f * (float)f / 128.0f);  // ln(10000)
+    const float arg = 1000.0f * t * w;
+    freq[f] = cosf(arg);
+    freq[128 + f] = sinf(arg);
+}
+
+F3DC_DEV float silu(float v) { return v / (1.0f + expf(-v)); }
+
+constexpr int kGemvThreads = 512;
+constexpr int kGemvMaxK = 4096;
+
+__global__ void __launch_bounds__(kGemvThreads) k_gemv(const float *x, int K, const bf16 *w, const bf16 *bias,
+                                                       float *y, int rows, int silu_in, int silu_out)
+{
+    __shared__ float xs[kGemvMaxK];
+    for (int k = threadIdx.x; k < K; k += blockDim.x) xs[k] = silu_in ? silu(x[k]) : x[k];
+    __syncthreads();
+    const int lane = threadIdx.x & 31, wpb = blockDim.x >> 5;
+    const int chunks = K / 256;  // 8 bf16 per lane per chunk
+    const uint4 *W4 = reinterpret_cast<const uint4 *>(w);
+    for (int r = (blockIdx.x * wpb + (threadIdx.x >> 5)) * 2; r < rows; r += gridDim.x * wpb * 2) {
+        const bool two = r + 1 < rows;
+        float acc0 = 0.f, acc1 = 0.f;
+        for (int q = 0; q < chunks; ++q) {
+            const int k0 = (q * 32 + lane) * 8;
+            const uint4 u0 = __ldg(W4 + ((size_t)r * K + k0) / 8);
+            const uint4 u1 = two ? __ldg(W4 + ((size_t)(r + 1) * K + k0) / 8) : make_uint4(0, 0, 0, 0);
+            float f0[8], f1[8];
+            bf16x8_to_f32(u0, f0);
+            bf16x8_to_f32(u1, f1);
+#pragma unroll
+            for (int j = 0; j < 8; ++j) {
+                acc0 = fmaf(f0[j], xs[k0 + j], acc0);
+                acc1 = fmaf(f1[j], xs[k0 + j], acc1);
+            }
+        }
+        acc0 = warp_sum(acc0);
+        acc1 = warp_sum(acc1);
+        if (lane == 0) {
+            float v0 = acc0 + (bias ? bf16_at(bias, r) : 0.f);
+            y[r] = silu_out ? silu(v0) : v0;
+            if (two) {
+                float v1 = acc1 + (bias ? bf16_at(bias, r + 1) : 0.f);
+                y[r + 1] = silu_out ? silu(v1) : v1;
+            }
+        }
+    }
+}
+
+int row_grid(int num_sms, int max_rows)
+{
+    const int wpb = kRowThreads / 32;
+    int g = num_sms * 4;
+    const int need = (max_rows + wpb - 1) / wpb;
+    return need < g ? (need > 0 ? need : 1) : g;
+}
+
+}  // namespace
+
+cudaError_t launch_gather_embed(const float *S, int N, int W, const int32_t *active_idx, const Plan *plan,
+                                const int32_t *tile_sample, const bf16 *in_w, const bf16 *in_b,
+                                const float *pos, float *x, int max_rows, int num_sms, uint32_t *err,
+                                cudaStream_t s)
+{
+    k_gather_embed<<<row_grid(num_sms, max_rows), kRowThreads, 0, s>>>(S, N, W, active_idx, plan, tile_sample,
+                                                                       in_w, in_b, pos, x, err);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_layernorm(const float *x, int W, const Plan *plan, int mode, const float *shift,
+                             const float *scale, const bf16 *g, const bf16 *b, bf16 *out, int max_rows,
+                             int num_sms, cudaStream_t s)
+{
+    const int grid = row_grid(num_sms, max_rows);
+    switch (W / 128) {
+    case 1: k_layernorm<1><<<grid, kRowThreads, 0, s>>>(x, W, plan, mode, shift, scale, g, b, out); break;
+    case 2: k_layernorm<2><<<grid, kRowThreads, 0, s>>>(x, W, plan, mode, shift, scale, g, b, out); break;
+    case 4: k_layernorm<4><<<grid, kRowThreads, 0, s>>>(x, W, plan, mode, shift, scale, g, b, out); break;
+    case 8: k_layernorm<8><<<grid, kRowThreads, 0, s>>>(x, W, plan, mode, shift, scale, g, b, out); break;
+    case 16: k_layernorm<16><<<grid, kRowThreads, 0, s>>>(x, W, plan, mode, shift, scale, g, b, out); break;
+    default: return cudaErrorInvalidValue;
+    }
+    return cudaGetLastError();
+}
+
+cudaError_t launch_final_layer(const float *x, int W, const Plan *plan, const float *shift,
+                               const float *scale, const bf16 *out_w, const bf16 *out_b, float *v_active,
+                               int max_rows, int num_sms, cudaStream_t s)
+{
+    const int grid = row_grid(num_sms, max_rows);
+    switch (W / 128) {
+    case 1: k_final_layer<1><<<grid, kRowThreads, 0, s>>>(x, W, plan, shift, scale, out_w, out_b, v_active); break;
+    case 2: k_final_layer<2><<<grid, kRowThreads, 0, s>>>(x, W, plan, shift, scale, out_w, out_b, v_active); break;
+    case 4: k_final_layer<4><<<grid, kRowThreads, 0, s>>>(x, W, plan, shift, scale, out_w, out_b, v_active); break;
+    case 8: k_final_layer<8><<<grid, kRowThreads, 0, s>>>(x, W, plan, shift, scale, out_w, out_b, v_active); break;
+    case 16: k_final_layer<16><<<grid, kRowThreads, 0, s>>>(x, W, plan, shift, scale, out_w, out_b, v_active); break;
+    default: return cudaErrorInvalidValue;
+    }
+    return cudaGetLastError();
+}
+
+cudaError_t launch_merge_euler(const MergeArgs &a, cudaStream_t s)
+{
+    if (a.dyn && (a.G > kMaxG || a.N % 32 != 0)) return cudaErrorInvalidValue;
+    const size_t total = (size_t)a.B * a.N;
+    const int grid = (int)((total + kMergeThreads - 1) / kMergeThreads);
+    k_merge_euler<<<grid, kMergeThreads, 0, s>>>(a);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_scatter_rows(const float *v_active, const Plan *plan, int B, int N, float *v_out,
+                                cudaStream_t s)
+{
+    dim3 grid((N + 255) / 256, B);
+    k_scatter_rows<<<grid, 256, 0, s>>>(v_active, plan, N, v_out);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_time_freq(float t, float *freq, cudaStream_t s)
+{
+    k_time_freq<<<1, 128, 0, s>>>(t, freq);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_gemv(const float *x, int K, const bf16 *w, const bf16 *b, float *y, int rows, int silu_in,
+                        int silu_out, int num_sms, cudaStream_t s)
+{
+    if (K % 256 != 0 || K > kGemvMaxK) return cudaErrorInvalidValue;
+    const int wpb = kGemvThreads / 32;
+    int grid = (rows + 2 * wpb - 1) / (2 * wpb);
+    if (grid > num_sms * 4) grid = num_sms * 4;
+    k_gemv<<<grid, kGemvThreads, 0, s>>>(x, K, w, b, y, rows, silu_in, silu_out);
+    return cudaGetLastError();
+}
+
+}  // namespace f3dc

@@ -1,0 +1,325 @@
+// k_select.cu -- K1: Spatiotemporal Stability Criterion scoring and
+// lowest-c selection (Sec. 4.1 V_i and Eq. ICE; Sec. 4.2 Eq. ssc and
+// Eq. normalize; Algorithm 1 function SSC), fused with the row plan of the
+// step (Sec. 4.2 index-based token compaction).
+//
+// One CTA of 1024 threads per sample.  Pass 1 streams the two newest
+// velocity slots (16 B + 16 B per token, coalesced uint4 loads) and reduces
+// min / max of V and A; pass 2 re-reads them (L2-resident), forms the score
+// in the same fp32 operation order as the definition and stores an order-
+// preserving 32-bit key per token in shared memory.  A 4 x 8-bit radix
+// select finds the c-th smallest key; an index-ordered scan then caches
+// every key below it plus the lowest-index ties, and compacts the active
+// tokens in ascending order.
+#include "common.cuh"
+#include "kernels.h"
+
+namespace f3dc {
+
+namespace {
+
+constexpr int kSelThreads = 1024;
+constexpr int kSelWarps = kSelThreads / 32;
+constexpr int kSelMaxTokens = 49152;  // 4-byte keys in shared memory
+
+F3DC_DEV void load_token(const uint16_t *v1, const uint16_t *v2, size_t tok, float &V, float &A)
+{
+    const uint4 p = __ldg(reinterpret_cast<const uint4 *>(v1) + tok);
+    const uint4 q = __ldg(reinterpret_cast<const uint4 *>(v2) + tok);
+    const uint32_t pw[4] = {p.x, p.y, p.z, p.w};
+    const uint32_t qw[4] = {q.x, q.y, q.z, q.w};
+    float sv = 0.0f, sa = 0.0f;
+#pragma unroll
+    for (int c = 0; c < 8; ++c) {
+        const uint32_t pu = (pw[c >> 1] >> ((c & 1) * 16)) & 0xFFFFu;
+        const uint32_t qu = (qw[c >> 1] >> ((c & 1) * 16)) & 0xFFFFu;
+        const float x = bf16_bits_to_f32(pu);
+        const float y = bf16_bits_to_f32(qu);
+        const float d = __fsub_rn(x, y);
+        sv = __fadd_rn(sv, __fmul_rn(x, x));
+        sa = __fadd_rn(sa, __fmul_rn(d, d));
+    }
+    V = __fsqrt_rn(sv);
+    A = __fsqrt_rn(sa);
+}
+
+// min-max normalisation; NaN stays NaN, a degenerate range gives 0.
+F3DC_DEV float norm1(float x, float mn, float mx)
+{
+    if (isnan(x)) return x;
+    if (!(mx > mn)) return 0.0f;
+    return __fdiv_rn(__fsub_rn(x, mn), __fsub_rn(mx, mn));
+}
+
+// Order-preserving key: equal floats (including -0 / +0) give equal keys,
+// every NaN gives the largest key (never cached before a number).
+F3DC_DEV uint32_t score_key(float s)
+{
+    if (isnan(s)) return 0xFFFFFFFFu;
+    if (s == 0.0f) s = 0.0f;
+    const uint32_t u = __float_as_uint(s);
+    return (u & 0x80000000u) ? ~u : (u | 0x80000000u);
+}
+
+F3DC_DEV int pad_tile(int a) { return (a + kTileRows - 1) / kTileRows * kTileRows; }
+
+F3DC_DEV int clamp_quota(int q, int N) { return q < 0 ? 0 : (q > N ? N : q); }
+
+// Row offset of sample b, total padded rows, and the sample's tiles.
+F3DC_DEV void write_plan(const SelectArgs &a, int b, int na, int &off)
+{
+    __shared__ int s_off;
+    if (threadIdx.x == 0) {
+        int o = 0;
+        for (int bb = 0; bb < b; ++bb) o += pad_tile(a.N - clamp_quota(a.quota[bb], a.N));
+        s_off = o;
+        if (a.plan) {
+            a.plan->n_active[b] = na;
+            a.plan->row_off[b] = o;
+            if (b == 0) {
+                int tot = 0;
+                for (int bb = 0; bb < a.B; ++bb) tot += pad_tile(a.N - clamp_quota(a.quota[bb], a.N));
+                a.plan->m_rows = tot;
+                a.plan->n_tiles = tot / kTileRows;
+            }
+        }
+    }
+    __syncthreads();
+    off = s_off;
+    if (a.tile_sample) {
+        const int t0 = off / kTileRows, nt = pad_tile(na) / kTileRows;
+        for (int t = threadIdx.x; t < nt; t += blockDim.x) a.tile_sample[t0 + t] = b;
+    }
+}
+
+__global__ void __launch_bounds__(kSelThreads, 1) k_ssc_select(const SelectArgs a)
+{
+    extern __shared__ uint32_t keys[];
+    __shared__ uint32_t hist[256];
+    __shared__ float red[4][kSelWarps];
+    __shared__ uint32_t wsum_lt[kSelWarps], wsum_eq[kSelWarps];
+    __shared__ uint32_t s_digit, s_rank;
+
+    const int b = blockIdx.x, tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    const int N = a.N;
+    const int c = clamp_quota(a.quota[b], N);
+    const int na = N - c;
+    const size_t base = (size_t)b * N;
+
+    int off = 0;
+    write_plan(a, b, na, off);
+    if (a.n_active && tid == 0) a.n_active[b] = na;
+
+    if (c == 0) {  // nothing cached: every token active, no scoring needed
+        for (int i = tid; i < N; i += kSelThreads) {
+            a.active_idx[base + i] = i;
+            if (a.mask) a.mask[base + i] = 0;
+            if (a.row_of_token) a.row_of_token[base + i] = off + i;
+        }
+        return;
+    }
+    if (c == N) {  // everything cached
+        for (int i = tid; i < N; i += kSelThreads) {
+            if (a.mask) a.mask[base + i] = 1;
+            if (a.row_of_token) a.row_of_token[base + i] = -1;
+        }
+        return;
+    }
+
+    // ---- pass 1: min / max of V and A (NaN never wins a comparison)
+    float mnV = INFINITY, mxV = -INFINITY, mnA = INFINITY, mxA = -INFINITY;
+    for (int i = tid; i < N; i += kSelThreads) {
+        float V, A;
+        load_token(a.v1, a.v2, base + i, V, A);
+        if (V < mnV) mnV = V;
+        if (V > mxV) mxV = V;
+        if (A < mnA) mnA = A;
+        if (A > mxA) mxA = A;
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+        mnV = fminf(mnV, __shfl_xor_sync(0xffffffffu, mnV, o));
+        mxV = fmaxf(mxV, __shfl_xor_sync(0xffffffffu, mxV, o));
+        mnA = fminf(mnA, __shfl_xor_sync(0xffffffffu, mnA, o));
+        mxA = fmaxf(mxA, __shfl_xor_sync(0xffffffffu, mxA, o));
+    }
+    if (lane == 0) {
+        red[0][warp] = mnV;
+        red[1][warp] = mxV;
+        red[2][warp] = mnA;
+        red[3][warp] = mxA;
+    }
+    __syncthreads();
+    mnV = red[0][lane];
+    mxV = red[1][lane];
+    mnA = red[2][lane];
+    mxA = red[3][lane];
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+        mnV = fminf(mnV, __shfl_xor_sync(0xffffffffu, mnV, o));
+        mxV = fmaxf(mxV, __shfl_xor_sync(0xffffffffu, mxV, o));
+        mnA = fminf(mnA, __shfl_xor_sync(0xffffffffu, mnA, o));
+        mxA = fmaxf(mxA, __shfl_xor_sync(0xffffffffu, mxA, o));
+    }
+
+    // ---- pass 2: C_i = w_a norm(A_i) + w_v norm(V_i) -> ordered keys
+    for (int i = tid; i < N; i += kSelThreads) {
+        float V, A;
+        load_token(a.v1, a.v2, base + i, V, A);
+        const float s = __fadd_rn(__fmul_rn(a.wa, norm1(A, mnA, mxA)), __fmul_rn(a.wv, norm1(V, mnV, mxV)));
+        keys[i] = score_key(s);
+    }
+    __syncthreads();
+
+    // ---- radix select: the c-th smallest key (1-based rank c)
+    uint32_t prefix = 0, hi_mask = 0;
+    uint32_t rank = (uint32_t)c;
+    for (int shift = 24; shift >= 0; shift -= 8) {
+        if (tid < 256) hist[tid] = 0;
+        __syncthreads();
+        for (int i0 = 0; i0 < N; i0 += kSelThreads) {
+            const int i = i0 + tid;
+            const bool in = i < N && (keys[i] & hi_mask) == prefix;
+            const uint32_t digit = in ? (keys[i] >> shift) & 255u : 256u;
+            const uint32_t peers = __match_any_sync(0xffffffffu, digit);
+            if (in && (__ffs(peers) - 1) == lane) atomicAdd(&hist[digit], (uint32_t)__popc(peers));
+        }
+        __syncthreads();
+        if (warp == 0) {
+            uint32_t loc[8], sum = 0;
+#pragma unroll
+            for (int j = 0; j < 8; ++j) {
+                loc[j] = hist[lane * 8 + j];
+                sum += loc[j];
+            }
+            uint32_t incl = sum;
+#pragma unroll
+            for (int o = 1; o < 32; o <<= 1) {
+                const uint32_t n = __shfl_up_sync(0xffffffffu, incl, o);
+                if (lane >= o) incl += n;
+            }
+            const uint32_t excl = incl - sum;
+            if (excl < rank && rank <= incl) {
+                uint32_t cum = excl;
+#pragma unroll
+                for (int j = 0; j < 8; ++j) {
+                    if (cum + loc[j] >= rank) {
+                        s_digit = (uint32_t)(lane * 8 + j);
+                        s_rank = rank - cum;
+                        break;
+                    }
+                    cum += loc[j];
+                }
+            }
+        }
+        __syncthreads();
+        prefix |= s_digit << shift;
+        hi_mask |= 255u << shift;
+        rank = s_rank;
+        __syncthreads();
+    }
+    const uint32_t thr = prefix;  // keys below thr are cached, plus the first `rank` ties
+
+    // ---- index-ordered compaction.  For token i with L(i) smaller keys and
+    // E(i) ties before it, the tie is cached iff E(i) < rank, and an active
+    // token lands at position i - L(i) - min(E(i), rank).
+    uint32_t run_lt = 0, run_eq = 0;
+    const uint32_t lt_mask = (1u << lane) - 1u;
+    for (int i0 = 0; i0 < N; i0 += kSelThreads) {
+        const int i = i0 + tid;
+        const bool valid = i < N;
+        const uint32_t k = valid ? keys[i] : 0xFFFFFFFFu;
+        const bool lt = valid && k < thr;
+        const bool eq = valid && k == thr;
+        const uint32_t blt = __ballot_sync(0xffffffffu, lt), beq = __ballot_sync(0xffffffffu, eq);
+        if (lane == 0) {
+            wsum_lt[warp] = __popc(blt);
+            wsum_eq[warp] = __popc(beq);
+        }
+        __syncthreads();
+        uint32_t plt = run_lt + __popc(blt & lt_mask), peq = run_eq + __popc(beq & lt_mask);
+        uint32_t tot_lt = 0, tot_eq = 0;
+        for (int w = 0; w < kSelWarps; ++w) {
+            const uint32_t x = wsum_lt[w], y = wsum_eq[w];
+            if (w < warp) {
+                plt += x;
+                peq += y;
+            }
+            tot_lt += x;
+            tot_eq += y;
+        }
+        if (valid) {
+            const bool cached = lt || (eq && peq < rank);
+            if (a.mask) a.mask[base + i] = cached ? 1 : 0;
+            if (!cached) {
+                const uint32_t pos = (uint32_t)i - plt - min(peq, rank);
+                if (pos >= (uint32_t)na) raise_error(a.err, kDevBadPlan);
+                else {
+                    a.active_idx[base + pos] = i;
+                    if (a.row_of_token) a.row_of_token[base + i] = off + (int)pos;
+                }
+            } else if (a.row_of_token) {
+                a.row_of_token[base + i] = -1;
+            }
+        }
+        run_lt += tot_lt;
+        run_eq += tot_eq;
+        __syncthreads();
+    }
+    if (tid == 0 && (uint32_t)N - run_lt - min(run_eq, rank) != (uint32_t)na) raise_error(a.err, kDevBadPlan);
+}
+
+__global__ void k_plan_from_counts(const int32_t *n_active, int B, int N, Plan *plan, int32_t *tile_sample,
+                                   uint32_t *err)
+{
+    __shared__ int offs[kMaxBatch + 1];
+    if (threadIdx.x == 0) {
+        int o = 0;
+        for (int b = 0; b < B; ++b) {
+            int na = n_active[b];
+            if (na < 0 || na > N) {
+                raise_error(err, kDevBadIndex);
+                na = na < 0 ? 0 : N;
+            }
+            offs[b] = o;
+            plan->n_active[b] = na;
+            plan->row_off[b] = o;
+            o += pad_tile(na);
+        }
+        offs[B] = o;
+        plan->m_rows = o;
+        plan->n_tiles = o / kTileRows;
+    }
+    __syncthreads();
+    for (int b = 0; b < B; ++b) {
+        const int t0 = offs[b] / kTileRows, t1 = offs[b + 1] / kTileRows;
+        for (int t = t0 + threadIdx.x; t < t1; t += blockDim.x) tile_sample[t] = b;
+    }
+}
+
+}  // namespace
+
+int ssc_select_max_tokens() { return kSelMaxTokens; }
+
+cudaError_t launch_ssc_select(const SelectArgs &a, cudaStream_t s)
+{
+    if (a.N > kSelMaxTokens || a.B < 1 || a.B > kMaxBatch) return cudaErrorInvalidValue;
+    const size_t smem = (size_t)a.N * sizeof(uint32_t);
+    cudaError_t e = cudaFuncSetAttribute(k_ssc_select, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
+    k_ssc_select<<<a.B, kSelThreads, smem, s>>>(a);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_plan_from_counts(const int32_t *n_active, const int32_t *active_idx, int B, int N,
+                                    Plan *plan, int32_t *tile_sample, int32_t *row_of_token, uint32_t *err,
+                                    cudaStream_t s)
+{
+    (void)active_idx;
+    (void)row_of_token;
+    if (B < 1 || B > kMaxBatch) return cudaErrorInvalidValue;
+    k_plan_from_counts<<<1, 256, 0, s>>>(n_active, B, N, plan, tile_sample, err);
+    return cudaGetLastError();
+}
+
+}  // namespace f3dc

@@ -1,0 +1,145 @@
+// kernels.h -- internal launch interface between the C-ABI layer (api.cu)
+// and the CUDA kernels of libf3dc.
+#pragma once
+
+#include <cuda.h>
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+namespace f3dc {
+
+constexpr int kTileRows = 128;   // rows per tile; every sample's packed rows start on a tile
+constexpr int kMaxBatch = 64;
+constexpr int kChannels = 8;
+
+typedef __nv_bfloat16 bf16;
+
+// Per-step row plan.  Active tokens of all samples are packed row-wise,
+// sample b's a_b rows starting at row_off[b] (a multiple of 128) and padded
+// to a multiple of 128 with finite rows, so every 128-row tile belongs to
+// one sample (tile_sample[] in a separate array).
+struct Plan {
+    int32_t n_tiles;               // padded rows / 128
+    int32_t m_rows;                // padded rows
+    int32_t n_active[kMaxBatch];   // a_b
+    int32_t row_off[kMaxBatch];    // first packed row of sample b
+};
+
+// ------------------------------------------------------------ selection
+struct SelectArgs {
+    const uint16_t *v1, *v2;   // bf16 [B, N, 8]
+    const int32_t *quota;      // [B]
+    int B, N;
+    float wa, wv;              // omega and 1 - omega, fp32
+    int32_t *active_idx;       // [B, N]
+    int32_t *n_active;         // [B], nullable
+    uint8_t *mask;             // [B, N], nullable
+    int32_t *row_of_token;     // [B, N], nullable: packed row or -1 if cached
+    Plan *plan;                // nullable
+    int32_t *tile_sample;      // nullable
+    uint32_t *err;
+};
+cudaError_t launch_ssc_select(const SelectArgs &a, cudaStream_t s);
+int ssc_select_max_tokens();
+
+// Plan from given active lists (diagnostic forward): counts -> plan,
+// tile_sample and row_of_token.
+cudaError_t launch_plan_from_counts(const int32_t *n_active, const int32_t *active_idx, int B, int N,
+                                    Plan *plan, int32_t *tile_sample, int32_t *row_of_token, uint32_t *err,
+                                    cudaStream_t s);
+
+// ------------------------------------------------------------ row kernels
+// x[r] = in_w S[b, i] + in_b + pos[i] for packed active row r; zero pad rows.
+cudaError_t launch_gather_embed(const float *S, int N, int W, const int32_t *active_idx, const Plan *plan,
+                                const int32_t *tile_sample, const bf16 *in_w, const bf16 *in_b,
+                                const float *pos, float *x, int max_rows, int num_sms, uint32_t *err,
+                                cudaStream_t s);
+
+// h = LN(x) (1 + scale) + shift (mode 0, fp32 mod vectors) or LN(x) g + b
+// (mode 1, bf16 affine).  rows from plan->m_rows.
+cudaError_t launch_layernorm(const float *x, int W, const Plan *plan, int mode, const float *shift,
+                             const float *scale, const bf16 *g, const bf16 *b, bf16 *out, int max_rows,
+                             int num_sms, cudaStream_t s);
+
+// v_active[r, c] = out_w (LN(x_r)(1 + scale) + shift) + out_b  (final layer)
+cudaError_t launch_final_layer(const float *x, int W, const Plan *plan, const float *shift,
+                               const float *scale, const bf16 *out_w, const bf16 *out_b, float *v_active,
+                               int max_rows, int num_sms, cudaStream_t s);
+
+// Cache merge + Euler + history write (+ dynamic voxels).
+struct MergeArgs {
+    float *S;                     // [B, N, 8]
+    const float *v_active;        // [rows, 8]
+    const int32_t *row_of_token;  // [B, N]
+    const uint16_t *v_prev1;      // bf16 [B, N, 8] (v_cache)
+    uint16_t *v_out;              // bf16 [B, N, 8] (v_t)
+    int B, N;
+    float dt;
+    const uint16_t *dec_w;        // bf16 [8, G]
+    int G;
+    int64_t *dyn;                 // nullable [B]
+    int max_rows;
+    uint32_t *err;
+};
+cudaError_t launch_merge_euler(const MergeArgs &a, cudaStream_t s);
+
+// Scatter packed rows back to sample-local positions (diagnostic forward).
+cudaError_t launch_scatter_rows(const float *v_active, const Plan *plan, int B, int N, float *v_out,
+                                cudaStream_t s);
+
+// ------------------------------------------------------------ t-embedding
+cudaError_t launch_time_freq(float t, float *freq, cudaStream_t s);
+// y[n] = act_out(sum_k act_in(x[k]) w[n, k] + b[n]); act = SiLU when flag set
+cudaError_t launch_gemv(const float *x, int K, const bf16 *w, const bf16 *b, float *y, int rows, int silu_in,
+                        int silu_out, int num_sms, cudaStream_t s);
+
+// ------------------------------------------------------------ GEMM
+enum GemmEpi { kEpiBias = 0, kEpiGelu = 1, kEpiResid = 2, kEpiQKNorm = 3 };
+
+struct GemmParams {
+    int M;                    // rows stored are < M
+    int N, K;
+    const int32_t *m_tiles_dev;   // nullable: tile count read on device
+    int m_tiles;                  // used when m_tiles_dev is null
+    void *out;
+    int ldo;                  // elements
+    const bf16 *bias;         // nullable
+    const float *gate;        // nullable (RESID)
+    const bf16 *qn_g, *kn_g;  // QKNORM gammas [W]
+    int width, dh;            // QKNORM: columns < 2*width are normalised per dh-group
+    uint32_t *err;
+};
+// bn in {64, 128, 256}
+cudaError_t launch_gemm(const CUtensorMap *ta, const CUtensorMap *tb, const GemmParams &p, int epi, int bn,
+                        int grid, cudaStream_t s);
+size_t gemm_smem_bytes(int bn);
+
+// ------------------------------------------------------------ attention
+struct AttnParams {
+    int heads, dh;
+    int q_col0, k_col0, v_col0;    // column of head 0 in the q / kv buffers
+    int mode;                      // 0 self (plan), 1 cross (b * nk_fixed), 2 single sequence
+    const int32_t *n_tiles_dev;    // nullable
+    int n_tiles;
+    const int32_t *tile_sample;    // modes 0, 1
+    const Plan *plan;              // mode 0
+    int nk_fixed;                  // modes 1, 2
+    int q_rows;                    // mode 2: rows stored are < q_rows
+    bf16 *out;
+    int ldo;
+    float scale_log2;              // log2(e) / sqrt(dh)
+    uint32_t *err;
+};
+cudaError_t launch_attention(const CUtensorMap *tq, const CUtensorMap *tk, const CUtensorMap *tv,
+                             const AttnParams &p, int grid, cudaStream_t s);
+size_t attn_smem_bytes(int dh);
+
+// ------------------------------------------------------------ host helpers
+// 2-D bf16 tensor map over a row-major [rows, cols] matrix with leading
+// dimension ld (elements), box [box_rows, box_cols], 128B (box_cols = 64) or
+// 64B (box_cols = 32) swizzle.  Returns false on failure.
+bool make_tmap_bf16(CUtensorMap *map, const void *base, uint64_t rows, uint64_t cols, uint64_t ld,
+                    uint32_t box_rows, uint32_t box_cols);
+
+}  // namespace f3dc

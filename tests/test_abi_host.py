@@ -1,0 +1,78 @@
+"""libf3dc.so loads without a GPU, exports every symbol include/f3dc.h
+declares, and its host-only schedule logic (Supp. Sec. D; Sec. 4.2 PCSC;
+Algorithm 1 phases and tau rule) agrees exactly with the oracle."""
+import ctypes as C
+
+import numpy as np
+import pytest
+
+from paper_2511_22533_gb300 import f3dc, synth
+
+
+@pytest.fixture(scope="module")
+def L():
+    return f3dc.lib()
+
+
+def test_exports_every_declared_symbol(L):
+    names = f3dc.declared_symbols()
+    assert len(names) >= 15
+    for n in names:
+        assert hasattr(L, n), n
+
+
+def test_weights_elems_matches_layout():
+    for name, shape in synth.SHAPES.items():
+        cfg = f3dc.config_for(shape)
+        _, total = synth.weight_offsets(shape)
+        assert f3dc.weights_elems(cfg) == total, name
+
+
+def test_time_schedule_matches_oracle(orc):
+    for eta, T in [(3.0, 25), (2.0, 25), (1.0, 8), (3.0, 50)]:
+        cfg = f3dc.config_for(synth.SHAPES["trellis_l"], steps=T, eta=eta)
+        np.testing.assert_array_equal(f3dc.time_schedule(cfg), orc.time_schedule(T, eta))
+
+
+@pytest.mark.parametrize("tau,mode", [(3, 0), (5, 0), (8, 0), (1, 0), (0, 0), (3, 1)])
+def test_pcsc_quota_matches_oracle(orc, tau, mode):
+    rng = np.random.default_rng(tau * 10 + mode)
+    shape = synth.SHAPES["trellis_l"]
+    for sigma in [0.0, 1.0, 6400.0, 65536.0, 2.6e5, 1e9] + list(rng.uniform(0, 3e5, 6)):
+        cfg = f3dc.config_for(shape, tau=tau, refresh_mode=mode)
+        consec = np.zeros(1, np.int32)
+        gate = orc.TauGate(tau, mode)
+        for k in range(1, 26):
+            q, ph = f3dc.pcsc_quota(cfg, sigma, k, consec)
+            oq, oph = orc.phase_quota(4096, 25, 0.2, 0.75, -0.07, 0.7, 3, 64, sigma, k)
+            assert (q, ph) == (gate(oq), oph), (sigma, k)
+
+
+def test_pcsc_quota_other_hyperparameters(orc):
+    shape = synth.SHAPES["scaled"]
+    for mu, xi, fc in [(-0.169, 0.8, 2), (-0.7, 0.9, 0), (-0.007, 0.7, 1)]:
+        cfg = f3dc.config_for(shape, mu=mu, xi=xi, f_corr=fc)
+        for k in range(1, 51):
+            q, ph = f3dc.pcsc_quota(cfg, 3.0e6, k)
+            assert (q, ph) == orc.phase_quota(32768, 50, 0.2, 0.75, mu, xi, fc, 64, 3.0e6, k)
+
+
+def test_invalid_arguments_are_reported(L):
+    cfg = f3dc.config_for(synth.SHAPES["trellis_l"])
+    with pytest.raises(f3dc.F3dcError) as e:
+        f3dc.pcsc_quota(cfg, 10.0, 0)
+    assert e.value.status == 1
+    with pytest.raises(f3dc.F3dcError) as e:
+        f3dc.pcsc_quota(cfg, float("nan"), 3)
+    assert e.value.status == 6
+    bad = f3dc.config_for(synth.SHAPES["trellis_l"], heads=7)
+    assert f3dc.weights_elems(bad) == 0
+    with pytest.raises(f3dc.F3dcError):
+        f3dc.time_schedule(bad)
+    bad = f3dc.config_for(synth.SHAPES["trellis_l"], channels=4)
+    assert f3dc.weights_elems(bad) == 0
+    # create rejects a bad config before touching any device
+    h = C.c_void_p()
+    st = L.f3dc_create(C.byref(bad), None, None, C.byref(h))
+    assert st == 1 and not h
+    assert b"channels" in L.f3dc_last_error(None)
