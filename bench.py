@@ -1,0 +1,464 @@
+"""Benchmark of the Fast3Dcache cached denoising step on GB300.
+
+Workload (the configuration the headline metric is quoted on): a
+TRELLIS-L-shaped sparse-structure flow transformer -- 16^3 x 8 latent (4096
+tokens), width 1024, 24 blocks, 16 heads, MLP 4x, cross-attention to 1374
+condition tokens of dim 1024, bf16 tensor-core arithmetic with fp32
+accumulation, 25 Euler steps with the three-phase PCSC schedule and the
+paper's default hyperparameters, batch 1 per GPU, random-init weights,
+seeded N(0,1) latents and condition tokens.  The anchor measurement sigma is
+fixed at 65536 dynamic voxels (25% of the 64^3 occupancy grid) so the active
+counts follow a TRELLIS-like budget; the stand-in decoder's own dynamic-voxel
+count is still computed at the anchor step in every sample.
+
+One benchmark step = one full sample (all 25 denoising steps: selection,
+transformer on the active tokens, merge + Euler, the anchor's voxel count).
+value = denoising steps per second over all GPUs.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl f3dc|reference]
+
+--impl reference times the CPU oracle (the plain C restatement of the
+paper) on the host cores instead, on a bounded sample of the same workload.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+from paper_2511_22533_gb300 import synth  # noqa: E402
+
+METRIC = "cached denoise steps/s at PCSC quota (1 GB300); tensor-pipe % of bf16 peak"
+UNIT = "steps/s"
+WORKLOAD = "trellis_l"
+SIGMA = 65536.0
+FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
+
+
+def parse():
+    p = argparse.ArgumentParser()
+    p.add_argument("--gpus", type=int, default=1)
+    p.add_argument("--steps", type=int, default=10)
+    p.add_argument("--warmup", type=int, default=3)
+    p.add_argument("--impl", default="f3dc", choices=["f3dc", "reference"])
+    return p.parse_args()
+
+
+def peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            d = json.load(f)
+        return d, "measured"
+    except Exception:
+        return FALLBACK_PEAKS, "fallback"
+
+
+# ------------------------------------------------------------------ work model
+
+def block_matmul_flops(a: int, W: int, Nc: int) -> float:
+    """Tensor-core FLOPs of one block on a active tokens (Supp. Sec. F terms
+    that are matrix products): QKV 6aW^2, out 2aW^2, CA-Q 2aW^2, CA-out
+    2aW^2, MLP 16aW^2, QK^T + PV 4a^2W, cross QK^T + PV 4aN_cW."""
+    return 28.0 * a * W * W + 4.0 * a * a * W + 4.0 * a * Nc * W
+
+
+def paper_block_flops(a: int, W: int, Nc: int, H: int, B: int = 1) -> float:
+    """The paper's per-block FLOPs count (Supp. Sec. F), N_tok = a."""
+    mod = 5 * B * W + 2 * B * W * 6 * W
+    ln = 7 * B * a * W
+    sa = 8 * B * a * W * W + 4 * B * a * a * W + 5 * B * H * a * a
+    ca = 4 * B * a * W * W + 4 * B * Nc * W * W + 4 * B * a * Nc * W + 5 * B * H * a * Nc
+    mlp = 16 * B * a * W * W + 20 * B * a * W
+    return mod + 3 * ln + sa + ca + mlp
+
+
+def sample_flops(quota_log, shape):
+    N, W, L, Nc, H = shape.tokens, shape.width, shape.blocks, shape.cond_tokens, shape.heads
+    mm = paper = 0.0
+    for c in quota_log[:, 0]:
+        a = N - int(c)
+        if a > 0:
+            mm += L * block_matmul_flops(a, W, Nc)
+            paper += L * paper_block_flops(a, W, Nc, H)
+    mm += L * 2.0 * Nc * (2 * W) * shape.cond_dim  # condition K / V, once per sample
+    return mm, paper
+
+
+# ------------------------------------------------------------------ ranks
+
+def rank_seed(rank: int) -> int:
+    """Each rank samples its own latents and condition (independent samples)."""
+    return 100 + rank
+
+
+def max_over_ranks(ms: float, world: int, device="cpu") -> float:
+    """The slowest rank's elapsed time (the whole job ends with it)."""
+    if world <= 1:
+        return ms
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([ms], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def whole_job_throughput(steps_per_sample: int, samples_per_rank: int, world: int, max_ms: float) -> float:
+    """Denoising steps per second over all ranks (weak scaling: every rank
+    runs its own samples)."""
+    return steps_per_sample * samples_per_rank * world / (max_ms / 1000.0)
+
+
+# ------------------------------------------------------------------ clocks
+
+class ClockSampler:
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.gpu = gpu_index
+        self.proc = None
+        self.path = None
+
+    def start(self):
+        fd, self.path = tempfile.mkstemp(suffix=".csv")
+        os.close(fd)
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.gpu), f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
+                 "-lms", "200"], stdout=open(self.path, "w"), stderr=subprocess.DEVNULL)
+        except Exception:
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"], "samples": 0}
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except Exception:
+            self.proc.kill()
+        sm, mx, reasons, n = [], [], set(), 0
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        with open(self.path) as f:
+            for line in f:
+                parts = [p.strip() for p in line.split(",")]
+                if len(parts) < 9:
+                    continue
+                try:
+                    sm.append(float(parts[1]))
+                    mx.append(float(parts[2]))
+                except ValueError:
+                    continue
+                n += 1
+                for name, v in zip(names, parts[5:9]):
+                    if v.lower().startswith("active"):
+                        reasons.add(name)
+        os.unlink(self.path)
+        loaded = [s for s in sm if mx and s > 0.5 * max(mx)] or sm
+        return {"sm_mhz": statistics.median(loaded) if loaded else None,
+                "sm_max_mhz": max(mx) if mx else None, "reasons": sorted(reasons), "samples": n}
+
+
+# ------------------------------------------------------------------ oracle leg
+
+def oracle_bounded_sample(orc, quota_log):
+    """Times the CPU oracle on a bounded sample of the workload and
+    extrapolates the whole 25-step sample: one transformer block (of 24) at
+    955 and at 2048 active tokens, the SSC score + selection and the merge /
+    Euler update at N = 4096, and the condition K / V of one block.  Block
+    time is interpolated linearly in FLOPs between the two measurements."""
+    shape = synth.SHAPES[WORKLOAD]
+    one = synth.ModelShape(shape.grid, shape.channels, shape.width, 1, shape.heads, shape.mlp_ratio,
+                           shape.cond_tokens, shape.cond_dim, shape.steps, shape.gamma_up)
+    blob = synth.weights_blob(one, 0)
+    m = orc.Model(one, blob)
+    cond = synth.cond_tokens(one, 1, 0)
+    S = synth.latents(one, 1, 0)[0]
+    hist = synth.velocity_history(shape.grid, 8, 1, seed=1)
+    t0 = time.perf_counter()
+    kv = m.cond_kv(cond[0])
+    t_kv = time.perf_counter() - t0
+    pts = []
+    for a in (955, 2048):
+        idx = np.arange(a, dtype=np.int32)
+        t0 = time.perf_counter()
+        m.forward(S, idx, 0.9, kv)
+        pts.append((block_matmul_flops(a, shape.width, shape.cond_tokens), time.perf_counter() - t0))
+    t0 = time.perf_counter()
+    s = orc.ssc_score(hist[2, 0], hist[1, 0], 0.7)
+    cached, idx = orc.select(s, 3141)
+    t_sel = time.perf_counter() - t0
+    va = np.zeros((len(idx), 8), np.float32)
+    t0 = time.perf_counter()
+    orc.merge_euler(S, idx, va, hist[2, 0], 0.01)
+    t_merge = time.perf_counter() - t0
+    (f0, s0), (f1, s1) = pts
+    slope = (s1 - s0) / (f1 - f0)
+    total = shape.blocks * t_kv
+    for c in quota_log[:, 0]:
+        a = shape.tokens - int(c)
+        if a > 0:
+            total += shape.blocks * max(s0 + slope * (block_matmul_flops(a, shape.width, shape.cond_tokens) - f0), 0.0)
+        if c > 0:
+            total += t_sel
+        total += t_merge
+    measured = t_kv + s0 + s1 + t_sel + t_merge
+    return shape.steps / total, measured
+
+
+def quota_log_host():
+    """The effective cache quotas of one benchmark sample (host-only logic
+    of the oracle: phases, PCSC with sigma = 65536, tau = 3)."""
+    import oracle
+    shape = synth.SHAPES[WORKLOAD]
+    gate = oracle.TauGate(3, 0)
+    q = []
+    for k in range(1, shape.steps + 1):
+        c, _ = oracle.phase_quota(shape.tokens, shape.steps, 0.2, 0.75, -0.07, 0.7, 3, shape.gamma_up, SIGMA, k)
+        q.append(gate(c))
+    return np.array(q, np.int32)[:, None]
+
+
+def run_reference(args):
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return 0
+    import oracle
+    oracle.build()
+    threads = os.cpu_count() or 1
+    os.environ.setdefault("OMP_NUM_THREADS", str(threads))
+    qlog = quota_log_host()
+    for _ in range(args.warmup):
+        oracle_bounded_sample(oracle, qlog)
+    vals, cpu_s = [], 0.0
+    for _ in range(args.steps):
+        v, meas = oracle_bounded_sample(oracle, qlog)
+        vals.append(v)
+        cpu_s += meas
+    value = statistics.median(vals)
+    sample = ("per step: 1 of 24 transformer blocks at 955 and 2048 active tokens, SSC score + selection "
+              "and merge/Euler at N=4096, condition K/V of one block; whole 25-step sample extrapolated "
+              "by FLOPs (blocks x interpolated block time over the PCSC quota schedule)")
+    line = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1000.0 * shape_steps() / value,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32",
+            "data": "synthetic", "config": config_block(args),
+            "cpu_baseline": {"value": value, "unit": UNIT, "cores": threads, "kind": "oracle", "sample": sample},
+            "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+            "cpu_seconds_measured": cpu_s}
+    print(json.dumps(line))
+    return 0
+
+
+def shape_steps():
+    return synth.SHAPES[WORKLOAD].steps
+
+
+def config_block(args):
+    shape = synth.SHAPES[WORKLOAD]
+    return {"workload": "TRELLIS-L-shaped sparse-structure flow DiT: 16^3x8 latent (4096 tokens), width 1024, "
+                        "24 blocks, 16 heads, MLP 4x, cross-attn to 1374 cond tokens dim 1024, bf16, 25 Euler "
+                        "steps, PCSC schedule (sigma 65536, mu -0.07, tau 3, xi 0.7, f_corr 3), batch 1 per GPU, "
+                        "random-init weights",
+            "tokens": shape.tokens, "width": shape.width, "blocks": shape.blocks, "heads": shape.heads,
+            "cond_tokens": shape.cond_tokens, "euler_steps": shape.steps, "batch_per_gpu": 1,
+            "global_batch": args.gpus, "sigma": SIGMA,
+            "l2": "inputs larger than L2: ~1.1 GB of weights streamed per denoising step",
+            "parallelism": f"replicas x{args.gpus} (independent samples per GPU)"}
+
+
+# ------------------------------------------------------------------ GPU arm
+
+def run_gpu(args):
+    import torch
+    import torch.distributed as dist
+
+    from paper_2511_22533_gb300 import f3dc
+
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    torch.cuda.set_device(local)
+    if world > 1:
+        os.environ.setdefault("MASTER_ADDR", "127.0.0.1")
+        dist.init_process_group("nccl", rank=rank, world_size=world)
+    if local == 0:
+        f3dc.lib()
+    if world > 1:
+        dist.barrier()
+    L = f3dc.lib()
+    shape = synth.SHAPES[WORKLOAD]
+    pk, pk_src = peaks()
+
+    blob = synth.weights_blob(shape, 0)
+    blob_d = torch.from_numpy(blob.view(np.int16)).cuda()
+    cfg = f3dc.config_for(shape, 1)
+    h = f3dc.Handle(cfg, blob_d)
+    del blob_d
+    noise = synth.latents(shape, 1, rank_seed(rank))
+    cond_np = synth.cond_tokens(shape, 1, rank_seed(rank))
+    noise_d = torch.from_numpy(noise).cuda()
+    cond_d = torch.from_numpy(cond_np.view(np.int16)).cuda()
+    S = torch.empty_like(noise_d)
+    sig = np.array([SIGMA])
+
+    def one_sample(quota_schedule=None, want_log=False):
+        S.copy_(noise_d)
+        return h.sample(S, cond_d, 1, sigma_override=sig, quota_schedule=quota_schedule, want_log=want_log)
+
+    # warm-up (the first also returns the quota log that defines the work)
+    qlog, sigma_meas = one_sample(want_log=True)
+    for _ in range(max(args.warmup - 1, 0)):
+        one_sample()
+    torch.cuda.synchronize()
+    assert h.device_status() == 0
+    mm_flops, paper_flops = sample_flops(qlog, shape)
+
+    def timed(n, fn):
+        if world > 1:
+            dist.barrier()
+        torch.cuda.synchronize()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record()
+        for _ in range(n):
+            fn()
+        e1.record()
+        torch.cuda.synchronize()
+        if world > 1:
+            dist.barrier()
+        return max_over_ranks(e0.elapsed_time(e1), world, device="cuda")
+
+    # ---- headline: cached sampler, device-resident inputs
+    n0 = h.launch_count()
+    clocks = ClockSampler(local)
+    clocks.start()
+    ms = timed(args.steps, one_sample)
+    clk = clocks.stop()
+    launches = h.launch_count() - n0
+    ms_per_sample = ms / args.steps
+    value = whole_job_throughput(shape.steps, args.steps, world, ms)
+
+    # ---- uncached comparison: the same kernels with quota 0 at every step
+    zeros = np.zeros((shape.steps, 1), np.int32)
+    one_sample(zeros)
+    n_unc = max(2, args.steps // 2)
+    ms_unc = timed(n_unc, lambda: one_sample(zeros)) / n_unc
+    zlog = zeros
+    mm_unc, _ = sample_flops(zlog, shape)
+
+    # ---- per-kernel CUDA-event timing of the same workload
+    h.profile(True)
+    n_prof = max(2, args.steps // 4)
+    for _ in range(n_prof):
+        one_sample()
+    stats = h.profile_read()
+    h.profile(False)
+
+    # ---- end to end through the public API with host buffers
+    import torch as _t
+    noise_h = _t.from_numpy(noise).pin_memory()
+    cond_h = _t.from_numpy(cond_np.view(np.int16)).pin_memory()
+    out_h = _t.empty_like(noise_h).pin_memory()
+    cond_e = _t.empty_like(cond_d)
+
+    def e2e_sample():
+        S.copy_(noise_h, non_blocking=True)
+        cond_e.copy_(cond_h, non_blocking=True)
+        h.sample(S, cond_e, 1, sigma_override=sig, want_log=False)
+        out_h.copy_(S, non_blocking=True)
+
+    e2e_sample()
+    ms_e2e = timed(args.steps, e2e_sample)
+    e2e_value = whole_job_throughput(shape.steps, args.steps, world, ms_e2e)
+    assert h.device_status() == 0
+
+    # ---- CPU baseline (oracle on the host cores), rank 0 at N = 1 only
+    cpu = None
+    if world == 1 and rank == 0:
+        import oracle
+        oracle.build()
+        v, meas = oracle_bounded_sample(oracle, qlog)
+        cpu = {"value": v, "unit": UNIT, "cores": os.cpu_count(), "kind": "oracle",
+               "sample": f"1 of 24 blocks at 955 and 2048 active tokens + SSC/selection + merge at N=4096 "
+                         f"({meas:.1f} s of CPU wall time), whole 25-step sample extrapolated by FLOPs"}
+
+    if rank != 0:
+        h.close()
+        if world > 1:
+            dist.destroy_process_group()
+        return 0
+
+    tensor_tflops = mm_flops / (ms_per_sample / 1000.0) / 1e12
+    fam = {s["name"]: s for s in stats}
+    dom = max(stats, key=lambda s: s["total_ms"])
+    if dom["flops"] > 0:
+        peak = pk["bf16_tflops_sustained"]
+        achieved = dom["flops"] / (dom["total_ms"] / 1000.0) / 1e12
+        roof = {"kernel": dom["name"], "bound": "tensor", "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
+                "frac": achieved / peak, "traffic": None, "peak_source": f"bf16_tflops_sustained ({pk_src})"}
+    else:
+        peak = pk["hbm_gbs"]
+        achieved = dom["bytes"] / (dom["total_ms"] / 1000.0) / 1e9
+        roof = {"kernel": dom["name"], "bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
+                "frac": achieved / peak, "traffic": None, "peak_source": f"hbm_gbs ({pk_src})"}
+    kernels = {}
+    for s in stats:
+        per = s["total_ms"] / n_prof
+        entry = {"launches_per_sample": s["launches"] / n_prof, "ms_per_sample": per}
+        if s["flops"] > 0:
+            entry["tflops"] = s["flops"] / (s["total_ms"] / 1000.0) / 1e12
+            entry["frac_bf16_sustained"] = entry["tflops"] / pk["bf16_tflops_sustained"]
+        if s["bytes"] > 0:
+            entry["gbs"] = s["bytes"] / (s["total_ms"] / 1000.0) / 1e9
+            entry["frac_hbm"] = entry["gbs"] / pk["hbm_gbs"]
+        kernels[s["name"]] = entry
+
+    line = {
+        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": ms_per_sample, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "bf16", "data": "synthetic", "config": config_block(args),
+        "samples_per_s": args.steps * world / (ms / 1000.0),
+        "tensor_pct_of_bf16_sustained": 100.0 * tensor_tflops / pk["bf16_tflops_sustained"],
+        "tensor_tflops_per_gpu": tensor_tflops,
+        "paper_flops_per_sample_T": paper_flops / 1e12,
+        "uncached": {"ms_per_sample": ms_unc, "steps_per_s": shape.steps * world / (ms_unc / 1000.0),
+                     "speedup_cached_vs_uncached": ms_unc / ms_per_sample,
+                     "tensor_tflops_per_gpu": mm_unc / (ms_unc / 1000.0) / 1e12},
+        "active_tokens_per_step": [shape.tokens - int(c) for c in qlog[:, 0]],
+        "sigma_measured_by_stand_in_decoder": float(sigma_meas[0]),
+        "roofline": roof, "kernels": kernels,
+        "cpu_baseline": cpu,
+        "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": int(noise.nbytes + cond_np.nbytes),
+                "d2h_bytes_per_step": int(noise.nbytes)},
+        "gpu_launches": int(launches),
+        "clocks": clk,
+    }
+    print(json.dumps(line))
+    h.close()
+    if world > 1:
+        dist.destroy_process_group()
+    return 0
+
+
+def main():
+    args = parse()
+    if args.impl == "reference":
+        return run_reference(args)
+    return run_gpu(args)
+
+
+if __name__ == "__main__":
+    sys.exit(main())

@@ -70,9 +70,9 @@ typedef enum f3dc_status {
 #define F3DC_REFRESH_LITERAL 1
 
 typedef struct f3dc_config {
-    int32_t grid;        /* cubic latent grid side D; N = D^3 tokens (N % 128 == 0) */
+    int32_t grid;        /* cubic latent grid side D; N = D^3 tokens (N % 32 == 0) */
     int32_t channels;    /* latent channels C; must be 8 */
-    int32_t width;       /* transformer width W (multiple of 256) */
+    int32_t width;       /* transformer width W (multiple of 128, <= 2048) */
     int32_t blocks;      /* transformer blocks L */
     int32_t heads;       /* attention heads H; W / H must be 32 or 64 */
     int32_t mlp_ratio;   /* MLP hidden = mlp_ratio * W; must be 4 */
@@ -214,6 +214,34 @@ f3dc_status f3dc_step(f3dc_handle *h, int32_t k, int32_t B, float *S_inout, void
 f3dc_status f3dc_sample(f3dc_handle *h, float *S_inout, const void *cond, int32_t B,
                         const double *sigma_override, const int32_t *quota_schedule,
                         int32_t *quota_log, double *sigma_out, void *stream);
+
+/* ---------------------------------------------------------------------- */
+/* Measurement support.                                                    */
+/* ---------------------------------------------------------------------- */
+
+/* Per-kernel-family totals collected while profiling is on. */
+typedef struct f3dc_kernel_stats {
+    char name[24];     /* kernel family, e.g. "gemm", "attn_self", "ssc_select" */
+    int64_t launches;  /* launches recorded */
+    double total_ms;   /* summed CUDA-event durations on the launching stream */
+    double flops;      /* algorithmic floating-point work of those launches */
+    double bytes;      /* algorithmic DRAM bytes of those launches */
+} f3dc_kernel_stats;
+
+/* Turns per-launch timing on (enable != 0) or off, clearing the totals.
+ * While on, every kernel launch is bracketed by CUDA events on its stream
+ * and each f3dc_step synchronizes its stream once at the end to read them;
+ * the algorithmic work of a launch is derived from the step's active-token
+ * counts (GEMM 2 M N K with M the active tokens; attention 4 W sum a_b^2 and
+ * 4 W M N_c; row kernels their read + write bytes). */
+f3dc_status f3dc_profile(f3dc_handle *h, int32_t enable);
+
+/* Copies up to `capacity` family totals into out (host) and sets *count.
+ * Synchronizes the handle's last stream. */
+f3dc_status f3dc_profile_read(f3dc_handle *h, f3dc_kernel_stats *out, int32_t capacity, int32_t *count);
+
+/* Number of kernels this handle has launched since it was created. */
+f3dc_status f3dc_launch_count(const f3dc_handle *h, int64_t *count);
 
 /* ---------------------------------------------------------------------- */
 /* Diagnostic entry points (kernel-level parity checks).                   */

@@ -176,6 +176,61 @@ std::vector<float> position_table(int grid, int W)
     return pos;
 }
 
+// ---------------------------------------------------------------- profiling
+enum KernelFamily {
+    KF_SELECT, KF_GATHER, KF_LN, KF_GEMM, KF_ATTN_SELF, KF_ATTN_CROSS, KF_FINAL, KF_MERGE, KF_TEMB, KF_GEMM_COND,
+    KF_PLAN, KF_SCATTER, KF_COUNT
+};
+const char *const kFamilyName[KF_COUNT] = {"ssc_select", "gather_embed", "layernorm",  "gemm",
+                                           "attn_self",  "attn_cross",   "final_layer", "merge_euler",
+                                           "temb_gemv",  "gemm_cond",    "plan",        "scatter"};
+
+// Algorithmic work of one launch as a function of the step's plan:
+//   c_m * M + c_sq * sum_b a_b^2 + c_tok * B N + c_sel * (tokens of samples
+//   that ran the selection) + c_fix, in flops or in DRAM bytes.
+struct Work {
+    double c_m = 0, c_sq = 0, c_tok = 0, c_sel = 0, c_fix = 0;
+    bool flops = false;
+};
+Work wm(double c, bool flops = false)
+{
+    Work w;
+    w.c_m = c;
+    w.flops = flops;
+    return w;
+}
+Work wfix(double c, bool flops = false)
+{
+    Work w;
+    w.c_fix = c;
+    w.flops = flops;
+    return w;
+}
+
+struct ProfRecord {
+    int fam;
+    cudaEvent_t e0, e1;
+    Work w;
+};
+
+struct Profiler {
+    bool on = false;
+    std::vector<cudaEvent_t> pool;
+    size_t next = 0;
+    std::vector<ProfRecord> pending;
+    int64_t launches[KF_COUNT] = {};
+    double ms[KF_COUNT] = {}, flops[KF_COUNT] = {}, bytes[KF_COUNT] = {};
+    void reset()
+    {
+        for (int i = 0; i < KF_COUNT; ++i) {
+            launches[i] = 0;
+            ms[i] = flops[i] = bytes[i] = 0.0;
+        }
+        pending.clear();
+        next = 0;
+    }
+};
+
 }  // namespace
 
 struct f3dc_handle {
@@ -207,6 +262,10 @@ struct f3dc_handle {
     cudaEvent_t quota_done[2] = {nullptr, nullptr};
     unsigned calls = 0;
 
+    Profiler prof;
+    int64_t launches = 0;
+    int last_B = 0;
+
     CUtensorMap tm_h, tm_att, tm_u, tm_cond, tm_q_self, tm_q_cross;
     std::vector<CUtensorMap> tm_qkv_w, tm_o_w, tm_cq_w, tm_co_w, tm_fc1_w, tm_fc2_w, tm_ckv_w, tm_kv_cross;
     int bn_qkv = 128, bn_w = 128, bn_fc1 = 128, bn_ckv = 128;
@@ -229,6 +288,74 @@ f3dc_status fail(f3dc_handle *h, f3dc_status st, const std::string &msg)
         if (e_ != cudaSuccess)                                                                     \
             return fail(h, F3DC_ERR_CUDA, std::string(#expr) + ": " + cudaGetErrorString(e_));     \
     } while (0)
+
+cudaEvent_t prof_event(f3dc_handle *h)
+{
+    Profiler &P = h->prof;
+    if (P.next == P.pool.size()) {
+        cudaEvent_t e = nullptr;
+        if (cudaEventCreate(&e) != cudaSuccess) return nullptr;
+        P.pool.push_back(e);
+    }
+    return P.pool[P.next++];
+}
+
+cudaEvent_t prof_begin(f3dc_handle *h, cudaStream_t s)
+{
+    if (!h->prof.on) return nullptr;
+    cudaEvent_t e = prof_event(h);
+    if (e) cudaEventRecord(e, s);
+    return e;
+}
+
+void prof_end(f3dc_handle *h, cudaStream_t s, int fam, const Work &w, cudaEvent_t e0)
+{
+    h->launches++;
+    if (!h->prof.on || !e0) return;
+    cudaEvent_t e1 = prof_event(h);
+    if (!e1) return;
+    cudaEventRecord(e1, s);
+    h->prof.pending.push_back(ProfRecord{fam, e0, e1, w});
+}
+
+// Launches one kernel through `expr`, bracketed by profiling events.
+#define LAUNCH(fam, work, expr)                                                                    \
+    do {                                                                                           \
+        cudaEvent_t e0_ = prof_begin(h, s);                                                        \
+        CK(expr);                                                                                  \
+        prof_end(h, s, (fam), (work), e0_);                                                        \
+    } while (0)
+
+// Reads the pending event pairs of the last step(s); the plan on the device
+// gives the active-token counts that turn each launch's Work into numbers.
+f3dc_status prof_drain(f3dc_handle *h, cudaStream_t s)
+{
+    Profiler &P = h->prof;
+    if (P.pending.empty()) return F3DC_OK;
+    CK(cudaStreamSynchronize(s));
+    Plan plan;
+    CK(cudaMemcpy(&plan, h->plan, sizeof(Plan), cudaMemcpyDeviceToHost));
+    const int B = h->last_B > 0 ? h->last_B : 1;
+    double M = 0, sq = 0, sel = 0;
+    for (int b = 0; b < B; ++b) {
+        const double a = plan.n_active[b];
+        M += a;
+        sq += a * a;
+        if (a > 0 && a < h->N) sel += h->N;
+    }
+    const double tok = (double)B * h->N;
+    for (const ProfRecord &r : P.pending) {
+        float ms = 0.f;
+        CK(cudaEventElapsedTime(&ms, r.e0, r.e1));
+        const double v = r.w.c_m * M + r.w.c_sq * sq + r.w.c_tok * tok + r.w.c_sel * sel + r.w.c_fix;
+        P.launches[r.fam] += 1;
+        P.ms[r.fam] += ms;
+        (r.w.flops ? P.flops : P.bytes)[r.fam] += v;
+    }
+    P.pending.clear();
+    P.next = 0;
+    return F3DC_OK;
+}
 
 template <typename T>
 cudaError_t dalloc(T **p, size_t count)
@@ -295,45 +422,61 @@ cudaError_t run_attention(f3dc_handle *h, int mode, const CUtensorMap &tq, const
 // h->tile_sample and h->active_idx (Sec. 4.2; Supp. Sec. F).
 f3dc_status run_dit(f3dc_handle *h, float t, const float *S, cudaStream_t s)
 {
-    const int W = h->W, L = h->L;
+    const int W = h->W, L = h->L, Wm = h->Wm;
+    const double dW = W, dWm = Wm;
     const Layout &ly = h->lay;
-    // timestep embedding and every block's modulation (adaLN)
-    CK(launch_time_freq(t, h->freq, s));
-    CK(launch_gemv(h->freq, 256, h->wt(ly.t_w1), h->wt(ly.t_b1), h->h1, W, 0, 1, h->num_sms, s));
-    CK(launch_gemv(h->h1, W, h->wt(ly.t_w2), h->wt(ly.t_b2), h->temb, W, 0, 0, h->num_sms, s));
-    CK(launch_gemv(h->temb, W, h->mod_w, h->mod_b, h->mod, h->mod_rows, 1, 0, h->num_sms, s));
-    // gather + embed the active tokens
-    CK(launch_gather_embed(S, h->N, W, h->active_idx, h->plan, h->tile_sample, h->wt(ly.in_w), h->wt(ly.in_b),
-                           h->pos, h->x, h->max_rows, h->num_sms, h->dev_err, s));
+    // timestep embedding and every block's modulation (adaLN): three GEMVs
+    // streaming the embedding and the repacked [L*6W + 2W, W] weights
+    const Work w_temb = wfix(2.0 * ((double)h->mod_rows * W + 256.0 * W + dW * W));
+    LAUNCH(KF_TEMB, Work(), launch_time_freq(t, h->freq, s));
+    LAUNCH(KF_TEMB, Work(), launch_gemv(h->freq, 256, h->wt(ly.t_w1), h->wt(ly.t_b1), h->h1, W, 0, 1, h->num_sms, s));
+    LAUNCH(KF_TEMB, Work(), launch_gemv(h->h1, W, h->wt(ly.t_w2), h->wt(ly.t_b2), h->temb, W, 0, 0, h->num_sms, s));
+    LAUNCH(KF_TEMB, w_temb, launch_gemv(h->temb, W, h->mod_w, h->mod_b, h->mod, h->mod_rows, 1, 0, h->num_sms, s));
+    // gather + embed the active tokens: 32 B latent + 4 B index in, 4W B out
+    LAUNCH(KF_GATHER, wm(36.0 + 4.0 * dW),
+           launch_gather_embed(S, h->N, W, h->active_idx, h->plan, h->tile_sample, h->wt(ly.in_w), h->wt(ly.in_b),
+                               h->pos, h->x, h->max_rows, h->num_sms, h->dev_err, s));
+    const Work w_ln = wm(6.0 * dW);  // fp32 row in, bf16 row out
+    Work w_self;
+    w_self.c_sq = 4.0 * dW;          // Q K^T and P V among each sample's active tokens
+    w_self.flops = true;
+    const Work w_cross = wm(4.0 * dW * h->Nc, true);
     for (int l = 0; l < L; ++l) {
         const BlockOffsets &b = ly.blk[l];
         const float *m = h->mod + (size_t)l * 6 * W;
         // self-attention among the active tokens
-        CK(launch_layernorm(h->x, W, h->plan, 0, m, m + W, nullptr, nullptr, h->h, h->max_rows, h->num_sms, s));
-        CK(run_gemm(h, h->tm_h, h->tm_qkv_w[l], 3 * W, W, h->bn_qkv, kEpiQKNorm, h->qkv, 3 * W, h->wt(b.qkv_b),
-                    nullptr, h->wt(b.qn_g), h->wt(b.kn_g), s));
-        CK(run_attention(h, 0, h->tm_q_self, h->tm_q_self, 0, W, 2 * W, s));
-        CK(run_gemm(h, h->tm_att, h->tm_o_w[l], W, W, h->bn_w, kEpiResid, h->x, W, h->wt(b.o_b), m + 2 * W,
-                    nullptr, nullptr, s));
+        LAUNCH(KF_LN, w_ln, launch_layernorm(h->x, W, h->plan, 0, m, m + W, nullptr, nullptr, h->h, h->max_rows,
+                                             h->num_sms, s));
+        LAUNCH(KF_GEMM, wm(2.0 * 3 * dW * dW, true),
+               run_gemm(h, h->tm_h, h->tm_qkv_w[l], 3 * W, W, h->bn_qkv, kEpiQKNorm, h->qkv, 3 * W, h->wt(b.qkv_b),
+                        nullptr, h->wt(b.qn_g), h->wt(b.kn_g), s));
+        LAUNCH(KF_ATTN_SELF, w_self, run_attention(h, 0, h->tm_q_self, h->tm_q_self, 0, W, 2 * W, s));
+        LAUNCH(KF_GEMM, wm(2.0 * dW * dW, true),
+               run_gemm(h, h->tm_att, h->tm_o_w[l], W, W, h->bn_w, kEpiResid, h->x, W, h->wt(b.o_b), m + 2 * W,
+                        nullptr, nullptr, s));
         // cross-attention to the condition
-        CK(launch_layernorm(h->x, W, h->plan, 1, nullptr, nullptr, h->wt(b.ln2_g), h->wt(b.ln2_b), h->h,
-                            h->max_rows, h->num_sms, s));
-        CK(run_gemm(h, h->tm_h, h->tm_cq_w[l], W, W, h->bn_w, kEpiBias, h->qc, W, h->wt(b.cq_b), nullptr,
-                    nullptr, nullptr, s));
-        CK(run_attention(h, 1, h->tm_q_cross, h->tm_kv_cross[l], 0, 0, W, s));
-        CK(run_gemm(h, h->tm_att, h->tm_co_w[l], W, W, h->bn_w, kEpiResid, h->x, W, h->wt(b.co_b), nullptr,
-                    nullptr, nullptr, s));
+        LAUNCH(KF_LN, w_ln, launch_layernorm(h->x, W, h->plan, 1, nullptr, nullptr, h->wt(b.ln2_g), h->wt(b.ln2_b),
+                                             h->h, h->max_rows, h->num_sms, s));
+        LAUNCH(KF_GEMM, wm(2.0 * dW * dW, true),
+               run_gemm(h, h->tm_h, h->tm_cq_w[l], W, W, h->bn_w, kEpiBias, h->qc, W, h->wt(b.cq_b), nullptr,
+                        nullptr, nullptr, s));
+        LAUNCH(KF_ATTN_CROSS, w_cross, run_attention(h, 1, h->tm_q_cross, h->tm_kv_cross[l], 0, 0, W, s));
+        LAUNCH(KF_GEMM, wm(2.0 * dW * dW, true),
+               run_gemm(h, h->tm_att, h->tm_co_w[l], W, W, h->bn_w, kEpiResid, h->x, W, h->wt(b.co_b), nullptr,
+                        nullptr, nullptr, s));
         // MLP
-        CK(launch_layernorm(h->x, W, h->plan, 0, m + 3 * W, m + 4 * W, nullptr, nullptr, h->h, h->max_rows,
-                            h->num_sms, s));
-        CK(run_gemm(h, h->tm_h, h->tm_fc1_w[l], h->Wm, W, h->bn_fc1, kEpiGelu, h->u, h->Wm, h->wt(b.fc1_b),
-                    nullptr, nullptr, nullptr, s));
-        CK(run_gemm(h, h->tm_u, h->tm_fc2_w[l], W, h->Wm, h->bn_w, kEpiResid, h->x, W, h->wt(b.fc2_b), m + 5 * W,
-                    nullptr, nullptr, s));
+        LAUNCH(KF_LN, w_ln, launch_layernorm(h->x, W, h->plan, 0, m + 3 * W, m + 4 * W, nullptr, nullptr, h->h,
+                                             h->max_rows, h->num_sms, s));
+        LAUNCH(KF_GEMM, wm(2.0 * dWm * dW, true),
+               run_gemm(h, h->tm_h, h->tm_fc1_w[l], Wm, W, h->bn_fc1, kEpiGelu, h->u, Wm, h->wt(b.fc1_b), nullptr,
+                        nullptr, nullptr, s));
+        LAUNCH(KF_GEMM, wm(2.0 * dW * dWm, true),
+               run_gemm(h, h->tm_u, h->tm_fc2_w[l], W, Wm, h->bn_w, kEpiResid, h->x, W, h->wt(b.fc2_b), m + 5 * W,
+                        nullptr, nullptr, s));
     }
     const float *fm = h->mod + (size_t)L * 6 * W;
-    CK(launch_final_layer(h->x, W, h->plan, fm, fm + W, h->wt(ly.out_w), h->wt(ly.out_b), h->v_active,
-                          h->max_rows, h->num_sms, s));
+    LAUNCH(KF_FINAL, wm(4.0 * dW + 32.0), launch_final_layer(h->x, W, h->plan, fm, fm + W, h->wt(ly.out_w),
+                                                             h->wt(ly.out_b), h->v_active, h->max_rows, h->num_sms, s));
     return F3DC_OK;
 }
 
@@ -380,6 +523,7 @@ void free_handle(f3dc_handle *h)
     if (h->h_quota) cudaFreeHost(h->h_quota);
     for (cudaEvent_t ev : h->quota_done)
         if (ev) cudaEventDestroy(ev);
+    for (cudaEvent_t ev : h->prof.pool) cudaEventDestroy(ev);
     delete h;
 }
 
@@ -624,7 +768,7 @@ f3dc_status f3dc_ssc_select(f3dc_handle *h, const void *v_prev1, const void *v_p
     a.n_active = n_active_out;
     a.mask = cached_mask_out;
     a.err = h->dev_err;
-    CK(launch_ssc_select(a, s));
+    LAUNCH(KF_SELECT, Work(), launch_ssc_select(a, s));
     return F3DC_OK;
 }
 
@@ -651,8 +795,9 @@ f3dc_status f3dc_set_cond(f3dc_handle *h, const void *cond, int32_t B, void *str
         p.bias = h->wt(h->lay.blk[l].ckv_b);
         p.err = h->dev_err;
         const int tiles = p.m_tiles * (p.N / h->bn_ckv);
-        CK(launch_gemm(&h->tm_cond, &h->tm_ckv_w[l], p, kEpiBias, h->bn_ckv, tiles < h->num_sms ? tiles : h->num_sms,
-                       s));
+        LAUNCH(KF_GEMM_COND, wfix(2.0 * rows * p.N * (double)p.K, true),
+               launch_gemm(&h->tm_cond, &h->tm_ckv_w[l], p, kEpiBias, h->bn_ckv,
+                           tiles < h->num_sms ? tiles : h->num_sms, s));
     }
     h->cond_B = B;
     return F3DC_OK;
@@ -691,7 +836,11 @@ f3dc_status f3dc_step(f3dc_handle *h, int32_t k, int32_t B, float *S_inout, void
     a.plan = h->plan;
     a.tile_sample = h->tile_sample;
     a.err = h->dev_err;
-    CK(launch_ssc_select(a, s));
+    h->last_B = B;
+    Work w_sel;
+    w_sel.c_sel = 33.0;  // two bf16 history slots (32 B) and the mask byte per token
+    w_sel.c_m = 4.0;     // one index per active token
+    LAUNCH(KF_SELECT, w_sel, launch_ssc_select(a, s));
 
     // FlowTransformer on the active tokens at t_k
     std::vector<float> t(h->T + 1);
@@ -715,7 +864,11 @@ f3dc_status f3dc_step(f3dc_handle *h, int32_t k, int32_t B, float *S_inout, void
     m.dyn = dyn_voxels_dev;
     m.max_rows = h->max_rows;
     m.err = h->dev_err;
-    CK(launch_merge_euler(m, s));
+    Work w_merge;
+    w_merge.c_tok = 96.0;  // S in/out (32 + 32 B), cached velocity in, v_t out (16 + 16 B)
+    w_merge.c_m = 32.0;    // fresh fp32 velocity of each active token
+    LAUNCH(KF_MERGE, w_merge, launch_merge_euler(m, s));
+    if (h->prof.on) return prof_drain(h, s);
     return F3DC_OK;
 }
 
@@ -791,10 +944,52 @@ f3dc_status f3dc_forward(f3dc_handle *h, float t, int32_t B, const float *S, con
     cudaStream_t s = (cudaStream_t)stream;
     h->last_stream = s;
     CK(cudaMemcpyAsync(h->active_idx, active_idx, (size_t)B * h->N * sizeof(int32_t), cudaMemcpyDeviceToDevice, s));
-    CK(launch_plan_from_counts(n_active, h->active_idx, B, h->N, h->plan, h->tile_sample, nullptr, h->dev_err, s));
+    h->last_B = B;
+    LAUNCH(KF_PLAN, Work(), launch_plan_from_counts(n_active, h->active_idx, B, h->N, h->plan, h->tile_sample,
+                                                    nullptr, h->dev_err, s));
     f3dc_status st = run_dit(h, t, S, s);
     if (st != F3DC_OK) return st;
-    CK(launch_scatter_rows(h->v_active, h->plan, B, h->N, v_out, s));
+    LAUNCH(KF_SCATTER, wm(64.0), launch_scatter_rows(h->v_active, h->plan, B, h->N, v_out, s));
+    if (h->prof.on) return prof_drain(h, s);
+    return F3DC_OK;
+}
+
+f3dc_status f3dc_profile(f3dc_handle *h, int32_t enable)
+{
+    if (!h) return fail(nullptr, F3DC_ERR_INVALID_ARG, "null handle");
+    CK(cudaStreamSynchronize(h->last_stream));
+    h->prof.reset();
+    h->prof.on = enable != 0;
+    return F3DC_OK;
+}
+
+f3dc_status f3dc_profile_read(f3dc_handle *h, f3dc_kernel_stats *out, int32_t capacity, int32_t *count)
+{
+    if (!h || !count || (capacity > 0 && !out)) return fail(h, F3DC_ERR_INVALID_ARG, "null argument");
+    f3dc_status st = prof_drain(h, h->last_stream);
+    if (st != F3DC_OK) return st;
+    int n = 0;
+    for (int f = 0; f < KF_COUNT; ++f) {
+        if (h->prof.launches[f] == 0) continue;
+        if (n < capacity) {
+            f3dc_kernel_stats &o = out[n];
+            memset(&o, 0, sizeof(o));
+            strncpy(o.name, kFamilyName[f], sizeof(o.name) - 1);
+            o.launches = h->prof.launches[f];
+            o.total_ms = h->prof.ms[f];
+            o.flops = h->prof.flops[f];
+            o.bytes = h->prof.bytes[f];
+        }
+        ++n;
+    }
+    *count = n;
+    return F3DC_OK;
+}
+
+f3dc_status f3dc_launch_count(const f3dc_handle *h, int64_t *count)
+{
+    if (!h || !count) return fail(nullptr, F3DC_ERR_INVALID_ARG, "null argument");
+    *count = h->launches;
     return F3DC_OK;
 }
 

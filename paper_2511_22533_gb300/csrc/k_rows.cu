@@ -291,13 +291,13 @@ __global__ void __launch_bounds__(kGemvThreads) k_gemv(const float *x, int K, co
     for (int k = threadIdx.x; k < K; k += blockDim.x) xs[k] = silu_in ? silu(x[k]) : x[k];
     __syncthreads();
     const int lane = threadIdx.x & 31, wpb = blockDim.x >> 5;
-    const int chunks = K / 256;  // 8 bf16 per lane per chunk
+    const int chunks = K / 8;  // 8 bf16 (one uint4) per lane per step
     const uint4 *W4 = reinterpret_cast<const uint4 *>(w);
     for (int r = (blockIdx.x * wpb + (threadIdx.x >> 5)) * 2; r < rows; r += gridDim.x * wpb * 2) {
         const bool two = r + 1 < rows;
         float acc0 = 0.f, acc1 = 0.f;
-        for (int q = 0; q < chunks; ++q) {
-            const int k0 = (q * 32 + lane) * 8;
+        for (int q = lane; q < chunks; q += 32) {
+            const int k0 = q * 8;
             const uint4 u0 = __ldg(W4 + ((size_t)r * K + k0) / 8);
             const uint4 u1 = two ? __ldg(W4 + ((size_t)(r + 1) * K + k0) / 8) : make_uint4(0, 0, 0, 0);
             float f0[8], f1[8];
@@ -400,7 +400,7 @@ cudaError_t launch_time_freq(float t, float *freq, cudaStream_t s)
 cudaError_t launch_gemv(const float *x, int K, const bf16 *w, const bf16 *b, float *y, int rows, int silu_in,
                         int silu_out, int num_sms, cudaStream_t s)
 {
-    if (K % 256 != 0 || K > kGemvMaxK) return cudaErrorInvalidValue;
+    if (K % 8 != 0 || K > kGemvMaxK) return cudaErrorInvalidValue;
     const int wpb = kGemvThreads / 32;
     int grid = (rows + 2 * wpb - 1) / (2 * wpb);
     if (grid > num_sms * 4) grid = num_sms * 4;

@@ -39,6 +39,11 @@ class Config(C.Structure):
                 ("omega", C.c_double), ("xi", C.c_double), ("rho_cfg_off", C.c_double)]
 
 
+class KernelStats(C.Structure):
+    _fields_ = [("name", C.c_char * 24), ("launches", C.c_int64), ("total_ms", C.c_double),
+                ("flops", C.c_double), ("bytes", C.c_double)]
+
+
 class Weights(C.Structure):
     _fields_ = [("layout_version", C.c_int32), ("blob", C.c_void_p), ("blob_elems", C.c_size_t)]
 
@@ -77,6 +82,9 @@ def lib():
                 "f3dc_step": ([_vp, C.c_int32, C.c_int32, _vp, _vp, _vp, _vp, _vp], C.c_int),
                 "f3dc_sample": ([_vp, _vp, _vp, C.c_int32, _f64p, _i32p, _i32p, _f64p, _vp], C.c_int),
                 "f3dc_forward": ([_vp, C.c_float, C.c_int32, _vp, _vp, _vp, _vp, _vp], C.c_int),
+                "f3dc_profile": ([_vp, C.c_int32], C.c_int),
+                "f3dc_profile_read": ([_vp, C.POINTER(KernelStats), C.c_int32, _i32p], C.c_int),
+                "f3dc_launch_count": ([_vp, C.POINTER(C.c_int64)], C.c_int),
                 "f3dc_gemm": ([_vp, _vp, _vp, _vp, _vp, C.c_int32, C.c_int32, C.c_int32, C.c_int32, _vp], C.c_int),
                 "f3dc_attention": ([_vp, C.c_int32, _vp, _vp, C.c_int32, _vp, C.c_int32, C.c_int32, C.c_int32,
                                     C.c_int32, _vp], C.c_int),
@@ -212,6 +220,21 @@ class Handle:
         self._ck(lib().f3dc_sample(self.h, _ptr(S), _ptr(cond), B, _np_ptr(so, _f64p), _np_ptr(qs, _i32p),
                                    _np_ptr(ql, _i32p), _np_ptr(sg, _f64p), _stream(stream)))
         return ql, sg
+
+    def profile(self, enable: bool):
+        self._ck(lib().f3dc_profile(self.h, 1 if enable else 0))
+
+    def profile_read(self):
+        arr = (KernelStats * 32)()
+        n = C.c_int32(0)
+        self._ck(lib().f3dc_profile_read(self.h, arr, 32, C.byref(n)))
+        return [{"name": arr[i].name.decode(), "launches": arr[i].launches, "total_ms": arr[i].total_ms,
+                 "flops": arr[i].flops, "bytes": arr[i].bytes} for i in range(min(n.value, 32))]
+
+    def launch_count(self) -> int:
+        n = C.c_int64(0)
+        self._ck(lib().f3dc_launch_count(self.h, C.byref(n)))
+        return n.value
 
     def forward(self, t, B, S, active_idx, n_active, v_out, stream=None):
         self._ck(lib().f3dc_forward(self.h, float(t), B, _ptr(S), _ptr(active_idx), _ptr(n_active), _ptr(v_out),

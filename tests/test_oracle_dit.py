@@ -146,3 +146,33 @@ def test_sample_pcsc_anchor_and_log(tiny, orc):
     assert ov["sigma"][0] == out["sigma"][0]
     c6, _ = orc.phase_quota(TINY.tokens, T, 0.2, 0.75, -0.07, 0.7, 3, TINY.gamma_up, 6400.0, ka + 1)
     assert ov["quota"][ka, 0] == c6
+
+
+def test_time_embedding_closed_form_at_t0(orc):
+    # at t = 0 every frequency has argument 0: the 256-dim sinusoid is
+    # [cos 0]*128 + [sin 0]*128 = [1]*128 + [0]*128, so the embedding reduces
+    # to Linear(SiLU(Linear(that vector))) with library-checked linear layers
+    shape = synth.ModelShape(4, 8, 48, 1, 2, 4, 5, 48, 4, 8)
+    blob = synth.weights_blob(shape, 9)
+    m = orc.Model(shape, blob)
+    freq = np.concatenate([np.ones(128), np.zeros(128)]).astype(np.float32)[None]
+    w1, b1 = synth.weight_view(blob, shape, "t_w1"), synth.weight_view(blob, shape, "t_b1")
+    w2, b2 = synth.weight_view(blob, shape, "t_w2"), synth.weight_view(blob, shape, "t_b2")
+    h1 = freq.astype(np.float64) @ w1.T.astype(np.float64) + b1
+    h1 = h1 / (1.0 + np.exp(-h1))
+    ref = h1 @ w2.T.astype(np.float64) + b2
+    np.testing.assert_allclose(m.time_embed(0.0), ref[0], rtol=1e-5, atol=1e-6)
+    # and t enters only through the sinusoid: two different times differ
+    assert np.abs(m.time_embed(0.5) - m.time_embed(0.0)).max() > 1e-3
+
+
+def test_modulation_is_linear_of_silu(orc):
+    shape = synth.ModelShape(4, 8, 48, 2, 2, 4, 5, 48, 4, 8)
+    blob = synth.weights_blob(shape, 10)
+    m = orc.Model(shape, blob)
+    temb = np.random.default_rng(0).standard_normal(48).astype(np.float32)
+    s = temb.astype(np.float64) / (1.0 + np.exp(-temb.astype(np.float64)))
+    for blk, name in ((1, "mod"), (-1, "fmod")):
+        w = synth.weight_view(blob, shape, name + "_w", blk).astype(np.float64)
+        b = synth.weight_view(blob, shape, name + "_b", blk).astype(np.float64)
+        np.testing.assert_allclose(m.modulation(temb, blk), w @ s + b, rtol=1e-5, atol=1e-6)
