@@ -240,7 +240,16 @@ f3dc_status f3dc_profile(f3dc_handle *h, int32_t enable);
  * Synchronizes the handle's last stream. */
 f3dc_status f3dc_profile_read(f3dc_handle *h, f3dc_kernel_stats *out, int32_t capacity, int32_t *count);
 
-/* Number of kernels this handle has launched since it was created. */
+/* f3dc_sample runs each run of consecutive steps that needs no host
+ * decision in between as one CUDA graph (captured on first use per batch
+ * size, latent buffer and step range, replayed afterwards; every step reads
+ * its quota and row plan from device memory).  enable = 0 launches every
+ * kernel directly instead.  Default: enabled.  Graphs are not used while
+ * profiling is on. */
+f3dc_status f3dc_set_graphs(f3dc_handle *h, int32_t enable);
+
+/* Number of kernels this handle has launched since it was created (a graph
+ * replay counts every kernel it contains). */
 f3dc_status f3dc_launch_count(const f3dc_handle *h, int64_t *count);
 
 /* ---------------------------------------------------------------------- */

@@ -266,6 +266,19 @@ struct f3dc_handle {
     int64_t launches = 0;
     int last_B = 0;
 
+    // CUDA graphs of sampler segments (runs of consecutive steps), replayed
+    // on a library-owned stream ordered with the caller's through events
+    struct SegmentGraph {
+        int B, k0, k1, ka;
+        float *S;
+        cudaGraphExec_t exec;
+        int64_t launches;
+    };
+    std::vector<SegmentGraph> graphs;
+    bool use_graphs = true;
+    cudaStream_t exec_stream = nullptr;
+    cudaEvent_t ev_in = nullptr, ev_out = nullptr;
+
     CUtensorMap tm_h, tm_att, tm_u, tm_cond, tm_q_self, tm_q_cross;
     std::vector<CUtensorMap> tm_qkv_w, tm_o_w, tm_cq_w, tm_co_w, tm_fc1_w, tm_fc2_w, tm_ckv_w, tm_kv_cross;
     int bn_qkv = 128, bn_w = 128, bn_fc1 = 128, bn_ckv = 128;
@@ -480,6 +493,51 @@ f3dc_status run_dit(f3dc_handle *h, float t, const float *S, cudaStream_t s)
     return F3DC_OK;
 }
 
+// Runs steps k0..k1 as one CUDA graph (captured on first use for this batch
+// size, latent buffer and step range; every step reads its quota and the row
+// plan from device memory, so the graph is valid for any quotas).
+f3dc_status run_segment_graph(f3dc_handle *h, int B, float *S, int k0, int k1, int ka, cudaStream_t s)
+{
+    f3dc_handle::SegmentGraph *g = nullptr;
+    for (auto &e : h->graphs)
+        if (e.B == B && e.S == S && e.k0 == k0 && e.k1 == k1 && e.ka == ka) g = &e;
+    if (!g) {
+        if (h->graphs.size() >= 8) {
+            cudaGraphExecDestroy(h->graphs.front().exec);
+            h->graphs.erase(h->graphs.begin());
+        }
+        const int64_t before = h->launches;
+        CK(cudaStreamBeginCapture(h->exec_stream, cudaStreamCaptureModeRelaxed));
+        f3dc_status st = F3DC_OK;
+        for (int k = k0; k <= k1 && st == F3DC_OK; ++k)
+            st = f3dc_step(h, k, B, S, h->ring, h->quota_dev + (size_t)k * B, k == ka ? h->dyn : nullptr,
+                           h->exec_stream);
+        cudaGraph_t graph = nullptr;
+        cudaError_t e = cudaStreamEndCapture(h->exec_stream, &graph);
+        const int64_t captured = h->launches - before;  // kernels per replay
+        h->launches = before;
+        if (st != F3DC_OK) {
+            if (graph) cudaGraphDestroy(graph);
+            return st;
+        }
+        CK(e);
+        cudaGraphExec_t exec = nullptr;
+        e = cudaGraphInstantiate(&exec, graph, 0);
+        cudaGraphDestroy(graph);
+        CK(e);
+        h->graphs.push_back(f3dc_handle::SegmentGraph{B, k0, k1, ka, S, exec, captured});
+        g = &h->graphs.back();
+    }
+    CK(cudaEventRecord(h->ev_in, s));
+    CK(cudaStreamWaitEvent(h->exec_stream, h->ev_in, 0));
+    CK(cudaGraphLaunch(g->exec, h->exec_stream));
+    CK(cudaEventRecord(h->ev_out, h->exec_stream));
+    CK(cudaStreamWaitEvent(s, h->ev_out, 0));
+    h->launches += g->launches;
+    h->last_stream = s;
+    return F3DC_OK;
+}
+
 bool build_maps(f3dc_handle *h)
 {
     const int W = h->W, Wm = h->Wm, dh = h->dh;
@@ -524,6 +582,10 @@ void free_handle(f3dc_handle *h)
     for (cudaEvent_t ev : h->quota_done)
         if (ev) cudaEventDestroy(ev);
     for (cudaEvent_t ev : h->prof.pool) cudaEventDestroy(ev);
+    for (auto &g : h->graphs) cudaGraphExecDestroy(g.exec);
+    if (h->ev_in) cudaEventDestroy(h->ev_in);
+    if (h->ev_out) cudaEventDestroy(h->ev_out);
+    if (h->exec_stream) cudaStreamDestroy(h->exec_stream);
     delete h;
 }
 
@@ -705,6 +767,9 @@ f3dc_status f3dc_create(const f3dc_config *cfg, const f3dc_weights *w, void *str
     CKC(cudaMallocHost(reinterpret_cast<void **>(&h->h_quota), (size_t)2 * (h->T + 1) * B * sizeof(int32_t)));
     CKC(cudaEventCreateWithFlags(&h->quota_done[0], cudaEventDisableTiming));
     CKC(cudaEventCreateWithFlags(&h->quota_done[1], cudaEventDisableTiming));
+    CKC(cudaStreamCreateWithFlags(&h->exec_stream, cudaStreamNonBlocking));
+    CKC(cudaEventCreateWithFlags(&h->ev_in, cudaEventDisableTiming));
+    CKC(cudaEventCreateWithFlags(&h->ev_out, cudaEventDisableTiming));
 #undef CKC
     if (!build_maps(h)) {
         free_handle(h);
@@ -897,29 +962,47 @@ f3dc_status f3dc_sample(f3dc_handle *h, float *S_inout, const void *cond, int32_
     if (sigma_override)
         for (int b = 0; b < B; ++b) sigma[b] = sigma_override[b];
     std::vector<int32_t> consec(B, 0);
-    const bool need_measure = !quota_schedule && !sigma_override;
+    const bool need_measure = !quota_schedule && !sigma_override && ka >= 1 && ka < T;
     bool have_measured = false;
-    for (int k = 1; k <= T; ++k) {
-        for (int b = 0; b < B; ++b) {
-            int phase = 0;
-            int c = quota_schedule ? quota_schedule[(size_t)(k - 1) * B + b] : phase_quota(h->cfg, sigma[b], k, &phase);
-            if (c < 0) c = 0;
-            if (c > N) c = N;
-            hq[(size_t)k * B + b] = tau_gate(h->cfg, c, &consec[b]);
-            if (quota_log) quota_log[(size_t)(k - 1) * B + b] = hq[(size_t)k * B + b];
+    // effective quotas (phase rule or caller schedule, then tau) of steps k0..k1
+    auto fill = [&](int k0, int k1) {
+        for (int k = k0; k <= k1; ++k)
+            for (int b = 0; b < B; ++b) {
+                int phase = 0;
+                int c = quota_schedule ? quota_schedule[(size_t)(k - 1) * B + b]
+                                       : phase_quota(h->cfg, sigma[b], k, &phase);
+                c = c < 0 ? 0 : (c > N ? N : c);
+                hq[(size_t)k * B + b] = tau_gate(h->cfg, c, &consec[b]);
+                if (quota_log) quota_log[(size_t)(k - 1) * B + b] = hq[(size_t)k * B + b];
+            }
+    };
+    auto run = [&](int k0, int k1) -> f3dc_status {
+        CK(cudaMemcpyAsync(h->quota_dev + (size_t)k0 * B, hq + (size_t)k0 * B, (size_t)(k1 - k0 + 1) * B * sizeof(int32_t),
+                           cudaMemcpyHostToDevice, s));
+        if (h->use_graphs && !h->prof.on) return run_segment_graph(h, B, S_inout, k0, k1, ka, s);
+        for (int k = k0; k <= k1; ++k) {
+            f3dc_status r = f3dc_step(h, k, B, S_inout, h->ring, h->quota_dev + (size_t)k * B,
+                                      k == ka ? h->dyn : nullptr, stream);
+            if (r != F3DC_OK) return r;
         }
-        int32_t *qd = h->quota_dev + (size_t)k * B;
-        CK(cudaMemcpyAsync(qd, hq + (size_t)k * B, (size_t)B * sizeof(int32_t), cudaMemcpyHostToDevice, s));
-        st = f3dc_step(h, k, B, S_inout, h->ring, qd, k == ka ? h->dyn : nullptr, stream);
-        if (st != F3DC_OK) return st;
-        if (k == ka && need_measure) {
-            std::vector<int64_t> d(B);
-            CK(cudaMemcpyAsync(d.data(), h->dyn, (size_t)B * sizeof(int64_t), cudaMemcpyDeviceToHost, s));
-            CK(cudaStreamSynchronize(s));
-            for (int b = 0; b < B; ++b) sigma[b] = measured[b] = (double)d[b];
-            have_measured = true;
-        }
+        return F3DC_OK;
+    };
+    if (need_measure) {
+        // Phase 1 up to the anchor, read sigma (Eq. 1 at k_a), then the rest
+        fill(1, ka);
+        if ((st = run(1, ka)) != F3DC_OK) return st;
+        std::vector<int64_t> d(B);
+        CK(cudaMemcpyAsync(d.data(), h->dyn, (size_t)B * sizeof(int64_t), cudaMemcpyDeviceToHost, s));
+        CK(cudaStreamSynchronize(s));
+        for (int b = 0; b < B; ++b) sigma[b] = measured[b] = (double)d[b];
+        have_measured = true;
+        fill(ka + 1, T);
+        if ((st = run(ka + 1, T)) != F3DC_OK) return st;
+    } else {
+        fill(1, T);
+        if ((st = run(1, T)) != F3DC_OK) return st;
     }
+    h->last_stream = s;
     if (sigma_out) {
         if (!have_measured && ka >= 1 && ka <= T) {
             std::vector<int64_t> d(B);
@@ -983,6 +1066,13 @@ f3dc_status f3dc_profile_read(f3dc_handle *h, f3dc_kernel_stats *out, int32_t ca
         ++n;
     }
     *count = n;
+    return F3DC_OK;
+}
+
+f3dc_status f3dc_set_graphs(f3dc_handle *h, int32_t enable)
+{
+    if (!h) return fail(nullptr, F3DC_ERR_INVALID_ARG, "null handle");
+    h->use_graphs = enable != 0;
     return F3DC_OK;
 }
 

@@ -66,6 +66,20 @@ F3DC_DEV bool mbar_try_wait(uint64_t *bar, uint32_t parity)
     return ok != 0;
 }
 
+// try_wait with a suspend-time hint: the thread sleeps until the phase
+// completes or about `hint_ns` passes, instead of spinning on issue slots.
+F3DC_DEV bool mbar_try_wait_sleep(uint64_t *bar, uint32_t parity, uint32_t hint_ns)
+{
+    uint32_t ok;
+    asm volatile(
+        "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, %3;\n"
+        " selp.u32 %0, 1, 0, p;\n}\n"
+        : "=r"(ok)
+        : "r"(smem_u32(bar)), "r"(parity), "r"(hint_ns)
+        : "memory");
+    return ok != 0;
+}
+
 // Waits for the phase with the given parity to complete.  Gives up (returns
 // false) when *abort is set by another thread or after kWaitLimitNs; in the
 // latter case it sets *abort and records kDevTimeout.
@@ -74,8 +88,7 @@ F3DC_DEV bool mbar_wait(uint64_t *bar, uint32_t parity, volatile int *abort, uin
     if (mbar_try_wait(bar, parity)) return true;
     const uint64_t t0 = globaltimer();
     while (true) {
-        for (int i = 0; i < 32; ++i)
-            if (mbar_try_wait(bar, parity)) return true;
+        if (mbar_try_wait_sleep(bar, parity, 100000u)) return true;
         if (*abort) return false;
         if (globaltimer() - t0 > kWaitLimitNs) {
             *abort = 1;
@@ -203,7 +216,20 @@ F3DC_DEV uint32_t f32_to_bf16_bits(float f)
     return (x + (((x >> 16) & 1u) + 0x7FFFu)) >> 16;
 }
 
-F3DC_DEV uint32_t pack_bf16x2(float lo, float hi) { return f32_to_bf16_bits(lo) | (f32_to_bf16_bits(hi) << 16); }
+// Exact software round-to-nearest-even with NaN canonicalised (the velocity
+// history, which must match the reference rounding bit for bit).
+F3DC_DEV uint32_t pack_bf16x2_exact(float lo, float hi)
+{
+    return f32_to_bf16_bits(lo) | (f32_to_bf16_bits(hi) << 16);
+}
+
+// Hardware round-to-nearest-even pack of two floats (activations, P).
+F3DC_DEV uint32_t pack_bf16x2(float lo, float hi)
+{
+    uint32_t r;
+    asm("cvt.rn.bf16x2.f32 %0, %1, %2;" : "=r"(r) : "f"(hi), "f"(lo));
+    return r;
+}
 
 F3DC_DEV float tanh_fast(float x)
 {

@@ -6,20 +6,24 @@
 //           tokens (Supp. Sec. F cross-attention)
 //   mode 2  one sequence (diagnostic entry point)
 //
-// Persistent kernel, one CTA per SM (192 threads), work item = (128-query
+// Persistent kernel, one CTA per SM (320 threads), work item = (128-query
 // tile, head):
 //   warp 0     TMA producer: Q tile once per item, K / V tiles of 128 keys
 //              into a 3-deep ring
 //   warp 1     TMEM allocator + tcgen05.mma issuer:
-//                S_j = Q K_j^T   (M=128, N=128, K=dh)      -> TMEM S[j%2]
-//                O_j = P_j V_j   (M=128, N=dh,  K=128 keys) -> TMEM O[j%2]
+//                S_j = Q K_j^T            (M=128, N=128, K=dh) -> TMEM S[j%2]
+//                O_j,h = P_j,h V_j,h  h=0,1 (M=128, N=dh, K=64)  -> TMEM O[j%2][h]
 //              issued as S_j, then O_(j-1), so the tensor core computes the
 //              next scores and the previous P V while the softmax runs
-//   warps 2-5  softmax, one thread per query row (TMEM lane = row):
-//              running max / sum, P_j = exp2(S_j scale - m) written as bf16
-//              to 128B-swizzled shared memory (the K-major A operand of the
-//              P V MMA), O accumulated in registers with the lazy rescale
-//              O <- (O + O_(j-1)) * exp2(m_(j-1) - m_j)
+//   warps 2-9  softmax, two threads per query row (TMEM lane = row): the
+//              thread of half h owns keys [64h, 64h + 64) of every tile and
+//              runs its own online softmax over them (running max / sum,
+//              P = exp2(S scale - m) as bf16 into its 64-key 128B-swizzled
+//              panel, the K-major A operand of its P V MMA, O accumulated in
+//              registers with the lazy rescale O <- (O + O_(j-1)) * alpha);
+//              the two halves of a row are combined once per work item.
+//              Two softmax warps per SM sub-partition hide each other's
+//              exponent and TMEM latencies.
 // V is the MN-major B operand of the P V MMA straight from its row-major
 // TMA tile.  Keys beyond a sample's count are masked to -inf before the
 // exponent; padding rows are finite by construction, so 0 * pad = 0.
@@ -30,7 +34,8 @@ namespace f3dc {
 
 namespace {
 
-constexpr int kAttnThreads = 192;
+constexpr int kAttnThreads = 320;
+constexpr int kSoftmaxThreads = 256;
 constexpr int kKVStages = 3;
 
 template <int DH>
@@ -41,8 +46,9 @@ struct AttnCfg {
     static constexpr uint32_t kSwz = DH == 64 ? kSwizzle128 : kSwizzle64;
     static constexpr int kPPanel = 128 * 128;           // 64 keys x 128 rows x 2 B
     static constexpr int kPBytes = 2 * kPPanel;
-    static constexpr size_t kSmem = 1024 + kTileBytes * (1 + 2 * kKVStages) + 2 * kPBytes + 512;
-    static constexpr uint32_t kTmemCols = 512;          // S0 S1 | O0 O1
+    static constexpr int kCombineBytes = 128 * (DH + 2) * 4;  // half-1 (m, l, O) per row
+    static constexpr size_t kSmem = 1024 + kTileBytes * (1 + 2 * kKVStages) + 2 * kPBytes + kCombineBytes + 512;
+    static constexpr uint32_t kTmemCols = 512;          // S0 S1 | O[0][0] O[0][1] O[1][0] O[1][1]
 };
 
 struct Item {
@@ -92,7 +98,8 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
     uint8_t *sK = sQ + Cfg::kTileBytes;
     uint8_t *sV = sK + kKVStages * Cfg::kTileBytes;
     uint8_t *sP = sV + kKVStages * Cfg::kTileBytes;
-    uint64_t *bars = reinterpret_cast<uint64_t *>(sP + 2 * Cfg::kPBytes);
+    float *sComb = reinterpret_cast<float *>(sP + 2 * Cfg::kPBytes);
+    uint64_t *bars = reinterpret_cast<uint64_t *>(sP + 2 * Cfg::kPBytes + Cfg::kCombineBytes);
     uint64_t *q_full = bars, *q_empty = bars + 1;
     uint64_t *kv_full = bars + 2, *kv_empty = kv_full + kKVStages;
     uint64_t *s_full = kv_empty + kKVStages, *s_empty = s_full + 2;
@@ -115,11 +122,11 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
         }
         for (int s = 0; s < 2; ++s) {
             mbar_init(&s_full[s], 1);
-            mbar_init(&s_empty[s], 128);
-            mbar_init(&p_full[s], 128);
+            mbar_init(&s_empty[s], kSoftmaxThreads);
+            mbar_init(&p_full[s], kSoftmaxThreads);
             mbar_init(&p_empty[s], 1);
             mbar_init(&o_full[s], 1);
-            mbar_init(&o_empty[s], 128);
+            mbar_init(&o_empty[s], kSoftmaxThreads);
         }
         mbar_init(drain, 1);
         *abort_flag = 0;
@@ -180,11 +187,11 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
                 const uint32_t p_addr = smem_u32(sP + pb * Cfg::kPBytes);
                 const uint32_t v_addr = smem_u32(sV + s * Cfg::kTileBytes);
 #pragma unroll
-                for (int kk = 0; kk < 8; ++kk) {
+                for (int kk = 0; kk < 8; ++kk) {  // keys 16kk..16kk+15, half kk / 4
                     const uint64_t ad = make_sdesc(p_addr + (kk >> 2) * Cfg::kPPanel + (kk & 3) * 32, 16, 1024,
                                                    kSwizzle128);
                     const uint64_t bd = make_sdesc(v_addr + kk * 16 * Cfg::kRowBytes, Cfg::kAtom, Cfg::kAtom, Cfg::kSwz);
-                    mma_bf16(tmem + 256 + pb * DH, ad, bd, idesc_o, kk > 0);
+                    mma_bf16(tmem + 256 + (pb * 2 + (kk >> 2)) * DH, ad, bd, idesc_o, (kk & 3) > 0);
                 }
                 mma_commit(&o_full[pb]);
                 mma_commit(&kv_empty[s]);
@@ -225,7 +232,8 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
         }
     } else {
         // ------------------------------------------------ softmax warps
-        const int q = warp & 3;
+        const int q = warp & 3;                  // TMEM lane quarter of this warp
+        const int half = (warp - 2) >> 2;        // keys [64 half, 64 half + 64) of each tile
         const int row = q * 32 + lane;
         const uint32_t tl = (uint32_t)(q * 32) << 16;
         uint32_t g = 0;
@@ -244,60 +252,65 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
                     break;
                 }
                 tc_fence_after();
-                const int valid = min(128, it.nk - j * 128);
-                const uint32_t s_addr = tmem + tl + sb * 128;
-                // pass 1: row max of the scaled, masked scores
-                float mx = -INFINITY;
-#pragma unroll 1
-                for (int c0 = 0; c0 < 128; c0 += 32) {
-                    uint32_t r[32];
-                    tmem_ld32(s_addr + c0, r);
-                    tmem_wait_ld();
+                const int valid = min(128, it.nk - j * 128) - 64 * half;  // valid keys of this half
+                const uint32_t s_addr = tmem + tl + sb * 128 + 64 * half;
+                uint32_t r0[32], r1[32];
+                tmem_ld32(s_addr, r0);
+                tmem_ld32(s_addr + 32, r1);
+                tmem_wait_ld();
+                float sv[64];
 #pragma unroll
-                    for (int c = 0; c < 32; ++c)
-                        if (c0 + c < valid) mx = fmaxf(mx, __uint_as_float(r[c]) * p.scale_log2);
+                for (int c = 0; c < 32; ++c) {
+                    sv[c] = __uint_as_float(r0[c]);
+                    sv[32 + c] = __uint_as_float(r1[c]);
                 }
-                const float m_new = fmaxf(m_run, mx);
-                const float alpha = exp2_fast(m_run - m_new);
+                if (valid < 64) {  // only the last key tile of a sequence is ragged
+#pragma unroll
+                    for (int c = 0; c < 64; ++c)
+                        if (c >= valid) sv[c] = -INFINITY;
+                }
+                float mx0 = fmaxf(sv[0], sv[1]), mx1 = fmaxf(sv[2], sv[3]);
+#pragma unroll
+                for (int c = 4; c < 64; c += 4) {
+                    mx0 = fmaxf(mx0, fmaxf(sv[c], sv[c + 1]));
+                    mx1 = fmaxf(mx1, fmaxf(sv[c + 2], sv[c + 3]));
+                }
+                const float mx = fmaxf(mx0, mx1);
+                tc_fence_before();
+                mbar_arrive(&s_empty[sb]);
+                // scores are scaled inside the exponent: exp2(s * scale - m)
+                const float m_new = fmaxf(m_run, mx * p.scale_log2);
+                // a half that has not seen a valid key yet (at most 64 keys in
+                // all) keeps m = -inf; subtract 0 instead so nothing is -inf - -inf
+                const float m_use = m_new == -INFINITY ? 0.f : m_new;
+                const float alpha = exp2_fast(m_run - m_use);
                 // P[sb] may still be read by the P V MMA of tile g-2
                 if (!mbar_wait(&p_empty[sb], sph ^ 1, abort_flag, p.err)) {
                     ok = false;
                     break;
                 }
-                // pass 2: P = exp2(s - m_new) -> bf16, 128B-swizzled K-major rows
                 float sum = 0.f;
-                uint8_t *prow = sP + sb * Cfg::kPBytes + row * 128;
-#pragma unroll 1
-                for (int c0 = 0; c0 < 128; c0 += 32) {
-                    uint32_t r[32];
-                    tmem_ld32(s_addr + c0, r);
-                    tmem_wait_ld();
-                    float pv[32];
+                uint8_t *panel = sP + sb * Cfg::kPBytes + half * Cfg::kPPanel + row * 128;
 #pragma unroll
-                    for (int c = 0; c < 32; ++c) {
-                        const float x = (c0 + c < valid) ? __uint_as_float(r[c]) * p.scale_log2 - m_new : -INFINITY;
-                        pv[c] = exp2_fast(x);
-                        sum += pv[c];
-                    }
-                    uint8_t *panel = prow + (c0 >> 6) * Cfg::kPPanel;
+                for (int ch = 0; ch < 8; ++ch) {  // 16-byte chunk ch of the 128-byte row
+                    float pv[8];
 #pragma unroll
-                    for (int ch = 0; ch < 4; ++ch) {
-                        const int chunk = ((c0 & 63) >> 3) + ch;  // 16-byte chunk within the 128-byte row
-                        uint4 u;
-                        u.x = pack_bf16x2(pv[ch * 8 + 0], pv[ch * 8 + 1]);
-                        u.y = pack_bf16x2(pv[ch * 8 + 2], pv[ch * 8 + 3]);
-                        u.z = pack_bf16x2(pv[ch * 8 + 4], pv[ch * 8 + 5]);
-                        u.w = pack_bf16x2(pv[ch * 8 + 6], pv[ch * 8 + 7]);
-                        *reinterpret_cast<uint4 *>(panel + ((chunk ^ (row & 7)) << 4)) = u;
+                    for (int e = 0; e < 8; ++e) {
+                        pv[e] = exp2_fast(fmaf(sv[ch * 8 + e], p.scale_log2, -m_use));
+                        sum += pv[e];
                     }
+                    uint4 u;
+                    u.x = pack_bf16x2(pv[0], pv[1]);
+                    u.y = pack_bf16x2(pv[2], pv[3]);
+                    u.z = pack_bf16x2(pv[4], pv[5]);
+                    u.w = pack_bf16x2(pv[6], pv[7]);
+                    *reinterpret_cast<uint4 *>(panel + ((ch ^ (row & 7)) << 4)) = u;
                 }
-                tc_fence_before();
-                mbar_arrive(&s_empty[sb]);
                 fence_proxy_async_smem();
                 mbar_arrive(&p_full[sb]);
                 l_run = l_run * alpha + sum;
                 m_run = m_new;
-                if (j >= 1) {  // fold O_(j-1), then rescale to the new max
+                if (j >= 1) {  // fold O_(j-1) of this half, then rescale to the new max
                     const uint32_t pb = (g - 1) & 1, pph = ((g - 1) >> 1) & 1;
                     if (!mbar_wait(&o_full[pb], pph, abort_flag, p.err)) {
                         ok = false;
@@ -307,7 +320,7 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
 #pragma unroll
                     for (int d0 = 0; d0 < DH; d0 += 32) {
                         uint32_t r[32];
-                        tmem_ld32(tmem + tl + 256 + pb * DH + d0, r);
+                        tmem_ld32(tmem + tl + 256 + (pb * 2 + half) * DH + d0, r);
                         tmem_wait_ld();
 #pragma unroll
                         for (int d = 0; d < 32; ++d) acc[d0 + d] += __uint_as_float(r[d]);
@@ -319,14 +332,14 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
                 for (int d = 0; d < DH; ++d) acc[d] *= alpha;
             }
             if (!ok) break;
-            {  // fold the last O
+            {  // fold the last O of this half
                 const uint32_t pb = (g - 1) & 1, pph = ((g - 1) >> 1) & 1;
                 if (!mbar_wait(&o_full[pb], pph, abort_flag, p.err)) break;
                 tc_fence_after();
 #pragma unroll
                 for (int d0 = 0; d0 < DH; d0 += 32) {
                     uint32_t r[32];
-                    tmem_ld32(tmem + tl + 256 + pb * DH + d0, r);
+                    tmem_ld32(tmem + tl + 256 + (pb * 2 + half) * DH + d0, r);
                     tmem_wait_ld();
 #pragma unroll
                     for (int d = 0; d < 32; ++d) acc[d0 + d] += __uint_as_float(r[d]);
@@ -334,20 +347,39 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
                 tc_fence_before();
                 mbar_arrive(&o_empty[pb]);
             }
-            const int orow = it.q_row0 + row;
-            if (orow < it.store_end) {
-                const float inv = 1.0f / l_run;
-                uint4 *dst = reinterpret_cast<uint4 *>(p.out + (size_t)orow * p.ldo + it.h * DH);
+            // combine the two halves of each row:
+            // O = (O_0 2^(m_0-m) + O_1 2^(m_1-m)) / (l_0 2^(m_0-m) + l_1 2^(m_1-m))
+            float *mine = sComb + row * (DH + 2);
+            if (half == 1) {
+                mine[0] = m_run;
+                mine[1] = l_run;
 #pragma unroll
-                for (int d = 0; d < DH; d += 8) {
-                    uint4 u;
-                    u.x = pack_bf16x2(acc[d + 0] * inv, acc[d + 1] * inv);
-                    u.y = pack_bf16x2(acc[d + 2] * inv, acc[d + 3] * inv);
-                    u.z = pack_bf16x2(acc[d + 4] * inv, acc[d + 5] * inv);
-                    u.w = pack_bf16x2(acc[d + 6] * inv, acc[d + 7] * inv);
-                    dst[d / 8] = u;
+                for (int d = 0; d < DH; ++d) mine[2 + d] = acc[d];
+            }
+            asm volatile("bar.sync 1, %0;" ::"n"(kSoftmaxThreads) : "memory");
+            if (half == 0) {
+                const float m1 = mine[0], l1 = mine[1];
+                const float m = fmaxf(m_run, m1);
+                const float a0 = exp2_fast(m_run - m), a1 = exp2_fast(m1 - m);
+                const float inv = 1.0f / (l_run * a0 + l1 * a1);
+                const int orow = it.q_row0 + row;
+                if (orow < it.store_end) {
+                    uint4 *dst = reinterpret_cast<uint4 *>(p.out + (size_t)orow * p.ldo + it.h * DH);
+#pragma unroll
+                    for (int d = 0; d < DH; d += 8) {
+                        float o[8];
+#pragma unroll
+                        for (int e = 0; e < 8; ++e) o[e] = (acc[d + e] * a0 + mine[2 + d + e] * a1) * inv;
+                        uint4 u;
+                        u.x = pack_bf16x2(o[0], o[1]);
+                        u.y = pack_bf16x2(o[2], o[3]);
+                        u.z = pack_bf16x2(o[4], o[5]);
+                        u.w = pack_bf16x2(o[6], o[7]);
+                        dst[d / 8] = u;
+                    }
                 }
             }
+            asm volatile("bar.sync 1, %0;" ::"n"(kSoftmaxThreads) : "memory");
         }
     }
     __syncthreads();

@@ -129,8 +129,12 @@ __global__ void __launch_bounds__(kRowThreads) k_layernorm(const float *x, int W
                 y[2] = y[2] * (1.f + sc.z) + sh.z;
                 y[3] = y[3] * (1.f + sc.w) + sh.w;
             } else {
-#pragma unroll
-                for (int u = 0; u < 4; ++u) y[u] = y[u] * bf16_at(g, n0 + u) + bf16_at(bb, n0 + u);
+                const uint2 gw = __ldg(reinterpret_cast<const uint2 *>(reinterpret_cast<const uint16_t *>(g) + n0));
+                const uint2 bw = __ldg(reinterpret_cast<const uint2 *>(reinterpret_cast<const uint16_t *>(bb) + n0));
+                y[0] = y[0] * bf16_bits_to_f32(gw.x & 0xFFFFu) + bf16_bits_to_f32(bw.x & 0xFFFFu);
+                y[1] = y[1] * bf16_bits_to_f32(gw.x >> 16) + bf16_bits_to_f32(bw.x >> 16);
+                y[2] = y[2] * bf16_bits_to_f32(gw.y & 0xFFFFu) + bf16_bits_to_f32(bw.y & 0xFFFFu);
+                y[3] = y[3] * bf16_bits_to_f32(gw.y >> 16) + bf16_bits_to_f32(bw.y >> 16);
             }
             uint2 pk;
             pk.x = pack_bf16x2(y[0], y[1]);

@@ -85,6 +85,7 @@ def lib():
                 "f3dc_profile": ([_vp, C.c_int32], C.c_int),
                 "f3dc_profile_read": ([_vp, C.POINTER(KernelStats), C.c_int32, _i32p], C.c_int),
                 "f3dc_launch_count": ([_vp, C.POINTER(C.c_int64)], C.c_int),
+                "f3dc_set_graphs": ([_vp, C.c_int32], C.c_int),
                 "f3dc_gemm": ([_vp, _vp, _vp, _vp, _vp, C.c_int32, C.c_int32, C.c_int32, C.c_int32, _vp], C.c_int),
                 "f3dc_attention": ([_vp, C.c_int32, _vp, _vp, C.c_int32, _vp, C.c_int32, C.c_int32, C.c_int32,
                                     C.c_int32, _vp], C.c_int),
@@ -230,6 +231,9 @@ class Handle:
         self._ck(lib().f3dc_profile_read(self.h, arr, 32, C.byref(n)))
         return [{"name": arr[i].name.decode(), "launches": arr[i].launches, "total_ms": arr[i].total_ms,
                  "flops": arr[i].flops, "bytes": arr[i].bytes} for i in range(min(n.value, 32))]
+
+    def set_graphs(self, enable: bool):
+        self._ck(lib().f3dc_set_graphs(self.h, 1 if enable else 0))
 
     def launch_count(self) -> int:
         n = C.c_int64(0)

@@ -297,3 +297,30 @@ def open_golden_column():
         if line and not line.startswith("#"):
             out.append(line.split()[3])
     return out
+
+
+def test_sample_graph_replay_matches_eager(orc):
+    # the sampler's CUDA-graph segments compute exactly what eager launches do,
+    # on the first (capturing) call and on later replays
+    c = Ctx(orc, TINY, 2)
+    sig = np.array([6400.0, 9000.0])
+    outs = []
+    for graphs in (False, True, True):
+        c.h.set_graphs(graphs)
+        S_d = dev_f32(c.S)
+        qlog, sigma = c.h.sample(S_d, dev_u16(c.cond), 2, sigma_override=sig)
+        outs.append((S_d.cpu().numpy(), qlog, sigma))
+    for S_g, q_g, s_g in outs[1:]:
+        np.testing.assert_array_equal(S_g, outs[0][0])
+        np.testing.assert_array_equal(q_g, outs[0][1])
+        np.testing.assert_array_equal(s_g, outs[0][2])
+    # the measured-sigma path splits the run at the anchor step
+    res = []
+    for graphs in (False, True):
+        c.h.set_graphs(graphs)
+        S_d = dev_f32(c.S)
+        res.append((S_d,) + c.h.sample(S_d, dev_u16(c.cond), 2))
+    np.testing.assert_array_equal(res[0][0].cpu().numpy(), res[1][0].cpu().numpy())
+    np.testing.assert_array_equal(res[0][1], res[1][1])
+    assert_clean(c.h)
+    c.h.close()
