@@ -11,19 +11,20 @@
 //   warp 0     TMA producer: Q tile once per item, K / V tiles of 128 keys
 //              into a 3-deep ring
 //   warp 1     TMEM allocator + tcgen05.mma issuer:
-//                S_j = Q K_j^T            (M=128, N=128, K=dh) -> TMEM S[j%2]
-//                O_j,h = P_j,h V_j,h  h=0,1 (M=128, N=dh, K=64)  -> TMEM O[j%2][h]
-//              issued as S_j, then O_(j-1), so the tensor core computes the
-//              next scores and the previous P V while the softmax runs
+//                S_j = Q K_j^T              (M=128, N=128, K=dh) -> TMEM S[j%2]
+//                O_h += P_j,h V_j,h  h=0,1  (M=128, N=dh,  K=64) -> TMEM O_h
+//              issued as S_j, then P V of tile j-1, so the tensor core computes
+//              the next scores and the previous P V while the softmax runs
 //   warps 2-9  softmax, two threads per query row (TMEM lane = row): the
 //              thread of half h owns keys [64h, 64h + 64) of every tile and
-//              runs its own online softmax over them (running max / sum,
+//              runs its own online softmax over them, writing
 //              P = exp2(S scale - m) as bf16 into its 64-key 128B-swizzled
-//              panel, the K-major A operand of its P V MMA, O accumulated in
-//              registers with the lazy rescale O <- (O + O_(j-1)) * alpha);
-//              the two halves of a row are combined once per work item.
-//              Two softmax warps per SM sub-partition hide each other's
-//              exponent and TMEM latencies.
+//              panel (the K-major A operand of its P V MMA).  O stays in TMEM
+//              for the whole item; the reference max m is only raised (and O,
+//              l rescaled in place) when a tile's max exceeds it by more than
+//              2^8, so most tiles need no O traffic at all.  The two halves
+//              of a row are combined once per work item.  Two softmax warps per
+//              SM sub-partition hide each other's exponent and TMEM latencies.
 // V is the MN-major B operand of the P V MMA straight from its row-major
 // TMA tile.  Keys beyond a sample's count are masked to -inf before the
 // exponent; padding rows are finite by construction, so 0 * pad = 0.
@@ -48,7 +49,7 @@ struct AttnCfg {
     static constexpr int kPBytes = 2 * kPPanel;
     static constexpr int kCombineBytes = 128 * (DH + 2) * 4;  // half-1 (m, l, O) per row
     static constexpr size_t kSmem = 1024 + kTileBytes * (1 + 2 * kKVStages) + 2 * kPBytes + kCombineBytes + 512;
-    static constexpr uint32_t kTmemCols = 512;          // S0 S1 | O[0][0] O[0][1] O[1][0] O[1][1]
+    static constexpr uint32_t kTmemCols = 512;          // S0 S1 | O_0 O_1
 };
 
 struct Item {
@@ -104,8 +105,8 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
     uint64_t *kv_full = bars + 2, *kv_empty = kv_full + kKVStages;
     uint64_t *s_full = kv_empty + kKVStages, *s_empty = s_full + 2;
     uint64_t *p_full = s_empty + 2, *p_empty = p_full + 2;
-    uint64_t *o_full = p_empty + 2, *o_empty = o_full + 2;
-    uint64_t *drain = o_empty + 2;
+    uint64_t *o_done = p_empty + 2, *o_free = o_done + 1;  // one phase per P V / per item
+    uint64_t *drain = o_free + 1;
     uint32_t *tmem_holder = reinterpret_cast<uint32_t *>(drain + 1);
     volatile int *abort_flag = reinterpret_cast<volatile int *>(tmem_holder + 1);
 
@@ -125,9 +126,9 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
             mbar_init(&s_empty[s], kSoftmaxThreads);
             mbar_init(&p_full[s], kSoftmaxThreads);
             mbar_init(&p_empty[s], 1);
-            mbar_init(&o_full[s], 1);
-            mbar_init(&o_empty[s], kSoftmaxThreads);
         }
+        mbar_init(o_done, 1);
+        mbar_init(o_free, kSoftmaxThreads);
         mbar_init(drain, 1);
         *abort_flag = 0;
         fence_mbar_init();
@@ -178,10 +179,12 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
             const uint32_t q_addr = smem_u32(sQ);
             uint32_t kv_it = 0, g = 0, item_it = 0;
             bool ok = true;
-            auto issue_pv = [&](uint32_t gp, uint32_t kvp) -> bool {
-                const uint32_t pb = gp & 1, pph = (gp >> 1) & 1;
-                if (!mbar_wait(&p_full[pb], pph, abort_flag, p.err)) return false;
-                if (!mbar_wait(&o_empty[pb], pph ^ 1, abort_flag, p.err)) return false;
+            // O_h (+)= P_h V_h for tile gp; the first tile of an item overwrites
+            // O, after the softmax has read the previous item's result
+            auto issue_pv = [&](uint32_t gp, uint32_t kvp, bool first) -> bool {
+                const uint32_t pb = gp & 1;
+                if (!mbar_wait(&p_full[pb], (gp >> 1) & 1, abort_flag, p.err)) return false;
+                if (first && !mbar_wait(o_free, (item_it & 1) ^ 1, abort_flag, p.err)) return false;
                 tc_fence_after();
                 const int s = kvp % kKVStages;
                 const uint32_t p_addr = smem_u32(sP + pb * Cfg::kPBytes);
@@ -191,9 +194,9 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
                     const uint64_t ad = make_sdesc(p_addr + (kk >> 2) * Cfg::kPPanel + (kk & 3) * 32, 16, 1024,
                                                    kSwizzle128);
                     const uint64_t bd = make_sdesc(v_addr + kk * 16 * Cfg::kRowBytes, Cfg::kAtom, Cfg::kAtom, Cfg::kSwz);
-                    mma_bf16(tmem + 256 + (pb * 2 + (kk >> 2)) * DH, ad, bd, idesc_o, (kk & 3) > 0);
+                    mma_bf16(tmem + 256 + (kk >> 2) * DH, ad, bd, idesc_o, !(first && (kk & 3) == 0));
                 }
-                mma_commit(&o_full[pb]);
+                mma_commit(o_done);
                 mma_commit(&kv_empty[s]);
                 mma_commit(&p_empty[pb]);
                 return true;
@@ -222,12 +225,12 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
                                  make_sdesc(k_addr + kk * 32, 16, Cfg::kAtom, Cfg::kSwz), idesc_s, kk > 0);
                     mma_commit(&s_full[sb]);
                     if (j == nkt - 1) mma_commit(q_empty);
-                    if (j >= 1 && !issue_pv(g - 1, kv_it - 1)) {
+                    if (j >= 1 && !issue_pv(g - 1, kv_it - 1, j == 1)) {
                         ok = false;
                         break;
                     }
                 }
-                if (ok && !issue_pv(g - 1, kv_it - 1)) ok = false;
+                if (ok && !issue_pv(g - 1, kv_it - 1, nkt == 1)) ok = false;
             }
         }
     } else {
@@ -236,14 +239,12 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
         const int half = (warp - 2) >> 2;        // keys [64 half, 64 half + 64) of each tile
         const int row = q * 32 + lane;
         const uint32_t tl = (uint32_t)(q * 32) << 16;
-        uint32_t g = 0;
-        for (int w = blockIdx.x; w < total; w += gridDim.x) {
+        const uint32_t o_addr = tmem + tl + 256 + half * DH;
+        uint32_t g = 0, item_it = 0;
+        for (int w = blockIdx.x; w < total; w += gridDim.x, ++item_it) {
             const Item it = decode_item(p, w);
             const int nkt = (it.nk + 127) / 128;
-            float m_run = -INFINITY, l_run = 0.f;
-            float acc[DH];
-#pragma unroll
-            for (int d = 0; d < DH; ++d) acc[d] = 0.f;
+            float m_ref = -INFINITY, l_run = 0.f;
             bool ok = true;
             for (int j = 0; j < nkt; ++j, ++g) {
                 const uint32_t sb = g & 1, sph = (g >> 1) & 1;
@@ -253,11 +254,12 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
                 }
                 tc_fence_after();
                 const int valid = min(128, it.nk - j * 128) - 64 * half;  // valid keys of this half
-                const uint32_t s_addr = tmem + tl + sb * 128 + 64 * half;
                 uint32_t r0[32], r1[32];
-                tmem_ld32(s_addr, r0);
-                tmem_ld32(s_addr + 32, r1);
+                tmem_ld32(tmem + tl + sb * 128 + 64 * half, r0);
+                tmem_ld32(tmem + tl + sb * 128 + 64 * half + 32, r1);
                 tmem_wait_ld();
+                tc_fence_before();
+                mbar_arrive(&s_empty[sb]);
                 float sv[64];
 #pragma unroll
                 for (int c = 0; c < 32; ++c) {
@@ -275,30 +277,50 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
                     mx0 = fmaxf(mx0, fmaxf(sv[c], sv[c + 1]));
                     mx1 = fmaxf(mx1, fmaxf(sv[c + 2], sv[c + 3]));
                 }
-                const float mx = fmaxf(mx0, mx1);
-                tc_fence_before();
-                mbar_arrive(&s_empty[sb]);
-                // scores are scaled inside the exponent: exp2(s * scale - m)
-                const float m_new = fmaxf(m_run, mx * p.scale_log2);
-                // a half that has not seen a valid key yet (at most 64 keys in
-                // all) keeps m = -inf; subtract 0 instead so nothing is -inf - -inf
-                const float m_use = m_new == -INFINITY ? 0.f : m_new;
-                const float alpha = exp2_fast(m_run - m_use);
+                const float mx = fmaxf(mx0, mx1) * p.scale_log2;
+                // raise the reference max only when it grew by more than 2^8
+                // (warp-uniform: TMEM loads / stores are warp-collective)
+                if (__any_sync(0xffffffffu, mx > m_ref + 8.0f)) {
+                    const float m_new = fmaxf(m_ref, mx);
+                    if (j > 0) {  // O holds tiles < j: wait for the last P V, rescale in place
+                        // (the s_full wait above implies the P V of tile g-2 is
+                        // done, so only phase g-1 of o_done can be outstanding)
+                        const float alpha = exp2_fast(m_ref - m_new);
+                        if (!mbar_wait(o_done, (g - 1) & 1, abort_flag, p.err)) {
+                            ok = false;
+                            break;
+                        }
+                        tc_fence_after();
+#pragma unroll
+                        for (int d0 = 0; d0 < DH; d0 += 32) {
+                            uint32_t r[32];
+                            tmem_ld32(o_addr + d0, r);
+                            tmem_wait_ld();
+#pragma unroll
+                            for (int d = 0; d < 32; ++d) r[d] = __float_as_uint(__uint_as_float(r[d]) * alpha);
+                            tmem_st32(o_addr + d0, r);
+                        }
+                        tmem_wait_st();
+                        l_run *= alpha;
+                    }
+                    m_ref = m_new;
+                }
+                // a half with no valid key yet keeps m = -inf: subtract 0 instead
+                const float m_use = m_ref == -INFINITY ? 0.f : m_ref;
                 // P[sb] may still be read by the P V MMA of tile g-2
                 if (!mbar_wait(&p_empty[sb], sph ^ 1, abort_flag, p.err)) {
                     ok = false;
                     break;
                 }
-                float sum = 0.f;
+                float sum0 = 0.f, sum1 = 0.f;
                 uint8_t *panel = sP + sb * Cfg::kPBytes + half * Cfg::kPPanel + row * 128;
 #pragma unroll
                 for (int ch = 0; ch < 8; ++ch) {  // 16-byte chunk ch of the 128-byte row
                     float pv[8];
 #pragma unroll
-                    for (int e = 0; e < 8; ++e) {
-                        pv[e] = exp2_fast(fmaf(sv[ch * 8 + e], p.scale_log2, -m_use));
-                        sum += pv[e];
-                    }
+                    for (int e = 0; e < 8; ++e) pv[e] = exp2_fast(fmaf(sv[ch * 8 + e], p.scale_log2, -m_use));
+                    sum0 += (pv[0] + pv[1]) + (pv[2] + pv[3]);
+                    sum1 += (pv[4] + pv[5]) + (pv[6] + pv[7]);
                     uint4 u;
                     u.x = pack_bf16x2(pv[0], pv[1]);
                     u.y = pack_bf16x2(pv[2], pv[3]);
@@ -307,51 +329,34 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
                     *reinterpret_cast<uint4 *>(panel + ((ch ^ (row & 7)) << 4)) = u;
                 }
                 fence_proxy_async_smem();
+                tc_fence_before();
                 mbar_arrive(&p_full[sb]);
-                l_run = l_run * alpha + sum;
-                m_run = m_new;
-                if (j >= 1) {  // fold O_(j-1) of this half, then rescale to the new max
-                    const uint32_t pb = (g - 1) & 1, pph = ((g - 1) >> 1) & 1;
-                    if (!mbar_wait(&o_full[pb], pph, abort_flag, p.err)) {
-                        ok = false;
-                        break;
-                    }
-                    tc_fence_after();
-#pragma unroll
-                    for (int d0 = 0; d0 < DH; d0 += 32) {
-                        uint32_t r[32];
-                        tmem_ld32(tmem + tl + 256 + (pb * 2 + half) * DH + d0, r);
-                        tmem_wait_ld();
-#pragma unroll
-                        for (int d = 0; d < 32; ++d) acc[d0 + d] += __uint_as_float(r[d]);
-                    }
-                    tc_fence_before();
-                    mbar_arrive(&o_empty[pb]);
-                }
-#pragma unroll
-                for (int d = 0; d < DH; ++d) acc[d] *= alpha;
+                l_run += sum0 + sum1;
             }
             if (!ok) break;
-            {  // fold the last O of this half
-                const uint32_t pb = (g - 1) & 1, pph = ((g - 1) >> 1) & 1;
-                if (!mbar_wait(&o_full[pb], pph, abort_flag, p.err)) break;
-                tc_fence_after();
+            // the item's last P V done: read this half's O, release it.  The
+            // s_full wait of the last tile only guarantees the P V of tile g-3,
+            // so up to two o_done phases are outstanding: wait for them in order
+            // (a single parity wait could be satisfied by the older phase).
+            if (!mbar_wait(o_done, (g - 2) & 1, abort_flag, p.err)) break;
+            if (!mbar_wait(o_done, (g - 1) & 1, abort_flag, p.err)) break;
+            tc_fence_after();
+            float acc[DH];
 #pragma unroll
-                for (int d0 = 0; d0 < DH; d0 += 32) {
-                    uint32_t r[32];
-                    tmem_ld32(tmem + tl + 256 + (pb * 2 + half) * DH + d0, r);
-                    tmem_wait_ld();
+            for (int d0 = 0; d0 < DH; d0 += 32) {
+                uint32_t r[32];
+                tmem_ld32(o_addr + d0, r);
+                tmem_wait_ld();
 #pragma unroll
-                    for (int d = 0; d < 32; ++d) acc[d0 + d] += __uint_as_float(r[d]);
-                }
-                tc_fence_before();
-                mbar_arrive(&o_empty[pb]);
+                for (int d = 0; d < 32; ++d) acc[d0 + d] = __uint_as_float(r[d]);
             }
+            tc_fence_before();
+            mbar_arrive(o_free);
             // combine the two halves of each row:
             // O = (O_0 2^(m_0-m) + O_1 2^(m_1-m)) / (l_0 2^(m_0-m) + l_1 2^(m_1-m))
             float *mine = sComb + row * (DH + 2);
             if (half == 1) {
-                mine[0] = m_run;
+                mine[0] = m_ref;
                 mine[1] = l_run;
 #pragma unroll
                 for (int d = 0; d < DH; ++d) mine[2 + d] = acc[d];
@@ -359,8 +364,8 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
             asm volatile("bar.sync 1, %0;" ::"n"(kSoftmaxThreads) : "memory");
             if (half == 0) {
                 const float m1 = mine[0], l1 = mine[1];
-                const float m = fmaxf(m_run, m1);
-                const float a0 = exp2_fast(m_run - m), a1 = exp2_fast(m1 - m);
+                const float m = fmaxf(m_ref, m1);
+                const float a0 = exp2_fast(m_ref - m), a1 = exp2_fast(m1 - m);
                 const float inv = 1.0f / (l_run * a0 + l1 * a1);
                 const int orow = it.q_row0 + row;
                 if (orow < it.store_end) {
