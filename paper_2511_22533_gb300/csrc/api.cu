@@ -5,6 +5,7 @@
 #include <cmath>
 #include <cstdio>
 #include <cstring>
+#include <mutex>
 #include <string>
 #include <vector>
 
@@ -254,6 +255,8 @@ struct f3dc_handle {
     int32_t *quota_dev = nullptr;
     int64_t *dyn = nullptr;
     uint32_t *dev_err = nullptr;
+    float *gemm_ws = nullptr;          // split-K partial tiles, one per SM
+    int32_t *gemm_cnt = nullptr;       // split-K per-tile arrival counters (kept at 0)
     cudaStream_t last_stream = nullptr;
     int cond_B = 0;
     // pinned per-step quota slots, two generations so one sampler call can
@@ -401,6 +404,9 @@ cudaError_t run_gemm(f3dc_handle *h, const CUtensorMap &ta, const CUtensorMap &t
     p.kn_g = kn;
     p.width = h->W;
     p.dh = h->dh;
+    p.ws = h->gemm_ws;
+    p.counters = h->gemm_cnt;
+    p.ws_units = h->num_sms;
     p.err = h->dev_err;
     int tiles = h->max_tiles * (N / bn);
     int grid = tiles < h->num_sms ? tiles : h->num_sms;
@@ -575,7 +581,8 @@ void free_handle(f3dc_handle *h)
 {
     void *ptrs[] = {h->wblob, h->mod_w, h->mod_b, h->pos, h->x, h->v_active, h->freq, h->h1, h->temb, h->mod,
                     h->h, h->qkv, h->att, h->qc, h->u, h->ckv, h->ring, h->plan, h->tile_sample, h->active_idx,
-                    h->row_of_token, h->n_active, h->mask, h->quota_dev, h->dyn, h->dev_err};
+                    h->row_of_token, h->n_active, h->mask, h->quota_dev, h->dyn, h->dev_err, h->gemm_ws,
+                    h->gemm_cnt};
     for (void *p : ptrs)
         if (p) cudaFree(p);
     if (h->h_quota) cudaFreeHost(h->h_quota);
@@ -764,6 +771,9 @@ f3dc_status f3dc_create(const f3dc_config *cfg, const f3dc_weights *w, void *str
     CKC(dalloc(&h->dyn, (size_t)B));
     CKC(dalloc(&h->dev_err, 1));
     CKC(cudaMemsetAsync(h->dev_err, 0, sizeof(uint32_t), s));
+    CKC(dalloc(&h->gemm_ws, gemm_ws_bytes(256, h->num_sms) / sizeof(float)));
+    CKC(dalloc(&h->gemm_cnt, (size_t)kGemmMaxCounterTiles));
+    CKC(cudaMemsetAsync(h->gemm_cnt, 0, kGemmMaxCounterTiles * sizeof(int32_t), s));
     CKC(cudaMallocHost(reinterpret_cast<void **>(&h->h_quota), (size_t)2 * (h->T + 1) * B * sizeof(int32_t)));
     CKC(cudaEventCreateWithFlags(&h->quota_done[0], cudaEventDisableTiming));
     CKC(cudaEventCreateWithFlags(&h->quota_done[1], cudaEventDisableTiming));
@@ -1112,7 +1122,27 @@ f3dc_status f3dc_gemm(const void *A, const void *B, const void *bias, const floa
     CK(cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev));
     const int tiles = p.m_tiles * (N / bn);
     const int epi = epilogue == F3DC_EPI_BIAS ? kEpiBias : (epilogue == F3DC_EPI_GELU ? kEpiGelu : kEpiResid);
-    CK(launch_gemm(&ta, &tb, p, epi, bn, tiles < sms ? tiles : sms, (cudaStream_t)stream));
+    cudaStream_t s = (cudaStream_t)stream;
+    // split-K workspace: allocated once per device on first use and kept for
+    // the life of the process (its counters return to 0 after every launch)
+    static std::mutex ws_lock;
+    static std::vector<std::pair<int, void *>> ws_per_device;
+    void *ws = nullptr;
+    {
+        std::lock_guard<std::mutex> g(ws_lock);
+        for (auto &e : ws_per_device)
+            if (e.first == dev) ws = e.second;
+        if (!ws) {
+            CK(cudaMalloc(&ws, gemm_ws_bytes(256, sms) + kGemmMaxCounterTiles * sizeof(int32_t)));
+            CK(cudaMemset(reinterpret_cast<char *>(ws) + gemm_ws_bytes(256, sms), 0,
+                          kGemmMaxCounterTiles * sizeof(int32_t)));
+            ws_per_device.push_back({dev, ws});
+        }
+    }
+    p.ws = reinterpret_cast<float *>(ws);
+    p.counters = reinterpret_cast<int32_t *>(reinterpret_cast<char *>(ws) + gemm_ws_bytes(256, sms));
+    p.ws_units = sms;
+    CK(launch_gemm(&ta, &tb, p, epi, bn, tiles < sms ? tiles : sms, s));
     return F3DC_OK;
 }
 

@@ -93,17 +93,54 @@ F3DC_DEV void rms_scale(float *v, int n, const bf16 *g, int gcol)
         v[j] = v[j] * rs * bf16_bits_to_f32(reinterpret_cast<const uint16_t *>(g)[gcol + j]);
 }
 
-template <int BN, int EPI>
-F3DC_DEV void epilogue_tile(const GemmParams &p, uint32_t tbase, int grow, int n0)
+// Accumulator sources for the epilogue: 32 fp32 values of this thread's row
+// at columns c0..c0+31 of the tile, from TMEM (the MMA's accumulator) or as
+// the split-order sum of the split-K partial tiles in the workspace.
+struct TmemSrc {
+    uint32_t tbase;
+    F3DC_DEV void operator()(int c0, float (&v)[32]) const
+    {
+        uint32_t r[32];
+        tmem_ld32(tbase + c0, r);
+        tmem_wait_ld();
+#pragma unroll
+        for (int j = 0; j < 32; ++j) v[j] = __uint_as_float(r[j]);
+    }
+};
+
+template <int BN>
+struct WsSrc {
+    const float *ws;  // partial tile of split s of this tile at ws + (tile + s*tiles)*128*BN
+    int tile, tiles, splits, row;
+    F3DC_DEV void operator()(int c0, float (&v)[32]) const
+    {
+#pragma unroll
+        for (int j = 0; j < 32; ++j) v[j] = 0.f;
+        for (int s = 0; s < splits; ++s) {
+            const float4 *src = reinterpret_cast<const float4 *>(
+                ws + ((size_t)(tile + s * tiles) * 128 + row) * BN + c0);
+#pragma unroll
+            for (int q = 0; q < 8; ++q) {
+                const float4 x = __ldcg(src + q);
+                v[4 * q + 0] += x.x;
+                v[4 * q + 1] += x.y;
+                v[4 * q + 2] += x.z;
+                v[4 * q + 3] += x.w;
+            }
+        }
+    }
+};
+
+template <int BN, int EPI, typename Src>
+F3DC_DEV void epilogue_tile(const GemmParams &p, const Src &src, int grow, int n0)
 {
     const bool row_ok = grow < p.M;
     if constexpr (EPI == kEpiQKNorm) {
 #pragma unroll 1
         for (int c0 = 0; c0 < BN; c0 += 64) {
-            uint32_t r0[32], r1[32];
-            tmem_ld32(tbase + c0, r0);
-            tmem_ld32(tbase + c0 + 32, r1);
-            tmem_wait_ld();
+            float a0[32], a1[32];
+            src(c0, a0);
+            src(c0 + 32, a1);
             const int col = n0 + c0;
             float b0[32], b1[32];
             load_bias32(p.bias, col, b0);
@@ -111,8 +148,8 @@ F3DC_DEV void epilogue_tile(const GemmParams &p, uint32_t tbase, int grow, int n
             float v[64];
 #pragma unroll
             for (int j = 0; j < 32; ++j) {
-                v[j] = __uint_as_float(r0[j]) + b0[j];
-                v[32 + j] = __uint_as_float(r1[j]) + b1[j];
+                v[j] = a0[j] + b0[j];
+                v[32 + j] = a1[j] + b1[j];
             }
             if (col < 2 * p.width) {
                 const bf16 *g = col < p.width ? p.qn_g : p.kn_g;
@@ -139,14 +176,13 @@ F3DC_DEV void epilogue_tile(const GemmParams &p, uint32_t tbase, int grow, int n
     } else {
 #pragma unroll 1
         for (int c0 = 0; c0 < BN; c0 += 32) {
-            uint32_t r[32];
-            tmem_ld32(tbase + c0, r);
-            tmem_wait_ld();
+            float v[32];
+            src(c0, v);
             const int col = n0 + c0;
-            float b[32], v[32];
+            float b[32];
             load_bias32(p.bias, col, b);
 #pragma unroll
-            for (int j = 0; j < 32; ++j) v[j] = __uint_as_float(r[j]) + b[j];
+            for (int j = 0; j < 32; ++j) v[j] += b[j];
             if constexpr (EPI == kEpiGelu) {
 #pragma unroll
                 for (int j = 0; j < 32; ++j) v[j] = gelu_tanh(v[j]);
@@ -172,6 +208,20 @@ F3DC_DEV void epilogue_tile(const GemmParams &p, uint32_t tbase, int grow, int n
     }
 }
 
+// Work decomposition shared by the three roles: unit u covers tile u % tiles
+// (m fastest) and K blocks [split * kb_per, ...) with split = u / tiles.
+struct Units {
+    int m_tiles, tiles, splits, kb_per, kb_n, total;
+    F3DC_DEV void decode(int u, int &m0, int &n0, int &kb0, int &kb1, int BN) const
+    {
+        const int t = u % tiles, s = u / tiles;
+        m0 = (t % m_tiles) * 128;
+        n0 = (t / m_tiles) * BN;
+        kb0 = s * kb_per;
+        kb1 = min(kb_n, kb0 + kb_per);
+    }
+};
+
 template <int BN, int EPI>
 __global__ void __launch_bounds__(kGemmThreads, 1)
     k_gemm(const __grid_constant__ CUtensorMap tma, const __grid_constant__ CUtensorMap tmb, const GemmParams p)
@@ -186,12 +236,25 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
     uint64_t *full = bars, *empty = bars + S, *accf = bars + 2 * S, *acce = accf + 2, *drain = acce + 2;
     uint32_t *tmem_holder = reinterpret_cast<uint32_t *>(drain + 1);
     volatile int *abort_flag = reinterpret_cast<volatile int *>(tmem_holder + 1);
+    volatile int *split_flag = reinterpret_cast<volatile int *>(tmem_holder + 2);
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int m_tiles = p.m_tiles_dev ? *p.m_tiles_dev : p.m_tiles;
-    const int n_tiles = p.N / BN;
-    const int total = m_tiles * n_tiles;
-    const int kb_n = p.K / kBK;
+    Units U;
+    U.m_tiles = p.m_tiles_dev ? *p.m_tiles_dev : p.m_tiles;
+    U.tiles = U.m_tiles * (p.N / BN);
+    U.kb_n = p.K / kBK;
+    // split K only when whole tiles would leave at least half the CTAs idle,
+    // keeping >= 4 K blocks per split and within the workspace
+    U.splits = 1;
+    if (p.ws && U.tiles > 0 && 2 * U.tiles <= (int)gridDim.x && U.tiles <= kGemmMaxCounterTiles) {
+        int sp = (int)gridDim.x / U.tiles;
+        sp = min(sp, U.kb_n / 4);
+        sp = min(sp, p.ws_units / U.tiles);
+        U.splits = max(sp, 1);
+    }
+    U.kb_per = (U.kb_n + U.splits - 1) / U.splits;
+    U.total = U.tiles * U.splits;
+    const int total = U.total;
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < S; ++s) {
@@ -223,8 +286,9 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
             uint32_t ph = 0;
             bool ok = true;
             for (int t = blockIdx.x; t < total && ok; t += gridDim.x) {
-                const int m0 = (t % m_tiles) * 128, n0 = (t / m_tiles) * BN;
-                for (int kb = 0; kb < kb_n; ++kb) {
+                int m0, n0, kb0, kb1;
+                U.decode(t, m0, n0, kb0, kb1, BN);
+                for (int kb = kb0; kb < kb1; ++kb) {
                     if (!mbar_wait(&empty[s], ph ^ 1, abort_flag, p.err)) {
                         ok = false;
                         break;
@@ -251,7 +315,9 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
                 if (!mbar_wait(&acce[buf], aph ^ 1, abort_flag, p.err)) break;
                 tc_fence_after();
                 const uint32_t d = tmem + buf * BN;
-                for (int kb = 0; kb < kb_n; ++kb) {
+                int m0, n0, kb0, kb1;
+                U.decode(t, m0, n0, kb0, kb1, BN);
+                for (int kb = kb0; kb < kb1; ++kb) {
                     if (!mbar_wait(&full[s], ph, abort_flag, p.err)) {
                         ok = false;
                         break;
@@ -261,7 +327,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
 #pragma unroll
                     for (int k = 0; k < kBK / 16; ++k)
                         mma_bf16(d, make_sdesc(a0 + k * 32, 16, 1024, kSwizzle128),
-                                 make_sdesc(b0 + k * 32, 16, 1024, kSwizzle128), idesc, (kb | k) != 0);
+                                 make_sdesc(b0 + k * 32, 16, 1024, kSwizzle128), idesc, (kb != kb0) || (k != 0));
                     mma_commit(&empty[s]);
                     if (++s == S) {
                         s = 0;
@@ -280,12 +346,47 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
             const uint32_t aph = (it >> 1) & 1;
             if (!mbar_wait(&accf[buf], aph, abort_flag, p.err)) break;
             tc_fence_after();
-            const int m0 = (t % m_tiles) * 128, n0 = (t / m_tiles) * BN;
-            const uint32_t tbase = tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(buf * BN);
-            epilogue_tile<BN, EPI>(p, tbase, m0 + row, n0);
+            int m0, n0, kb0, kb1;
+            U.decode(t, m0, n0, kb0, kb1, BN);
+            const TmemSrc tsrc{tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(buf * BN)};
+            if (U.splits == 1) {
+                epilogue_tile<BN, EPI>(p, tsrc, m0 + row, n0);
+                tc_fence_before();
+                mbar_arrive(&acce[buf]);
+                continue;
+            }
+            // split K: store this split's fp32 partial row, free TMEM, and let
+            // the last CTA to finish the tile reduce the splits in order
+            float *wrow = p.ws + ((size_t)t * 128 + row) * BN;
+#pragma unroll 1
+            for (int c0 = 0; c0 < BN; c0 += 32) {
+                float v[32];
+                tsrc(c0, v);
+#pragma unroll
+                for (int q4 = 0; q4 < 8; ++q4)
+                    __stcg(reinterpret_cast<float4 *>(wrow + c0) + q4,
+                           make_float4(v[4 * q4], v[4 * q4 + 1], v[4 * q4 + 2], v[4 * q4 + 3]));
+            }
             tc_fence_before();
             mbar_arrive(&acce[buf]);
+            const int tile = t % U.tiles;
+            __threadfence();
+            asm volatile("bar.sync 2, 128;" ::: "memory");
+            if (threadIdx.x == 64) {
+                const int prev = atomicAdd(p.counters + tile, 1);
+                const int last = prev == U.splits - 1;
+                if (last) p.counters[tile] = 0;  // ready for the next launch
+                *split_flag = last;
+            }
+            asm volatile("bar.sync 2, 128;" ::: "memory");
+            if (*split_flag) {
+                __threadfence();
+                const WsSrc<BN> wsrc{p.ws, tile, U.tiles, U.splits, row};
+                epilogue_tile<BN, EPI>(p, wsrc, m0 + row, n0);
+            }
+            asm volatile("bar.sync 2, 128;" ::: "memory");
         }
+
     }
     __syncthreads();
     if (*abort_flag) {

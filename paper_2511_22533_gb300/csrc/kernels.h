@@ -108,12 +108,23 @@ struct GemmParams {
     const float *gate;        // nullable (RESID)
     const bf16 *qn_g, *kn_g;  // QKNORM gammas [W]
     int width, dh;            // QKNORM: columns < 2*width are normalised per dh-group
+    // split-K workspace (nullable: no split).  When the tile count leaves
+    // SMs idle the kernel splits each tile's K range over several CTAs, which
+    // write fp32 partial tiles to ws; the last CTA of a tile (per-tile arrival
+    // counter in `counters`, left at 0) sums them in split order and applies
+    // the epilogue.
+    float *ws;
+    int32_t *counters;
+    int ws_units;             // partial tiles the workspace holds
     uint32_t *err;
 };
 // bn in {64, 128, 256}
 cudaError_t launch_gemm(const CUtensorMap *ta, const CUtensorMap *tb, const GemmParams &p, int epi, int bn,
                         int grid, cudaStream_t s);
 size_t gemm_smem_bytes(int bn);
+// bytes of split-K workspace for `units` partial tiles of width bn
+inline size_t gemm_ws_bytes(int bn, int units) { return (size_t)units * 128 * bn * sizeof(float); }
+constexpr int kGemmMaxCounterTiles = 1024;
 
 // ------------------------------------------------------------ attention
 struct AttnParams {

@@ -109,6 +109,20 @@ def test_forward_trellis_width_two_blocks(orc):
     c.h.close()
 
 
+def test_forward_trellis_width_few_active(orc):
+    # 300 and 77 active tokens at TRELLIS width: every projection (QKV with the
+    # QK norm, out, cross-Q, cross-out, fc1 + GELU, fc2) runs with split K
+    shape = synth.ModelShape(16, 8, 1024, 1, 16, 4, 1374, 1024, 25, 64)
+    c = Ctx(orc, shape, 2, seed=8)
+    g = np.random.default_rng(8)
+    lists = [np.sort(g.choice(4096, 300, replace=False)), np.sort(g.choice(4096, 77, replace=False))]
+    got = _forward_gpu(c.h, 0.7, c.S, lists)
+    for b in range(2):
+        _assert_vel(got[b], c.m.forward(c.S[b], lists[b], 0.7, c.kv[b]), f"sample {b}")
+    assert_clean(c.h)
+    c.h.close()
+
+
 def test_forward_ragged_batch8(orc):
     # batch 8 with ragged active counts in [400, 4096] (TRELLIS width, 1 block);
     # three samples are checked against the oracle, all eight run packed

@@ -13,6 +13,9 @@ pytestmark = pytest.mark.gpu
 
 SHAPES = [(1229, 1024, 1024), (4096, 3072, 1024), (1000, 4096, 1024), (1229, 1024, 4096), (100, 256, 128),
           (1, 64, 64), (257, 384, 128), (300, 128, 256)]
+# few row tiles: the kernel splits K over CTAs and reduces the partials in
+# split order (workspace + per-tile arrival counters)
+SPLIT_SHAPES = [(955, 1024, 1024), (300, 1024, 4096), (128, 256, 1024), (640, 3072, 1024), (413, 1024, 4096)]
 
 
 def _inputs(M, N, K, seed):
@@ -31,7 +34,7 @@ def _ref(orc, A, Bw, bias, rows):
     return orc.linear(a, w, synth.bf16_bits_to_f32(bias)).astype(np.float64)
 
 
-@pytest.mark.parametrize("M,N,K", SHAPES)
+@pytest.mark.parametrize("M,N,K", SHAPES + SPLIT_SHAPES)
 def test_gemm_bias(orc, M, N, K):
     A, Bw, bias, _, rows = _inputs(M, N, K, M + N + K)
     out = torch.zeros((M, N), dtype=torch.bfloat16, device="cuda")
@@ -44,7 +47,7 @@ def test_gemm_bias(orc, M, N, K):
     assert np.all(np.abs(got - ref) <= 2.0 ** -7 * np.abs(ref) + 1e-3)
 
 
-@pytest.mark.parametrize("M,N,K", SHAPES[:4])
+@pytest.mark.parametrize("M,N,K", SHAPES[:4] + SPLIT_SHAPES[:2])
 def test_gemm_gelu(orc, M, N, K):
     A, Bw, bias, _, rows = _inputs(M, N, K, 7 + M)
     out = torch.zeros((M, N), dtype=torch.bfloat16, device="cuda")
@@ -57,7 +60,7 @@ def test_gemm_gelu(orc, M, N, K):
     assert np.max(np.abs(got - ref)) < 2e-2 * max(1.0, np.abs(ref).max())
 
 
-@pytest.mark.parametrize("M,N,K", SHAPES[:4] + SHAPES[6:])
+@pytest.mark.parametrize("M,N,K", SHAPES[:4] + SHAPES[6:] + SPLIT_SHAPES)
 @pytest.mark.parametrize("with_gate", [True, False])
 def test_gemm_residual(orc, M, N, K, with_gate):
     A, Bw, bias, gate, rows = _inputs(M, N, K, 11 + N)
@@ -90,3 +93,17 @@ def test_gemm_no_bias_and_repeat_is_deterministic(orc):
     assert torch.equal(outs[0], outs[1])
     ref = orc.linear(synth.bf16_bits_to_f32(A[rows]), synth.bf16_bits_to_f32(Bw))
     assert rel_l2(outs[0].float().cpu().numpy()[rows], ref) < 4e-3
+
+
+def test_gemm_split_k_repeat_is_deterministic(orc):
+    # the split partials are always summed in split order by whichever CTA
+    # arrives last, so repeated launches agree bit for bit
+    M, N, K = 300, 1024, 4096
+    A, Bw, bias, gate, rows = _inputs(M, N, K, 21)
+    outs = []
+    for _ in range(3):
+        x = torch.zeros((M, N), dtype=torch.float32, device="cuda")
+        f3dc.gemm(dev_bf16(A), dev_bf16(Bw), dev_bf16(bias), dev_f32(gate), x, M, N, K, f3dc.EPI_RESID)
+        outs.append(x)
+    torch.cuda.synchronize()
+    assert torch.equal(outs[0], outs[1]) and torch.equal(outs[0], outs[2])
