@@ -234,6 +234,8 @@ struct Profiler {
 
 }  // namespace
 
+void f3dc::set_host_error(const std::string &msg) { g_last_error = msg; }
+
 struct f3dc_handle {
     f3dc_config cfg;
     int N = 0, W = 0, Wm = 0, H = 0, dh = 0, L = 0, Nc = 0, Dc = 0, G = 0, T = 0;
@@ -404,7 +406,10 @@ cudaError_t run_gemm(f3dc_handle *h, const CUtensorMap &ta, const CUtensorMap &t
     p.kn_g = kn;
     p.width = h->W;
     p.dh = h->dh;
-    p.ws = h->gemm_ws;
+    // split K stays off in the step: at 400-1229 active tokens it measured
+    // slower than whole tiles (the partial round trip through L2 and the
+    // last-arriving CTA's reduction cost more than the shorter K loop saves)
+    p.ws = nullptr;
     p.counters = h->gemm_cnt;
     p.ws_units = h->num_sms;
     p.err = h->dev_err;
@@ -1142,7 +1147,7 @@ f3dc_status f3dc_gemm(const void *A, const void *B, const void *bias, const floa
     p.ws = reinterpret_cast<float *>(ws);
     p.counters = reinterpret_cast<int32_t *>(reinterpret_cast<char *>(ws) + gemm_ws_bytes(256, sms));
     p.ws_units = sms;
-    CK(launch_gemm(&ta, &tb, p, epi, bn, tiles < sms ? tiles : sms, s));
+    CK(launch_gemm(&ta, &tb, p, epi, bn, gemm_grid(tiles, sms), s));
     return F3DC_OK;
 }
 

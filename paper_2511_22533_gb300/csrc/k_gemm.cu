@@ -69,7 +69,7 @@ F3DC_DEV void load_bias32(const bf16 *bias, int col, float (&b)[32])
     }
 }
 
-F3DC_DEV void store_bf16x32(bf16 *dst, const float (&v)[32])
+F3DC_DEV void store_bf16x32(bf16 *dst, const float *v)
 {
     uint4 *p = reinterpret_cast<uint4 *>(dst);
 #pragma unroll
@@ -98,7 +98,7 @@ F3DC_DEV void rms_scale(float *v, int n, const bf16 *g, int gcol)
 // the split-order sum of the split-K partial tiles in the workspace.
 struct TmemSrc {
     uint32_t tbase;
-    F3DC_DEV void operator()(int c0, float (&v)[32]) const
+    F3DC_DEV void operator()(int c0, float *v) const
     {
         uint32_t r[32];
         tmem_ld32(tbase + c0, r);
@@ -112,21 +112,31 @@ template <int BN>
 struct WsSrc {
     const float *ws;  // partial tile of split s of this tile at ws + (tile + s*tiles)*128*BN
     int tile, tiles, splits, row;
-    F3DC_DEV void operator()(int c0, float (&v)[32]) const
+    // 4 columns at a time: the loads of every split are issued before the
+    // in-order sum, so the reduction costs one L2 latency per 4 columns
+    F3DC_DEV void operator()(int c0, float *v) const
     {
+        const size_t split_stride4 = (size_t)tiles * 128 * BN / 4;
+        const float4 *base = reinterpret_cast<const float4 *>(ws + ((size_t)tile * 128 + row) * BN + c0);
 #pragma unroll
-        for (int j = 0; j < 32; ++j) v[j] = 0.f;
-        for (int s = 0; s < splits; ++s) {
-            const float4 *src = reinterpret_cast<const float4 *>(
-                ws + ((size_t)(tile + s * tiles) * 128 + row) * BN + c0);
+        for (int c4 = 0; c4 < 8; ++c4) {
+            float4 part[kGemmMaxSplits];
 #pragma unroll
-            for (int q = 0; q < 8; ++q) {
-                const float4 x = __ldcg(src + q);
-                v[4 * q + 0] += x.x;
-                v[4 * q + 1] += x.y;
-                v[4 * q + 2] += x.z;
-                v[4 * q + 3] += x.w;
-            }
+            for (int s = 0; s < kGemmMaxSplits; ++s)
+                if (s < splits) part[s] = __ldcg(base + s * split_stride4 + c4);
+            float4 a = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+            for (int s = 0; s < kGemmMaxSplits; ++s)
+                if (s < splits) {
+                    a.x += part[s].x;
+                    a.y += part[s].y;
+                    a.z += part[s].z;
+                    a.w += part[s].w;
+                }
+            v[4 * c4 + 0] = a.x;
+            v[4 * c4 + 1] = a.y;
+            v[4 * c4 + 2] = a.z;
+            v[4 * c4 + 3] = a.w;
         }
     }
 };
@@ -138,18 +148,18 @@ F3DC_DEV void epilogue_tile(const GemmParams &p, const Src &src, int grow, int n
     if constexpr (EPI == kEpiQKNorm) {
 #pragma unroll 1
         for (int c0 = 0; c0 < BN; c0 += 64) {
-            float a0[32], a1[32];
-            src(c0, a0);
-            src(c0 + 32, a1);
-            const int col = n0 + c0;
-            float b0[32], b1[32];
-            load_bias32(p.bias, col, b0);
-            load_bias32(p.bias, col + 32, b1);
             float v[64];
+            src(c0, v);
+            src(c0 + 32, v + 32);
+            const int col = n0 + c0;
+            {
+                float b[32];
+                load_bias32(p.bias, col, b);
 #pragma unroll
-            for (int j = 0; j < 32; ++j) {
-                v[j] = a0[j] + b0[j];
-                v[32 + j] = a1[j] + b1[j];
+                for (int j = 0; j < 32; ++j) v[j] += b[j];
+                load_bias32(p.bias, col + 32, b);
+#pragma unroll
+                for (int j = 0; j < 32; ++j) v[32 + j] += b[j];
             }
             if (col < 2 * p.width) {
                 const bf16 *g = col < p.width ? p.qn_g : p.kn_g;
@@ -163,14 +173,8 @@ F3DC_DEV void epilogue_tile(const GemmParams &p, const Src &src, int grow, int n
             }
             if (row_ok) {
                 bf16 *dst = reinterpret_cast<bf16 *>(p.out) + (size_t)grow * p.ldo + col;
-                float lo[32], hi[32];
-#pragma unroll
-                for (int j = 0; j < 32; ++j) {
-                    lo[j] = v[j];
-                    hi[j] = v[32 + j];
-                }
-                store_bf16x32(dst, lo);
-                store_bf16x32(dst + 32, hi);
+                store_bf16x32(dst, v);
+                store_bf16x32(dst + 32, v + 32);
             }
         }
     } else {
@@ -243,15 +247,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
     U.m_tiles = p.m_tiles_dev ? *p.m_tiles_dev : p.m_tiles;
     U.tiles = U.m_tiles * (p.N / BN);
     U.kb_n = p.K / kBK;
-    // split K only when whole tiles would leave at least half the CTAs idle,
-    // keeping >= 4 K blocks per split and within the workspace
-    U.splits = 1;
-    if (p.ws && U.tiles > 0 && 2 * U.tiles <= (int)gridDim.x && U.tiles <= kGemmMaxCounterTiles) {
-        int sp = (int)gridDim.x / U.tiles;
-        sp = min(sp, U.kb_n / 4);
-        sp = min(sp, p.ws_units / U.tiles);
-        U.splits = max(sp, 1);
-    }
+    U.splits = gemm_split_count(U.tiles, (int)gridDim.x, U.kb_n, p.ws_units, p.ws != nullptr);
     U.kb_per = (U.kb_n + U.splits - 1) / U.splits;
     U.total = U.tiles * U.splits;
     const int total = U.total;

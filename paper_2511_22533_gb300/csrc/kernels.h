@@ -7,6 +7,8 @@
 #include <cuda_runtime.h>
 #include <stdint.h>
 
+#include <string>
+
 namespace f3dc {
 
 constexpr int kTileRows = 128;   // rows per tile; every sample's packed rows start on a tile
@@ -126,6 +128,28 @@ size_t gemm_smem_bytes(int bn);
 inline size_t gemm_ws_bytes(int bn, int units) { return (size_t)units * 128 * bn * sizeof(float); }
 constexpr int kGemmMaxCounterTiles = 1024;
 
+// Split-K rule (shared by the kernel and the host): split a tile's K range
+// only when whole tiles would leave at least half of the `grid` CTAs idle,
+// keeping >= 4 K blocks (of 64) per split and within `ws_units` partial tiles.
+// The count is rounded so that ceil(kb_n / splits) K blocks per split leave
+// no split empty (an empty split would contribute a stale accumulator).
+constexpr int kGemmMaxSplits = 16;
+__host__ __device__ inline int gemm_split_count(int tiles, int grid, int kb_n, int ws_units, bool have_ws)
+{
+    if (!have_ws || tiles <= 0 || 2 * tiles > grid || tiles > kGemmMaxCounterTiles) return 1;
+    int sp = grid / tiles;
+    if (sp > kb_n / 4) sp = kb_n / 4;
+    if (sp > ws_units / tiles) sp = ws_units / tiles;
+    if (sp > kGemmMaxSplits) sp = kGemmMaxSplits;
+    if (sp <= 1) return 1;
+    const int per = (kb_n + sp - 1) / sp;
+    return (kb_n + per - 1) / per;
+}
+
+// Grid of a GEMM whose tile count is known on the host: one CTA per tile,
+// or every SM when few tiles leave room to split K.
+inline int gemm_grid(int tiles, int sms) { return 2 * tiles <= sms ? sms : (tiles < sms ? tiles : sms); }
+
 // ------------------------------------------------------------ attention
 struct AttnParams {
     int heads, dh;
@@ -147,6 +171,9 @@ cudaError_t launch_attention(const CUtensorMap *tq, const CUtensorMap *tk, const
 size_t attn_smem_bytes(int dh);
 
 // ------------------------------------------------------------ host helpers
+// Records the message f3dc_last_error(NULL) returns on this thread.
+void set_host_error(const std::string &msg);
+
 // 2-D bf16 tensor map over a row-major [rows, cols] matrix with leading
 // dimension ld (elements), box [box_rows, box_cols], 128B (box_cols = 64) or
 // 64B (box_cols = 32) swizzle.  Returns false on failure.
