@@ -287,6 +287,31 @@ f3dc_status f3dc_forward(f3dc_handle *h, float t, int32_t B, const float *S,
 f3dc_status f3dc_gemm(const void *A, const void *B, const void *bias, const float *gate,
                       void *out, int32_t M, int32_t N, int32_t K, int32_t epilogue, void *stream);
 
+/* f3dc_gemm for callers that must not allocate device memory.  The paper has
+ * no counterpart: this is a library service.  Code running while a CUDA graph
+ * is captured in global mode cannot call cudaMalloc, some frameworks own all
+ * device memory through their own pool and forbid side allocations, and
+ * latency-critical loops must not enter the driver's allocator; f3dc_gemm,
+ * which allocates its split-K workspace on first use per device, serves none
+ * of them.  This call computes the same result as f3dc_gemm (same tiling,
+ * same split rule, same summation order), with the same arguments and
+ * errors, but takes the split-K workspace from a fixed 20 MiB array (plus
+ * 4 KiB of counters) compiled into libf3dc; every GPU that loads the library
+ * holds that array until the process exits.  It calls no allocation routine.
+ *   - The first call on a device resolves the array's device address (with
+ *     that device current); make that first call before any stream capture.
+ *   - A problem whose split-K partials would exceed 20 MiB is rejected with
+ *     F3DC_ERR_INVALID_ARG and a message giving both sizes; on a GB300 (152
+ *     SMs) every shape fits, since a split never uses more partial tiles than
+ *     the device has SMs.
+ *   - All calls share the array and it keeps the previous call's contents:
+ *     the call clears the arrival counters on `stream` before its launch, and
+ *     calls whose executions overlap on the GPU (different streams, or
+ *     different host threads without ordering) race on it.
+ * Failures are described by f3dc_last_error(NULL).  Asynchronous on `stream`. */
+f3dc_status f3dc_gemm_noalloc(const void *A, const void *B, const void *bias, const float *gate, void *out,
+                              int32_t M, int32_t N, int32_t K, int32_t epilogue, void *stream);
+
 /* Single-sequence multi-head attention softmax(q k^T / sqrt(dh)) v with the
  * tensor-core flash kernel.
  *   q: device bf16 [nq, ldq] (head h at columns h*dh); k, v: device bf16

@@ -87,6 +87,8 @@ def lib():
                 "f3dc_launch_count": ([_vp, C.POINTER(C.c_int64)], C.c_int),
                 "f3dc_set_graphs": ([_vp, C.c_int32], C.c_int),
                 "f3dc_gemm": ([_vp, _vp, _vp, _vp, _vp, C.c_int32, C.c_int32, C.c_int32, C.c_int32, _vp], C.c_int),
+                "f3dc_gemm_noalloc": ([_vp, _vp, _vp, _vp, _vp, C.c_int32, C.c_int32, C.c_int32, C.c_int32, _vp],
+                                      C.c_int),
                 "f3dc_attention": ([_vp, C.c_int32, _vp, _vp, C.c_int32, _vp, C.c_int32, C.c_int32, C.c_int32,
                                     C.c_int32, _vp], C.c_int),
             }
@@ -250,6 +252,12 @@ class Handle:
 def gemm(A, Bw, bias, gate, out, M, N, K, epilogue, stream=None):
     _check(lib().f3dc_gemm(_ptr(A), _ptr(Bw), _ptr(bias), _ptr(gate), _ptr(out), M, N, K, epilogue,
                            _stream(stream)))
+
+
+def gemm_noalloc(A, Bw, bias, gate, out, M, N, K, epilogue, stream=None):
+    """f3dc_gemm without any allocation (split-K scratch in a static array)."""
+    _check(lib().f3dc_gemm_noalloc(_ptr(A), _ptr(Bw), _ptr(bias), _ptr(gate), _ptr(out), M, N, K, epilogue,
+                                   _stream(stream)))
 
 
 def attention(q, ldq, k, v, ldkv, out, nq, nk, heads, dh, stream=None):
