@@ -9,12 +9,13 @@
 // Persistent kernel, one CTA per SM (320 threads), work item = (128-query
 // tile, head):
 //   warp 0     TMA producer: Q tile once per item, K / V tiles of 128 keys
-//              into a 3-deep ring
+//              into a 4-deep ring
 //   warp 1     TMEM allocator + tcgen05.mma issuer:
 //                S_j = Q K_j^T              (M=128, N=128, K=dh) -> TMEM S[j%2]
 //                O_h += P_j,h V_j,h  h=0,1  (M=128, N=dh,  K=64) -> TMEM O_h
-//              issued as S_j, then P V of tile j-1, so the tensor core computes
-//              the next scores and the previous P V while the softmax runs
+//              S runs two tiles ahead: S_(j+2) is issued as soon as the
+//              softmax has read S_j, before P V of tile j, so the scores of
+//              the next tiles are ready whenever the softmax gets to them
 //   warps 2-9  softmax, two threads per query row (TMEM lane = row): the
 //              thread of half h owns keys [64h, 64h + 64) of every tile and
 //              runs its own online softmax over them, writing
@@ -37,7 +38,8 @@ namespace {
 
 constexpr int kAttnThreads = 320;
 constexpr int kSoftmaxThreads = 256;
-constexpr int kKVStages = 3;
+constexpr int kSoftmaxWarps = kSoftmaxThreads / 32;  // arrivals per phase (one per warp)
+constexpr int kKVStages = 4;
 
 template <int DH>
 struct AttnCfg {
@@ -47,8 +49,9 @@ struct AttnCfg {
     static constexpr uint32_t kSwz = DH == 64 ? kSwizzle128 : kSwizzle64;
     static constexpr int kPPanel = 128 * 128;           // 64 keys x 128 rows x 2 B
     static constexpr int kPBytes = 2 * kPPanel;
-    static constexpr int kCombineBytes = 128 * (DH + 2) * 4;  // half-1 (m, l, O) per row
-    static constexpr size_t kSmem = 1024 + kTileBytes * (1 + 2 * kKVStages) + 2 * kPBytes + kCombineBytes + 512;
+    static constexpr int kCombineBytes = 128 * (DH + 2) * 4;  // half-1 (m, l, O) per row, aliases P
+    static_assert(kCombineBytes <= 2 * kPBytes, "combine scratch must fit in the P buffers");
+    static constexpr size_t kSmem = 1024 + kTileBytes * (1 + 2 * kKVStages) + 2 * kPBytes + 512;
     static constexpr uint32_t kTmemCols = 512;          // S0 S1 | O_0 O_1
 };
 
@@ -99,13 +102,17 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
     uint8_t *sK = sQ + Cfg::kTileBytes;
     uint8_t *sV = sK + kKVStages * Cfg::kTileBytes;
     uint8_t *sP = sV + kKVStages * Cfg::kTileBytes;
-    float *sComb = reinterpret_cast<float *>(sP + 2 * Cfg::kPBytes);
-    uint64_t *bars = reinterpret_cast<uint64_t *>(sP + 2 * Cfg::kPBytes + Cfg::kCombineBytes);
+    // the end-of-item combine runs when every P V of the item is done, so
+    // its scratch can live in the P buffers
+    float *sComb = reinterpret_cast<float *>(sP);
+    uint64_t *bars = reinterpret_cast<uint64_t *>(sP + 2 * Cfg::kPBytes);
     uint64_t *q_full = bars, *q_empty = bars + 1;
     uint64_t *kv_full = bars + 2, *kv_empty = kv_full + kKVStages;
     uint64_t *s_full = kv_empty + kKVStages, *s_empty = s_full + 2;
     uint64_t *p_full = s_empty + 2, *p_empty = p_full + 2;
-    uint64_t *o_done = p_empty + 2, *o_free = o_done + 1;  // one phase per P V / per item
+    // p_empty[t % 2] completes once per P V of (global) tile index t and
+    // doubles as the "O holds tiles <= t" signal; o_free completes once per item
+    uint64_t *o_free = p_empty + 2;
     uint64_t *drain = o_free + 1;
     uint32_t *tmem_holder = reinterpret_cast<uint32_t *>(drain + 1);
     volatile int *abort_flag = reinterpret_cast<volatile int *>(tmem_holder + 1);
@@ -123,12 +130,11 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
         }
         for (int s = 0; s < 2; ++s) {
             mbar_init(&s_full[s], 1);
-            mbar_init(&s_empty[s], kSoftmaxThreads);
-            mbar_init(&p_full[s], kSoftmaxThreads);
+            mbar_init(&s_empty[s], kSoftmaxWarps);
+            mbar_init(&p_full[s], kSoftmaxWarps);
             mbar_init(&p_empty[s], 1);
         }
-        mbar_init(o_done, 1);
-        mbar_init(o_free, kSoftmaxThreads);
+        mbar_init(o_free, kSoftmaxWarps);
         mbar_init(drain, 1);
         *abort_flag = 0;
         fence_mbar_init();
@@ -177,16 +183,33 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
             constexpr uint32_t idesc_s = make_idesc_bf16(128, 128, 0, 0);
             constexpr uint32_t idesc_o = make_idesc_bf16(128, DH, 0, 1);
             const uint32_t q_addr = smem_u32(sQ);
-            uint32_t kv_it = 0, g = 0, item_it = 0;
+            uint32_t kv_base = 0, g_base = 0, item_it = 0;  // global tile / kv-stage counters
             bool ok = true;
-            // O_h (+)= P_h V_h for tile gp; the first tile of an item overwrites
-            // O, after the softmax has read the previous item's result
-            auto issue_pv = [&](uint32_t gp, uint32_t kvp, bool first) -> bool {
-                const uint32_t pb = gp & 1;
-                if (!mbar_wait(&p_full[pb], (gp >> 1) & 1, abort_flag, p.err)) return false;
+            // S for tile j of the item: needs its K tile and a free S buffer
+            // (the softmax has read S of tile j-2)
+            auto issue_s = [&](uint32_t gt, uint32_t kvt, bool last) -> bool {
+                const int s = kvt % kKVStages;
+                const uint32_t sb = gt & 1;
+                if (!mbar_wait(&kv_full[s], (kvt / kKVStages) & 1, abort_flag, p.err)) return false;
+                if (!mbar_wait(&s_empty[sb], ((gt >> 1) & 1) ^ 1, abort_flag, p.err)) return false;
+                tc_fence_after();
+                const uint32_t k_addr = smem_u32(sK + s * Cfg::kTileBytes);
+#pragma unroll
+                for (int kk = 0; kk < DH / 16; ++kk)
+                    mma_bf16(tmem + sb * 128, make_sdesc(q_addr + kk * 32, 16, Cfg::kAtom, Cfg::kSwz),
+                             make_sdesc(k_addr + kk * 32, 16, Cfg::kAtom, Cfg::kSwz), idesc_s, kk > 0);
+                mma_commit(&s_full[sb]);
+                if (last) mma_commit(q_empty);
+                return true;
+            };
+            // O_h (+)= P_h V_h for tile gt; the item's first tile overwrites O,
+            // after the softmax has read the previous item's result
+            auto issue_pv = [&](uint32_t gt, uint32_t kvt, bool first) -> bool {
+                const uint32_t pb = gt & 1;
+                if (!mbar_wait(&p_full[pb], (gt >> 1) & 1, abort_flag, p.err)) return false;
                 if (first && !mbar_wait(o_free, (item_it & 1) ^ 1, abort_flag, p.err)) return false;
                 tc_fence_after();
-                const int s = kvp % kKVStages;
+                const int s = kvt % kKVStages;
                 const uint32_t p_addr = smem_u32(sP + pb * Cfg::kPBytes);
                 const uint32_t v_addr = smem_u32(sV + s * Cfg::kTileBytes);
 #pragma unroll
@@ -196,41 +219,25 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
                     const uint64_t bd = make_sdesc(v_addr + kk * 16 * Cfg::kRowBytes, Cfg::kAtom, Cfg::kAtom, Cfg::kSwz);
                     mma_bf16(tmem + 256 + (kk >> 2) * DH, ad, bd, idesc_o, !(first && (kk & 3) == 0));
                 }
-                mma_commit(o_done);
                 mma_commit(&kv_empty[s]);
                 mma_commit(&p_empty[pb]);
                 return true;
             };
+            // every item has at least one key tile: a sample without active
+            // tokens owns no query tile, and the entry points reject nk < 1
             for (int w = blockIdx.x; w < total && ok; w += gridDim.x, ++item_it) {
                 const Item it = decode_item(p, w);
                 if (!mbar_wait(q_full, item_it & 1, abort_flag, p.err)) break;
                 tc_fence_after();
-                const int nkt = (it.nk + 127) / 128;
-                for (int j = 0; j < nkt; ++j, ++kv_it, ++g) {
-                    const int s = kv_it % kKVStages;
-                    if (!mbar_wait(&kv_full[s], (kv_it / kKVStages) & 1, abort_flag, p.err)) {
-                        ok = false;
-                        break;
-                    }
-                    const uint32_t sb = g & 1;
-                    if (!mbar_wait(&s_empty[sb], ((g >> 1) & 1) ^ 1, abort_flag, p.err)) {
-                        ok = false;
-                        break;
-                    }
-                    tc_fence_after();
-                    const uint32_t k_addr = smem_u32(sK + s * Cfg::kTileBytes);
-#pragma unroll
-                    for (int kk = 0; kk < DH / 16; ++kk)
-                        mma_bf16(tmem + sb * 128, make_sdesc(q_addr + kk * 32, 16, Cfg::kAtom, Cfg::kSwz),
-                                 make_sdesc(k_addr + kk * 32, 16, Cfg::kAtom, Cfg::kSwz), idesc_s, kk > 0);
-                    mma_commit(&s_full[sb]);
-                    if (j == nkt - 1) mma_commit(q_empty);
-                    if (j >= 1 && !issue_pv(g - 1, kv_it - 1, j == 1)) {
-                        ok = false;
-                        break;
-                    }
+                const uint32_t nkt = (uint32_t)((it.nk + 127) / 128);
+                ok = issue_s(g_base, kv_base, nkt == 1);
+                if (ok && nkt > 1) ok = issue_s(g_base + 1, kv_base + 1, nkt == 2);
+                for (uint32_t j = 0; j < nkt && ok; ++j) {
+                    if (j + 2 < nkt && !issue_s(g_base + j + 2, kv_base + j + 2, j + 3 == nkt)) ok = false;
+                    if (ok && !issue_pv(g_base + j, kv_base + j, j == 0)) ok = false;
                 }
-                if (ok && !issue_pv(g - 1, kv_it - 1, nkt == 1)) ok = false;
+                g_base += nkt;
+                kv_base += nkt;
             }
         }
     } else {
@@ -241,6 +248,17 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
         const uint32_t tl = (uint32_t)(q * 32) << 16;
         const uint32_t o_addr = tmem + tl + 256 + half * DH;
         uint32_t g = 0, item_it = 0;
+        // P V completions are awaited strictly in order: tile t on
+        // p_empty[t % 2] with parity (t / 2) % 2.  Tile g awaits P V of g - 2
+        // before it reuses that P buffer, and P V of g + 1 cannot start before
+        // P of g + 1 is written, so no barrier is ever more than one phase
+        // past the softmax's count and a parity wait cannot confuse phases
+        uint32_t pv_seen = 0;  // P V of tiles < pv_seen known complete
+        auto wait_pv_through = [&](uint32_t t) -> bool {
+            for (; pv_seen <= t; ++pv_seen)
+                if (!mbar_wait(&p_empty[pv_seen & 1], (pv_seen >> 1) & 1, abort_flag, p.err)) return false;
+            return true;
+        };
         for (int w = blockIdx.x; w < total; w += gridDim.x, ++item_it) {
             const Item it = decode_item(p, w);
             const int nkt = (it.nk + 127) / 128;
@@ -259,7 +277,8 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
                 tmem_ld32(tmem + tl + sb * 128 + 64 * half + 32, r1);
                 tmem_wait_ld();
                 tc_fence_before();
-                mbar_arrive(&s_empty[sb]);
+                __syncwarp();
+                if (lane == 0) mbar_arrive(&s_empty[sb]);  // one arrival per warp
                 float sv[64];
 #pragma unroll
                 for (int c = 0; c < 32; ++c) {
@@ -282,11 +301,9 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
                 // (warp-uniform: TMEM loads / stores are warp-collective)
                 if (__any_sync(0xffffffffu, mx > m_ref + 8.0f)) {
                     const float m_new = fmaxf(m_ref, mx);
-                    if (j > 0) {  // O holds tiles < j: wait for the last P V, rescale in place
-                        // (the s_full wait above implies the P V of tile g-2 is
-                        // done, so only phase g-1 of o_done can be outstanding)
+                    if (j > 0) {  // O holds tiles < j: wait for their P V, rescale in place
                         const float alpha = exp2_fast(m_ref - m_new);
-                        if (!mbar_wait(o_done, (g - 1) & 1, abort_flag, p.err)) {
+                        if (!wait_pv_through(g - 1)) {
                             ok = false;
                             break;
                         }
@@ -308,7 +325,7 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
                 // a half with no valid key yet keeps m = -inf: subtract 0 instead
                 const float m_use = m_ref == -INFINITY ? 0.f : m_ref;
                 // P[sb] may still be read by the P V MMA of tile g-2
-                if (!mbar_wait(&p_empty[sb], sph ^ 1, abort_flag, p.err)) {
+                if (g >= 2 && !wait_pv_through(g - 2)) {
                     ok = false;
                     break;
                 }
@@ -328,18 +345,15 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
                     u.w = pack_bf16x2(pv[6], pv[7]);
                     *reinterpret_cast<uint4 *>(panel + ((ch ^ (row & 7)) << 4)) = u;
                 }
-                fence_proxy_async_smem();
+                fence_proxy_async_smem();  // every lane orders its own P stores
                 tc_fence_before();
-                mbar_arrive(&p_full[sb]);
+                __syncwarp();
+                if (lane == 0) mbar_arrive(&p_full[sb]);
                 l_run += sum0 + sum1;
             }
             if (!ok) break;
-            // the item's last P V done: read this half's O, release it.  The
-            // s_full wait of the last tile only guarantees the P V of tile g-3,
-            // so up to two o_done phases are outstanding: wait for them in order
-            // (a single parity wait could be satisfied by the older phase).
-            if (!mbar_wait(o_done, (g - 2) & 1, abort_flag, p.err)) break;
-            if (!mbar_wait(o_done, (g - 1) & 1, abort_flag, p.err)) break;
+            // every P V of the item done: read this half's O, release it
+            if (!wait_pv_through(g - 1)) break;
             tc_fence_after();
             float acc[DH];
 #pragma unroll
@@ -351,7 +365,8 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
                 for (int d = 0; d < 32; ++d) acc[d0 + d] = __uint_as_float(r[d]);
             }
             tc_fence_before();
-            mbar_arrive(o_free);
+            __syncwarp();
+            if (lane == 0) mbar_arrive(o_free);
             // combine the two halves of each row:
             // O = (O_0 2^(m_0-m) + O_1 2^(m_1-m)) / (l_0 2^(m_0-m) + l_1 2^(m_1-m))
             float *mine = sComb + row * (DH + 2);

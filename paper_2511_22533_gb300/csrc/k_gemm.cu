@@ -259,8 +259,8 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
         }
         mbar_init(&accf[0], 1);
         mbar_init(&accf[1], 1);
-        mbar_init(&acce[0], 128);
-        mbar_init(&acce[1], 128);
+        mbar_init(&acce[0], 4);  // one arrival per epilogue warp
+        mbar_init(&acce[1], 4);
         mbar_init(drain, 1);
         *abort_flag = 0;
         fence_mbar_init();
@@ -348,7 +348,8 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
             if (U.splits == 1) {
                 epilogue_tile<BN, EPI>(p, tsrc, m0 + row, n0);
                 tc_fence_before();
-                mbar_arrive(&acce[buf]);
+                __syncwarp();
+                if (lane == 0) mbar_arrive(&acce[buf]);
                 continue;
             }
             // split K: store this split's fp32 partial row, free TMEM, and let
@@ -364,7 +365,8 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
                            make_float4(v[4 * q4], v[4 * q4 + 1], v[4 * q4 + 2], v[4 * q4 + 3]));
             }
             tc_fence_before();
-            mbar_arrive(&acce[buf]);
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&acce[buf]);
             const int tile = t % U.tiles;
             __threadfence();
             asm volatile("bar.sync 2, 128;" ::: "memory");
