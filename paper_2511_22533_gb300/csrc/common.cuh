@@ -260,6 +260,40 @@ F3DC_DEV float exp2_fast(float x)
     return y;
 }
 
+// three-input maximum (one instruction on sm_100 and later)
+F3DC_DEV float fmax3(float a, float b, float c)
+{
+    float r;
+    asm("max.f32 %0, %1, %2, %3;" : "=f"(r) : "f"(a), "f"(b), "f"(c));
+    return r;
+}
+
+// packed pairs of fp32 for the paired FMA / add instructions of sm_100+
+struct f32x2 {
+    float x, y;
+};
+F3DC_DEV f32x2 ffma2(f32x2 a, f32x2 b, f32x2 c)
+{
+    uint64_t pa, pb, pc, d;
+    asm("mov.b64 %0, {%1, %2};" : "=l"(pa) : "f"(a.x), "f"(a.y));
+    asm("mov.b64 %0, {%1, %2};" : "=l"(pb) : "f"(b.x), "f"(b.y));
+    asm("mov.b64 %0, {%1, %2};" : "=l"(pc) : "f"(c.x), "f"(c.y));
+    asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(d) : "l"(pa), "l"(pb), "l"(pc));
+    f32x2 r;
+    asm("mov.b64 {%0, %1}, %2;" : "=f"(r.x), "=f"(r.y) : "l"(d));
+    return r;
+}
+F3DC_DEV f32x2 fadd2(f32x2 a, f32x2 b)
+{
+    uint64_t pa, pb, d;
+    asm("mov.b64 %0, {%1, %2};" : "=l"(pa) : "f"(a.x), "f"(a.y));
+    asm("mov.b64 %0, {%1, %2};" : "=l"(pb) : "f"(b.x), "f"(b.y));
+    asm("add.f32x2 %0, %1, %2;" : "=l"(d) : "l"(pa), "l"(pb));
+    f32x2 r;
+    asm("mov.b64 {%0, %1}, %2;" : "=f"(r.x), "=f"(r.y) : "l"(d));
+    return r;
+}
+
 F3DC_DEV float gelu_tanh(float x)
 {
     const float k0 = 0.7978845608028654f;  // sqrt(2/pi)

