@@ -11,21 +11,27 @@
 //   warp 0     TMA producer: Q tile once per item, K / V tiles of 128 keys
 //              into a 4-deep ring
 //   warp 1     TMEM allocator + tcgen05.mma issuer:
-//                S_j = Q K_j^T              (M=128, N=128, K=dh) -> TMEM S[j%2]
-//                O_h += P_j,h V_j,h  h=0,1  (M=128, N=dh,  K=64) -> TMEM O_h
+//                S_j = Q K_j^T     (M=128, N=128, K=dh)  -> TMEM S[j%2]
+//                O_e += P_j V_j    (M=128, N=dh, K=128)  -> TMEM O_e, e = j%2,
+//                                   with P_j read from TMEM P_e
 //              S runs two tiles ahead: S_(j+2) is issued as soon as the
 //              softmax has read S_j, before P V of tile j, so the scores of
 //              the next tiles are ready whenever the softmax gets to them
 //   warps 2-9  softmax, two threads per query row (TMEM lane = row): the
-//              thread of half h owns keys [64h, 64h + 64) of every tile and
-//              runs its own online softmax over them, writing
-//              P = exp2(S scale - m) as bf16 into its 64-key 128B-swizzled
-//              panel (the K-major A operand of its P V MMA).  O stays in TMEM
-//              for the whole item; the reference max m is only raised (and O,
-//              l rescaled in place) when a tile's max exceeds it by more than
-//              2^8, so most tiles need no O traffic at all.  The two halves
-//              of a row are combined once per work item.  Two softmax warps per
-//              SM sub-partition hide each other's exponent and TMEM latencies.
+//              thread of parity e owns the key tiles j with j%2 == e (all
+//              128 keys of each) and runs its own online softmax over them,
+//              writing P = exp2(S scale - m) as bf16 pairs into TMEM P_e
+//              (the A operand of its P V MMA, read straight from TMEM, so P
+//              costs no shared-memory bandwidth).
+//              O_e stays in TMEM for the whole item; the reference max m is
+//              only raised (and O_e, l rescaled in place) when a tile's max
+//              exceeds it by more than 2^8, so most tiles need no O traffic.
+//              The two parities of a row are combined once per work item.
+//              The exponent unit (16 results per clock per SM) bounds the
+//              softmax; because the two warps of an SM sub-partition work on
+//              different tiles, one warp's TMEM load, maximum and barrier
+//              phases overlap the other's exponents instead of leaving the
+//              unit idle.
 // V is the MN-major B operand of the P V MMA straight from its row-major
 // TMA tile.  Keys beyond a sample's count are masked to -inf before the
 // exponent; padding rows are finite by construction, so 0 * pad = 0.
@@ -47,12 +53,13 @@ struct AttnCfg {
     static constexpr int kTileBytes = 128 * kRowBytes;  // Q, K or V tile
     static constexpr uint32_t kAtom = 8 * kRowBytes;    // 8-row swizzle atom
     static constexpr uint32_t kSwz = DH == 64 ? kSwizzle128 : kSwizzle64;
-    static constexpr int kPPanel = 128 * 128;           // 64 keys x 128 rows x 2 B
-    static constexpr int kPBytes = 2 * kPPanel;
-    static constexpr int kCombineBytes = 128 * (DH + 2) * 4;  // half-1 (m, l, O) per row, aliases P
-    static_assert(kCombineBytes <= 2 * kPBytes, "combine scratch must fit in the P buffers");
-    static constexpr size_t kSmem = 1024 + kTileBytes * (1 + 2 * kKVStages) + 2 * kPBytes + 512;
-    static constexpr uint32_t kTmemCols = 512;          // S0 S1 | O_0 O_1
+    static constexpr int kCombineBytes = 128 * DH * 4;  // parity-1 O, one row per softmax row
+    static constexpr size_t kSmem = 1024 + kTileBytes * (1 + 2 * kKVStages) + kCombineBytes + 512 + 128 * 8;
+    // TMEM columns: S_0 S_1 (fp32, 128 each) | O_0 O_1 (fp32, DH each) |
+    // P_0 P_1 (bf16 pairs, 64 each)
+    static constexpr uint32_t kColO = 256, kColP = 256 + 2 * DH;
+    static constexpr uint32_t kTmemCols = 512;
+    static_assert(kColP + 128 <= kTmemCols, "TMEM layout");
 };
 
 struct Item {
@@ -101,18 +108,20 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
     uint8_t *sQ = smem;
     uint8_t *sK = sQ + Cfg::kTileBytes;
     uint8_t *sV = sK + kKVStages * Cfg::kTileBytes;
-    uint8_t *sP = sV + kKVStages * Cfg::kTileBytes;
-    // the end-of-item combine runs when every P V of the item is done, so
-    // its scratch can live in the P buffers
-    float *sComb = reinterpret_cast<float *>(sP);
-    uint64_t *bars = reinterpret_cast<uint64_t *>(sP + 2 * Cfg::kPBytes);
+    // the end-of-item combine hands parity 1's O and (m, l) to parity 0
+    float *sComb = reinterpret_cast<float *>(sV + kKVStages * Cfg::kTileBytes);
+    uint64_t *bars = reinterpret_cast<uint64_t *>(reinterpret_cast<uint8_t *>(sComb) + Cfg::kCombineBytes);
+    float2 *sML = reinterpret_cast<float2 *>(reinterpret_cast<uint8_t *>(bars) + 512);
     uint64_t *q_full = bars, *q_empty = bars + 1;
     uint64_t *kv_full = bars + 2, *kv_empty = kv_full + kKVStages;
-    uint64_t *s_full = kv_empty + kKVStages, *s_empty = s_full + 2;
-    uint64_t *p_full = s_empty + 2, *p_empty = p_full + 2;
-    // p_empty[t % 2] completes once per P V of (global) tile index t and
-    // doubles as the "O holds tiles <= t" signal; o_free completes once per item
-    uint64_t *o_free = p_empty + 2;
+    // Key tile g (counted over the CTA's whole run) always sits in K/V stage
+    // g % kKVStages, so kv_empty[g % kKVStages] completes exactly when P V of
+    // tile g does: the producer reuses the stage on it, and the softmax takes
+    // it as "O_(g%2) holds tile g and P_(g%2) is free".  p_full[e] (four
+    // softmax warps of parity e) certifies P of the tile and that its S was
+    // read, so it also frees S buffer e.  o_free completes once per item.
+    uint64_t *s_full = kv_empty + kKVStages, *p_full = s_full + 2;
+    uint64_t *o_free = p_full + 2;
     uint64_t *drain = o_free + 1;
     uint32_t *tmem_holder = reinterpret_cast<uint32_t *>(drain + 1);
     volatile int *abort_flag = reinterpret_cast<volatile int *>(tmem_holder + 1);
@@ -128,11 +137,9 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
             mbar_init(&kv_full[s], 1);
             mbar_init(&kv_empty[s], 1);
         }
-        for (int s = 0; s < 2; ++s) {
+        for (int s = 0; s < 2; ++s) {  // one S / P buffer per tile parity, four warps each
             mbar_init(&s_full[s], 1);
-            mbar_init(&s_empty[s], kSoftmaxWarps);
-            mbar_init(&p_full[s], kSoftmaxWarps);
-            mbar_init(&p_empty[s], 1);
+            mbar_init(&p_full[s], kSoftmaxWarps / 2);
         }
         mbar_init(o_free, kSoftmaxWarps);
         mbar_init(drain, 1);
@@ -179,217 +186,265 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
         }
     } else if (warp == 1) {
         // ------------------------------------------------ MMA issuer
+        // Barrier reads take a long time even when the phase is complete, so
+        // each tile tests its two barriers back to back (one exposed
+        // latency) and takes the bounded wait only if a test fails; the
+        // steady-state loop carries no other branches.
         if (lane == 0) {
             constexpr uint32_t idesc_s = make_idesc_bf16(128, 128, 0, 0);
             constexpr uint32_t idesc_o = make_idesc_bf16(128, DH, 0, 1);
-            const uint32_t q_addr = smem_u32(sQ);
-            uint32_t kv_base = 0, g_base = 0, item_it = 0;  // global tile / kv-stage counters
-            bool ok = true;
-            // S for tile j of the item: needs its K tile and a free S buffer
-            // (the softmax has read S of tile j-2)
-            auto issue_s = [&](uint32_t gt, uint32_t kvt, bool last) -> bool {
-                const int s = kvt % kKVStages;
-                const uint32_t sb = gt & 1;
-                if (!mbar_wait(&kv_full[s], (kvt / kKVStages) & 1, abort_flag, p.err)) return false;
-                if (!mbar_wait(&s_empty[sb], ((gt >> 1) & 1) ^ 1, abort_flag, p.err)) return false;
-                tc_fence_after();
-                const uint32_t k_addr = smem_u32(sK + s * Cfg::kTileBytes);
+            // descriptors of the stage bases; a K step of 16 elements inside a
+            // 128B / 64B swizzle atom advances the start address by 32 bytes,
+            // i.e. the descriptor by 2
+            const uint64_t q_desc = make_sdesc(smem_u32(sQ), 16, Cfg::kAtom, Cfg::kSwz);
+            const uint64_t k_desc0 = make_sdesc(smem_u32(sK), 16, Cfg::kAtom, Cfg::kSwz);
+            const uint64_t v_desc0 = make_sdesc(smem_u32(sV), Cfg::kAtom, Cfg::kAtom, Cfg::kSwz);
+            constexpr uint64_t kStageStep = Cfg::kTileBytes >> 4, kVRowStep = (16 * Cfg::kRowBytes) >> 4;
+            auto s_mmas = [&](uint32_t gt) {  // S_gt = Q K_gt^T into S buffer gt % 2
+                const uint64_t kd = k_desc0 + (gt % kKVStages) * kStageStep;
 #pragma unroll
                 for (int kk = 0; kk < DH / 16; ++kk)
-                    mma_bf16(tmem + sb * 128, make_sdesc(q_addr + kk * 32, 16, Cfg::kAtom, Cfg::kSwz),
-                             make_sdesc(k_addr + kk * 32, 16, Cfg::kAtom, Cfg::kSwz), idesc_s, kk > 0);
-                mma_commit(&s_full[sb]);
-                if (last) mma_commit(q_empty);
-                return true;
+                    mma_bf16(tmem + (gt & 1) * 128, q_desc + 2 * kk, kd + 2 * kk, idesc_s, kk > 0);
+                mma_commit(&s_full[gt & 1]);
             };
-            // O_h (+)= P_h V_h for tile gt; the item's first tile overwrites O,
-            // after the softmax has read the previous item's result
-            auto issue_pv = [&](uint32_t gt, uint32_t kvt, bool first) -> bool {
+            // O_e (+)= P_e V for tile gt of parity e = gt % 2, P_e read from
+            // TMEM (8 columns per 16 keys); `fresh` overwrites O_e (the item's
+            // first tile of each parity)
+            auto pv_mmas = [&](uint32_t gt, bool fresh) {
                 const uint32_t pb = gt & 1;
-                if (!mbar_wait(&p_full[pb], (gt >> 1) & 1, abort_flag, p.err)) return false;
-                if (first && !mbar_wait(o_free, (item_it & 1) ^ 1, abort_flag, p.err)) return false;
-                tc_fence_after();
-                const int s = kvt % kKVStages;
-                const uint32_t p_addr = smem_u32(sP + pb * Cfg::kPBytes);
-                const uint32_t v_addr = smem_u32(sV + s * Cfg::kTileBytes);
+                const uint64_t vd = v_desc0 + (gt % kKVStages) * kStageStep;
 #pragma unroll
-                for (int kk = 0; kk < 8; ++kk) {  // keys 16kk..16kk+15, half kk / 4
-                    const uint64_t ad = make_sdesc(p_addr + (kk >> 2) * Cfg::kPPanel + (kk & 3) * 32, 16, 1024,
-                                                   kSwizzle128);
-                    const uint64_t bd = make_sdesc(v_addr + kk * 16 * Cfg::kRowBytes, Cfg::kAtom, Cfg::kAtom, Cfg::kSwz);
-                    mma_bf16(tmem + 256 + (kk >> 2) * DH, ad, bd, idesc_o, !(first && (kk & 3) == 0));
-                }
-                mma_commit(&kv_empty[s]);
-                mma_commit(&p_empty[pb]);
-                return true;
+                for (int kk = 0; kk < 8; ++kk)  // keys 16kk..16kk+15
+                    mma_bf16_ts(tmem + Cfg::kColO + pb * DH, tmem + Cfg::kColP + pb * 64 + kk * 8,
+                                vd + kk * kVRowStep, idesc_o, !(fresh && kk == 0));
+                mma_commit(&kv_empty[gt % kKVStages]);
             };
+            auto kv_ready = [&](uint32_t gt) { return mbar_test(&kv_full[gt % kKVStages], (gt / kKVStages) & 1); };
+            auto kv_wait = [&](uint32_t gt) {
+                return mbar_wait(&kv_full[gt % kKVStages], (gt / kKVStages) & 1, abort_flag, p.err);
+            };
+            auto p_ready = [&](uint32_t gt) { return mbar_test(&p_full[gt & 1], (gt >> 1) & 1); };
+            auto p_wait = [&](uint32_t gt) { return mbar_wait(&p_full[gt & 1], (gt >> 1) & 1, abort_flag, p.err); };
+            uint32_t g = 0, item_it = 0;  // global key tile at the start of the item
+            bool ok = true;
             // every item has at least one key tile: a sample without active
             // tokens owns no query tile, and the entry points reject nk < 1
             for (int w = blockIdx.x; w < total && ok; w += gridDim.x, ++item_it) {
                 const Item it = decode_item(p, w);
-                if (!mbar_wait(q_full, item_it & 1, abort_flag, p.err)) break;
-                tc_fence_after();
                 const uint32_t nkt = (uint32_t)((it.nk + 127) / 128);
-                ok = issue_s(g_base, kv_base, nkt == 1);
-                if (ok && nkt > 1) ok = issue_s(g_base + 1, kv_base + 1, nkt == 2);
-                for (uint32_t j = 0; j < nkt && ok; ++j) {
-                    if (j + 2 < nkt && !issue_s(g_base + j + 2, kv_base + j + 2, j + 3 == nkt)) ok = false;
-                    if (ok && !issue_pv(g_base + j, kv_base + j, j == 0)) ok = false;
+                // S of the first two tiles: their S buffers were freed by the
+                // previous item's P (waited on before its P V)
+                if (!mbar_wait(q_full, item_it & 1, abort_flag, p.err)) break;
+                if (!kv_wait(g)) break;
+                tc_fence_after();
+                s_mmas(g);
+                if (nkt > 1) {
+                    if (!kv_wait(g + 1)) break;
+                    tc_fence_after();
+                    s_mmas(g + 1);
                 }
-                g_base += nkt;
-                kv_base += nkt;
+                // O_0 / O_1 are overwritten by this item's first P V: the
+                // softmax must have read the previous item's result
+                if (!mbar_wait(o_free, (item_it & 1) ^ 1, abort_flag, p.err)) break;
+                // steady state: P_j ready -> S_(j+2), P V_j
+                uint32_t j = 0;
+                for (; j + 2 < nkt; ++j) {
+                    const uint32_t gt = g + j;
+                    const bool r = p_ready(gt) & kv_ready(gt + 2);
+                    if (!r && !(p_wait(gt) && kv_wait(gt + 2))) {
+                        ok = false;
+                        break;
+                    }
+                    tc_fence_after();
+                    s_mmas(gt + 2);
+                    pv_mmas(gt, j < 2);
+                }
+                if (!ok) break;
+                mma_commit(q_empty);  // every S of the item issued: Q may be replaced
+                for (; j < nkt; ++j) {
+                    const uint32_t gt = g + j;
+                    if (!p_ready(gt) && !p_wait(gt)) {
+                        ok = false;
+                        break;
+                    }
+                    tc_fence_after();
+                    pv_mmas(gt, j < 2);
+                }
+                g += nkt;
             }
         }
     } else {
         // ------------------------------------------------ softmax warps
-        const int q = warp & 3;                  // TMEM lane quarter of this warp
-        const int half = (warp - 2) >> 2;        // keys [64 half, 64 half + 64) of each tile
+        const int q = warp & 3;                // TMEM lane quarter of this warp
+        const int par = (warp - 2) >> 2;       // key tiles g with g % 2 == par
         const int row = q * 32 + lane;
         const uint32_t tl = (uint32_t)(q * 32) << 16;
-        const uint32_t o_addr = tmem + tl + 256 + half * DH;
-        uint32_t g = 0, item_it = 0;
-        // P V completions are awaited strictly in order: tile t on
-        // p_empty[t % 2] with parity (t / 2) % 2.  Tile g awaits P V of g - 2
-        // before it reuses that P buffer, and P V of g + 1 cannot start before
-        // P of g + 1 is written, so no barrier is ever more than one phase
-        // past the softmax's count and a parity wait cannot confuse phases
-        uint32_t pv_seen = 0;  // P V of tiles < pv_seen known complete
-        auto wait_pv_through = [&](uint32_t t) -> bool {
-            for (; pv_seen <= t; ++pv_seen)
-                if (!mbar_wait(&p_empty[pv_seen & 1], (pv_seen >> 1) & 1, abort_flag, p.err)) return false;
-            return true;
-        };
+        const uint32_t s_addr = tmem + tl + par * 128;
+        const uint32_t o_addr = tmem + tl + Cfg::kColO + par * DH;
+        const uint32_t p_addr = tmem + tl + Cfg::kColP + par * 64;
+        uint32_t g = 0, item_it = 0;  // global key-tile counter at the start of the item
+        // s_full[par] completes once per tile of this parity, in tile order
+        // (tile t with parity (t / 2) % 2); P V of tile t is awaited on
+        // kv_empty[t % 4] with parity (t / 4) % 2.  A warp waits for P V of
+        // its previous tile (t - 2) before it writes P again, and P V of its
+        // next tile cannot start before that, so no barrier it reads is ever
+        // more than one phase ahead of it.
         for (int w = blockIdx.x; w < total; w += gridDim.x, ++item_it) {
             const Item it = decode_item(p, w);
             const int nkt = (it.nk + 127) / 128;
             float m_ref = -INFINITY, l_run = 0.f;
-            bool ok = true;
-            for (int j = 0; j < nkt; ++j, ++g) {
-                const uint32_t sb = g & 1, sph = (g >> 1) & 1;
-                if (!mbar_wait(&s_full[sb], sph, abort_flag, p.err)) {
+            bool ok = true, any = false;
+            uint32_t g_last = 0;
+            for (int j = (int)((par - g) & 1); j < nkt; j += 2) {
+                const uint32_t gt = g + (uint32_t)j, ph = (gt >> 1) & 1;
+                if (!mbar_wait(&s_full[par], ph, abort_flag, p.err)) {
                     ok = false;
                     break;
                 }
                 tc_fence_after();
-                const int valid = min(128, it.nk - j * 128) - 64 * half;  // valid keys of this half
-                uint32_t r0[32], r1[32];
-                tmem_ld32(tmem + tl + sb * 128 + 64 * half, r0);
-                tmem_ld32(tmem + tl + sb * 128 + 64 * half + 32, r1);
-                tmem_wait_ld();
-                tc_fence_before();
-                __syncwarp();
-                if (lane == 0) mbar_arrive(&s_empty[sb]);  // one arrival per warp
-                float sv[64];
+                // pass 1: the tile's maximum (S stays in TMEM for pass 2)
+                const int valid = it.nk - j * 128;  // < 128 only on the last, ragged key tile
+                float mx4[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
 #pragma unroll
-                for (int c = 0; c < 32; ++c) {
-                    sv[c] = __uint_as_float(r0[c]);
-                    sv[32 + c] = __uint_as_float(r1[c]);
-                }
-                if (valid < 64) {  // only the last key tile of a sequence is ragged
+                for (int hb = 0; hb < 2; ++hb) {  // two halves of 64 keys
+                    uint32_t r0[32], r1[32];
+                    tmem_ld32(s_addr + 64 * hb, r0);
+                    tmem_ld32(s_addr + 64 * hb + 32, r1);
+                    tmem_wait_ld();
+                    float sv[64];
 #pragma unroll
-                    for (int c = 0; c < 64; ++c)
-                        if (c >= valid) sv[c] = -INFINITY;
-                }
-                // four independent chains of three-input maxima
-                float mx4[4];
+                    for (int c = 0; c < 32; ++c) {
+                        sv[c] = __uint_as_float(r0[c]);
+                        sv[32 + c] = __uint_as_float(r1[c]);
+                    }
+                    if (valid < 128) {
 #pragma unroll
-                for (int c = 0; c < 4; ++c) mx4[c] = fmaxf(sv[c], sv[4 + c]);
+                        for (int c = 0; c < 64; ++c)
+                            if (64 * hb + c >= valid) sv[c] = -INFINITY;
+                    }
+                    // four independent chains of three-input maxima
 #pragma unroll
-                for (int c = 8; c < 64; c += 8) {
+                    for (int c = 0; c < 64; c += 8) {
 #pragma unroll
-                    for (int e = 0; e < 4; ++e) mx4[e] = fmax3(mx4[e], sv[c + e], sv[c + 4 + e]);
+                        for (int e = 0; e < 4; ++e) mx4[e] = fmax3(mx4[e], sv[c + e], sv[c + 4 + e]);
+                    }
                 }
                 const float mx = fmax3(mx4[0], mx4[1], fmaxf(mx4[2], mx4[3])) * p.scale_log2;
                 // raise the reference max only when it grew by more than 2^8
-                // (warp-uniform: TMEM loads / stores are warp-collective)
-                if (__any_sync(0xffffffffu, mx > m_ref + 8.0f)) {
+                // (warp-uniform: TMEM loads / stores are warp-collective); O
+                // and l are rescaled once P V of this parity's previous tile
+                // is done
+                const bool raise = __any_sync(0xffffffffu, mx > m_ref + 8.0f);
+                float alpha = 1.f;
+                if (raise) {
                     const float m_new = fmaxf(m_ref, mx);
-                    if (j > 0) {  // O holds tiles < j: wait for their P V, rescale in place
-                        const float alpha = exp2_fast(m_ref - m_new);
-                        if (!wait_pv_through(g - 1)) {
-                            ok = false;
-                            break;
-                        }
-                        tc_fence_after();
-#pragma unroll
-                        for (int d0 = 0; d0 < DH; d0 += 32) {
-                            uint32_t r[32];
-                            tmem_ld32(o_addr + d0, r);
-                            tmem_wait_ld();
-#pragma unroll
-                            for (int d = 0; d < 32; ++d) r[d] = __float_as_uint(__uint_as_float(r[d]) * alpha);
-                            tmem_st32(o_addr + d0, r);
-                        }
-                        tmem_wait_st();
-                        l_run *= alpha;
-                    }
+                    alpha = exp2_fast(m_ref - m_new);
                     m_ref = m_new;
                 }
-                // a half with no valid key yet keeps m = -inf: subtract 0 instead
                 const float m_use = m_ref == -INFINITY ? 0.f : m_ref;
-                // P[sb] may still be read by the P V MMA of tile g-2
-                if (g >= 2 && !wait_pv_through(g - 2)) {
+                // P_par and O_par: P V of this parity's previous tile must be done
+                if (gt >= 2 && !mbar_wait(&kv_empty[(gt - 2) % kKVStages], ((gt - 2) / kKVStages) & 1, abort_flag, p.err)) {
                     ok = false;
                     break;
                 }
-                // exponent arguments and row sums two lanes per paired instruction
+                if (raise && any) {  // O_par holds this parity's earlier tiles: rescale in place
+                    tc_fence_after();
+#pragma unroll
+                    for (int d0 = 0; d0 < DH; d0 += 16) {
+                        uint32_t r[16];
+                        tmem_ld16(o_addr + d0, r);
+                        tmem_wait_ld();
+#pragma unroll
+                        for (int d = 0; d < 16; ++d) r[d] = __float_as_uint(__uint_as_float(r[d]) * alpha);
+                        tmem_st16(o_addr + d0, r);
+                    }
+                    l_run *= alpha;
+                }
+                // pass 2: exponent arguments and row sums two lanes per paired
+                // instruction; P goes to TMEM as bf16 pairs (keys 2c, 2c+1
+                // in column c, the lower key in the low half)
                 f32x2 sum0 = {0.f, 0.f}, sum1 = {0.f, 0.f};
                 const f32x2 sc2 = {p.scale_log2, p.scale_log2}, nm2 = {-m_use, -m_use};
-                uint8_t *panel = sP + sb * Cfg::kPBytes + half * Cfg::kPPanel + row * 128;
 #pragma unroll
-                for (int ch = 0; ch < 8; ++ch) {  // 16-byte chunk ch of the 128-byte row
-                    float pv[8];
+                for (int hb = 0; hb < 2; ++hb) {  // keys [64 hb, 64 hb + 64) -> columns [32 hb, 32 hb + 32)
+                    float sv[64];
+                    {
+                        uint32_t r0[32], r1[32];
+                        tmem_ld32(s_addr + 64 * hb, r0);
+                        tmem_ld32(s_addr + 64 * hb + 32, r1);
+                        tmem_wait_ld();
 #pragma unroll
-                    for (int e = 0; e < 8; e += 2) {
-                        const f32x2 x = ffma2({sv[ch * 8 + e], sv[ch * 8 + e + 1]}, sc2, nm2);
-                        pv[e] = exp2_fast(x.x);
-                        pv[e + 1] = exp2_fast(x.y);
+                        for (int c = 0; c < 32; ++c) {
+                            sv[c] = __uint_as_float(r0[c]);
+                            sv[32 + c] = __uint_as_float(r1[c]);
+                        }
                     }
-                    sum0 = fadd2(sum0, {pv[0], pv[1]});
-                    sum1 = fadd2(sum1, {pv[2], pv[3]});
-                    sum0 = fadd2(sum0, {pv[4], pv[5]});
-                    sum1 = fadd2(sum1, {pv[6], pv[7]});
-                    uint4 u;
-                    u.x = pack_bf16x2(pv[0], pv[1]);
-                    u.y = pack_bf16x2(pv[2], pv[3]);
-                    u.z = pack_bf16x2(pv[4], pv[5]);
-                    u.w = pack_bf16x2(pv[6], pv[7]);
-                    *reinterpret_cast<uint4 *>(panel + ((ch ^ (row & 7)) << 4)) = u;
+                    if (valid < 128) {
+#pragma unroll
+                        for (int c = 0; c < 64; ++c)
+                            if (64 * hb + c >= valid) sv[c] = -INFINITY;
+                    }
+                    uint32_t pw[32];
+#pragma unroll
+                    for (int c = 0; c < 32; c += 2) {
+                        const int k0 = 2 * c;
+                        const f32x2 x0 = ffma2({sv[k0], sv[k0 + 1]}, sc2, nm2);
+                        const f32x2 x1 = ffma2({sv[k0 + 2], sv[k0 + 3]}, sc2, nm2);
+                        const f32x2 e0 = {exp2_fast(x0.x), exp2_fast(x0.y)};
+                        const f32x2 e1 = {exp2_fast(x1.x), exp2_fast(x1.y)};
+                        sum0 = fadd2(sum0, e0);
+                        sum1 = fadd2(sum1, e1);
+                        pw[c] = pack_bf16x2(e0.x, e0.y);
+                        pw[c + 1] = pack_bf16x2(e1.x, e1.y);
+                    }
+                    tmem_st32(p_addr + 32 * hb, pw);
                 }
-                fence_proxy_async_smem();  // every lane orders its own P stores
-                tc_fence_before();
-                __syncwarp();
-                if (lane == 0) mbar_arrive(&p_full[sb]);
+                tmem_wait_st();
                 l_run += (sum0.x + sum0.y) + (sum1.x + sum1.y);
+                tc_fence_before();  // P (and a rescaled O) written before P V may start
+                __syncwarp();
+                if (lane == 0) mbar_arrive(&p_full[par]);
+                any = true;
+                g_last = gt;
             }
+            g += (uint32_t)nkt;
             if (!ok) break;
-            // every P V of the item done: read this half's O, release it
-            if (!wait_pv_through(g - 1)) break;
-            tc_fence_after();
+            // every P V of this parity done: read O_par, release it (a parity
+            // without tiles in this item contributes m = -inf, l = 0, O = 0)
             float acc[DH];
 #pragma unroll
-            for (int d0 = 0; d0 < DH; d0 += 32) {
-                uint32_t r[32];
-                tmem_ld32(o_addr + d0, r);
-                tmem_wait_ld();
+            for (int d = 0; d < DH; ++d) acc[d] = 0.f;
+            if (any) {
+                if (!mbar_wait(&kv_empty[g_last % kKVStages], (g_last / kKVStages) & 1, abort_flag, p.err)) break;
+                tc_fence_after();
 #pragma unroll
-                for (int d = 0; d < 32; ++d) acc[d0 + d] = __uint_as_float(r[d]);
+                for (int d0 = 0; d0 < DH; d0 += 32) {
+                    uint32_t r[32];
+                    tmem_ld32(o_addr + d0, r);
+                    tmem_wait_ld();
+#pragma unroll
+                    for (int d = 0; d < 32; ++d) acc[d0 + d] = __uint_as_float(r[d]);
+                }
             }
             tc_fence_before();
             __syncwarp();
             if (lane == 0) mbar_arrive(o_free);
-            // combine the two halves of each row:
+            // combine the two parities of each row:
             // O = (O_0 2^(m_0-m) + O_1 2^(m_1-m)) / (l_0 2^(m_0-m) + l_1 2^(m_1-m))
-            float *mine = sComb + row * (DH + 2);
-            if (half == 1) {
-                mine[0] = m_ref;
-                mine[1] = l_run;
+            // parity 1's O: float4 d4 of row r at r * DH + 4 (d4 ^ (r % (DH / 4))),
+            // so a warp's row-per-lane accesses hit distinct banks
+            constexpr int kV4 = DH / 4;
+            float4 *mine = reinterpret_cast<float4 *>(sComb + row * DH);
+            if (par == 1) {
+                sML[row] = make_float2(m_ref, l_run);
 #pragma unroll
-                for (int d = 0; d < DH; ++d) mine[2 + d] = acc[d];
+                for (int d4 = 0; d4 < kV4; ++d4)
+                    mine[d4 ^ (row & (kV4 - 1))] = make_float4(acc[4 * d4], acc[4 * d4 + 1], acc[4 * d4 + 2], acc[4 * d4 + 3]);
             }
             asm volatile("bar.sync 1, %0;" ::"n"(kSoftmaxThreads) : "memory");
-            if (half == 0) {
-                const float m1 = mine[0], l1 = mine[1];
+            if (par == 0) {
+                const float2 ml1 = sML[row];
+                const float m1 = ml1.x, l1 = ml1.y;
                 const float m = fmaxf(m_ref, m1);
                 const float a0 = exp2_fast(m_ref - m), a1 = exp2_fast(m1 - m);
                 const float inv = 1.0f / (l_run * a0 + l1 * a1);
@@ -398,9 +453,11 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
                     uint4 *dst = reinterpret_cast<uint4 *>(p.out + (size_t)orow * p.ldo + it.h * DH);
 #pragma unroll
                     for (int d = 0; d < DH; d += 8) {
+                        const float4 b0 = mine[(d / 4) ^ (row & (kV4 - 1))], b1 = mine[(d / 4 + 1) ^ (row & (kV4 - 1))];
+                        const float ob[8] = {b0.x, b0.y, b0.z, b0.w, b1.x, b1.y, b1.z, b1.w};
                         float o[8];
 #pragma unroll
-                        for (int e = 0; e < 8; ++e) o[e] = (acc[d + e] * a0 + mine[2 + d + e] * a1) * inv;
+                        for (int e = 0; e < 8; ++e) o[e] = (acc[d + e] * a0 + ob[e] * a1) * inv;
                         uint4 u;
                         u.x = pack_bf16x2(o[0], o[1]);
                         u.y = pack_bf16x2(o[2], o[3]);
