@@ -135,6 +135,33 @@ F3DC_DEV void tma_load_2d(void *smem_dst, const CUtensorMap *map, int x, int y, 
         : "memory");
 }
 
+// Tiled TMA store of a shared-memory box to global memory (bulk-group
+// completion), and the same as an element-wise fp32 add into global memory.
+// Coordinates: x = innermost (column), y = row; the box is clipped at the
+// tensor's extent.
+F3DC_DEV void tma_store_2d(const CUtensorMap *map, const void *smem_src, int x, int y)
+{
+    asm volatile("cp.async.bulk.tensor.2d.global.shared::cta.bulk_group [%0, {%1, %2}], [%3];" ::"l"((uint64_t)map),
+                 "r"(x), "r"(y), "r"(smem_u32(smem_src))
+                 : "memory");
+}
+F3DC_DEV void tma_reduce_add_2d(const CUtensorMap *map, const void *smem_src, int x, int y)
+{
+    asm volatile("cp.reduce.async.bulk.tensor.2d.global.shared::cta.add.tile.bulk_group [%0, {%1, %2}], [%3];" ::"l"(
+                     (uint64_t)map),
+                 "r"(x), "r"(y), "r"(smem_u32(smem_src))
+                 : "memory");
+}
+F3DC_DEV void bulk_commit() { asm volatile("cp.async.bulk.commit_group;" ::: "memory"); }
+// at most N committed bulk groups may still be reading their shared-memory source
+template <int N>
+F3DC_DEV void bulk_wait_read()
+{
+    asm volatile("cp.async.bulk.wait_group.read %0;" ::"n"(N) : "memory");
+}
+// every committed bulk group complete (writes performed)
+F3DC_DEV void bulk_wait_all() { asm volatile("cp.async.bulk.wait_group 0;" ::: "memory"); }
+
 // Orders this thread's generic-proxy shared-memory writes before later
 // async-proxy (tensor core / TMA) reads of the same memory.
 F3DC_DEV void fence_proxy_async_smem() { asm volatile("fence.proxy.async.shared::cta;" ::: "memory"); }

@@ -13,7 +13,11 @@
 //              two accumulator buffers so the epilogue of tile i overlaps
 //              the MMAs of tile i+1
 //   warps 2-5  epilogue: tcgen05.ld (thread = row), fused bias / GELU /
-//              per-head RMSNorm / gated fp32 residual, global stores
+//              per-head RMSNorm / gated fp32 residual; each 128-row chunk
+//              of 32 bf16 (or 16 fp32) columns is staged in 64B-swizzled
+//              shared memory (three buffers) and written by one TMA tensor
+//              store (residual: TMA fp32 reduce-add into x), so the output
+//              leaves in whole rows instead of one 16-byte piece per thread
 // Tiles are walked m-fastest so the CTAs in flight share weight tiles in L2.
 // The tile count can come from device memory (the step's row plan), so the
 // same launch serves any number of active tokens.
@@ -32,13 +36,18 @@ constexpr int kGemmThreads = 192;
 constexpr int kBK = 64;
 constexpr int kAStage = 128 * kBK * 2;
 
+// output staging: 128 rows x 64 bytes (32 bf16 or 16 fp32 columns)
+constexpr int kOutChunkBytes = 128 * 64;
+constexpr int kOutBufs = 3;
+
 template <int BN>
 struct GemmCfg {
     static constexpr int kBStage = BN * kBK * 2;
     static constexpr int kStages = BN == 256 ? 4 : (BN == 128 ? 6 : 8);
     static constexpr uint32_t kTmemCols = 2 * BN;
     static constexpr size_t kBarBytes = 256;
-    static constexpr size_t kSmem = 1024 + (size_t)kStages * (kAStage + kBStage) + kBarBytes;
+    static constexpr size_t kSmem =
+        1024 + (size_t)kStages * (kAStage + kBStage) + (size_t)kOutBufs * kOutChunkBytes + kBarBytes;
 };
 
 F3DC_DEV bool mbar_wait_bounded(uint64_t *bar, uint32_t parity, uint64_t ns)
@@ -66,20 +75,6 @@ F3DC_DEV void load_bias32(const bf16 *bias, int col, float (&b)[32])
             b[q * 8 + 2 * j] = bf16_bits_to_f32(w[j] & 0xFFFFu);
             b[q * 8 + 2 * j + 1] = bf16_bits_to_f32(w[j] >> 16);
         }
-    }
-}
-
-F3DC_DEV void store_bf16x32(bf16 *dst, const float *v)
-{
-    uint4 *p = reinterpret_cast<uint4 *>(dst);
-#pragma unroll
-    for (int q = 0; q < 4; ++q) {
-        uint4 u;
-        u.x = pack_bf16x2(v[q * 8 + 0], v[q * 8 + 1]);
-        u.y = pack_bf16x2(v[q * 8 + 2], v[q * 8 + 3]);
-        u.z = pack_bf16x2(v[q * 8 + 4], v[q * 8 + 5]);
-        u.w = pack_bf16x2(v[q * 8 + 6], v[q * 8 + 7]);
-        p[q] = u;
     }
 }
 
@@ -141,10 +136,57 @@ struct WsSrc {
     }
 };
 
-template <int BN, int EPI, typename Src>
-F3DC_DEV void epilogue_tile(const GemmParams &p, const Src &src, int grow, int n0)
+// Output staging shared by the epilogue warps: a chunk is one 128-row box of
+// 64-byte rows, 16-byte piece c of row r at 64 r + 16 (c ^ ((r / 2) % 4))
+// (the TMA 64B swizzle), which spreads a warp's row-per-lane stores over all
+// banks.  The box is written by thread 64 with a TMA store; before a buffer
+// is reused three chunks later its store has finished reading it.
+struct OutStage {
+    uint8_t *buf;             // kOutBufs x kOutChunkBytes
+    const CUtensorMap *map;   // output tensor: bf16 [M, N] or fp32 [M, N] (RESID, reduce-add)
+    int row;                  // this thread's row of the tile
+    int ck;                   // chunks emitted so far by this CTA
+    F3DC_DEV uint8_t *slot() const { return buf + (ck % kOutBufs) * kOutChunkBytes; }
+    F3DC_DEV void put16(int c, uint4 u) const
+    {
+        *reinterpret_cast<uint4 *>(slot() + row * 64 + ((c ^ ((row >> 1) & 3)) << 4)) = u;
+    }
+    // publish the chunk just written and send it to (x, y) of the output
+    template <bool kReduce>
+    F3DC_DEV void emit(int x, int y)
+    {
+        fence_proxy_async_smem();
+        asm volatile("bar.sync 3, 128;" ::: "memory");
+        if (threadIdx.x == 64) {
+            if (kReduce)
+                tma_reduce_add_2d(map, slot(), x, y);
+            else
+                tma_store_2d(map, slot(), x, y);
+            bulk_commit();
+            // the chunk before this one has been read: its buffer, and every
+            // older one, may be rewritten after the next barrier
+            bulk_wait_read<1>();
+        }
+        ++ck;
+    }
+};
+
+F3DC_DEV void put_bf16x32(OutStage &o, const float *v)
 {
-    const bool row_ok = grow < p.M;
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+        uint4 u;
+        u.x = pack_bf16x2(v[q * 8 + 0], v[q * 8 + 1]);
+        u.y = pack_bf16x2(v[q * 8 + 2], v[q * 8 + 3]);
+        u.z = pack_bf16x2(v[q * 8 + 4], v[q * 8 + 5]);
+        u.w = pack_bf16x2(v[q * 8 + 6], v[q * 8 + 7]);
+        o.put16(q, u);
+    }
+}
+
+template <int BN, int EPI, typename Src>
+F3DC_DEV void epilogue_tile(const GemmParams &p, const Src &src, OutStage &o, int m0, int n0)
+{
     if constexpr (EPI == kEpiQKNorm) {
 #pragma unroll 1
         for (int c0 = 0; c0 < BN; c0 += 64) {
@@ -171,11 +213,10 @@ F3DC_DEV void epilogue_tile(const GemmParams &p, const Src &src, int grow, int n
                     rms_scale(v + 32, 32, g, gc + 32);
                 }
             }
-            if (row_ok) {
-                bf16 *dst = reinterpret_cast<bf16 *>(p.out) + (size_t)grow * p.ldo + col;
-                store_bf16x32(dst, v);
-                store_bf16x32(dst + 32, v + 32);
-            }
+            put_bf16x32(o, v);
+            o.template emit<false>(col, m0);
+            put_bf16x32(o, v + 32);
+            o.template emit<false>(col + 32, m0);
         }
     } else {
 #pragma unroll 1
@@ -191,22 +232,23 @@ F3DC_DEV void epilogue_tile(const GemmParams &p, const Src &src, int grow, int n
 #pragma unroll
                 for (int j = 0; j < 32; ++j) v[j] = gelu_tanh(v[j]);
             }
-            if (!row_ok) continue;
             if constexpr (EPI == kEpiResid) {
-                float *dst = reinterpret_cast<float *>(p.out) + (size_t)grow * p.ldo + col;
+                // x += gate * y as an fp32 reduce-add of gate * y, 16 columns per chunk
 #pragma unroll
-                for (int q = 0; q < 8; ++q) {
-                    float4 x = reinterpret_cast<float4 *>(dst)[q];
-                    float4 g = p.gate ? __ldg(reinterpret_cast<const float4 *>(p.gate + col) + q)
-                                      : make_float4(1.f, 1.f, 1.f, 1.f);
-                    x.x += g.x * v[4 * q + 0];
-                    x.y += g.y * v[4 * q + 1];
-                    x.z += g.z * v[4 * q + 2];
-                    x.w += g.w * v[4 * q + 3];
-                    reinterpret_cast<float4 *>(dst)[q] = x;
+                for (int h = 0; h < 2; ++h) {
+#pragma unroll
+                    for (int q = 0; q < 4; ++q) {
+                        const float4 g = p.gate ? __ldg(reinterpret_cast<const float4 *>(p.gate + col + 16 * h) + q)
+                                                : make_float4(1.f, 1.f, 1.f, 1.f);
+                        const float *w = v + 16 * h + 4 * q;
+                        o.put16(q, make_uint4(__float_as_uint(g.x * w[0]), __float_as_uint(g.y * w[1]),
+                                              __float_as_uint(g.z * w[2]), __float_as_uint(g.w * w[3])));
+                    }
+                    o.template emit<true>(col + 16 * h, m0);
                 }
             } else {
-                store_bf16x32(reinterpret_cast<bf16 *>(p.out) + (size_t)grow * p.ldo + col, v);
+                put_bf16x32(o, v);
+                o.template emit<false>(col, m0);
             }
         }
     }
@@ -228,7 +270,8 @@ struct Units {
 
 template <int BN, int EPI>
 __global__ void __launch_bounds__(kGemmThreads, 1)
-    k_gemm(const __grid_constant__ CUtensorMap tma, const __grid_constant__ CUtensorMap tmb, const GemmParams p)
+    k_gemm(const __grid_constant__ CUtensorMap tma, const __grid_constant__ CUtensorMap tmb,
+           const __grid_constant__ CUtensorMap tmo, const GemmParams p)
 {
     using Cfg = GemmCfg<BN>;
     constexpr int S = Cfg::kStages;
@@ -236,7 +279,8 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
     uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     uint8_t *sa = smem;
     uint8_t *sb = smem + S * kAStage;
-    uint64_t *bars = reinterpret_cast<uint64_t *>(sb + S * Cfg::kBStage);
+    uint8_t *so = sb + S * Cfg::kBStage;  // output staging (1024-aligned)
+    uint64_t *bars = reinterpret_cast<uint64_t *>(so + kOutBufs * kOutChunkBytes);
     uint64_t *full = bars, *empty = bars + S, *accf = bars + 2 * S, *acce = accf + 2, *drain = acce + 2;
     uint32_t *tmem_holder = reinterpret_cast<uint32_t *>(drain + 1);
     volatile int *abort_flag = reinterpret_cast<volatile int *>(tmem_holder + 1);
@@ -300,35 +344,44 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
             }
         }
     } else if (warp == 1) {
+        // Barrier reads take long even when the phase is complete: the
+        // issuer tests the next stage's `full` barrier before issuing the
+        // current stage's MMAs, so the read overlaps them, and takes the
+        // bounded wait only when the test found the stage not yet loaded.
         if (lane == 0) {
             constexpr uint32_t idesc = make_idesc_bf16(128, BN, 0, 0);
+            // stage-0 descriptors; stage s adds s * stage bytes / 16, a K
+            // step of 16 elements inside the 128B swizzle atom adds 2
+            const uint64_t a_desc0 = make_sdesc(smem_u32(sa), 16, 1024, kSwizzle128);
+            const uint64_t b_desc0 = make_sdesc(smem_u32(sb), 16, 1024, kSwizzle128);
             int s = 0, it = 0;
             uint32_t ph = 0;
             bool ok = true;
+            bool ready = mbar_test(&full[0], 0);
             for (int t = blockIdx.x; t < total && ok; t += gridDim.x, ++it) {
                 const int buf = it & 1;
                 const uint32_t aph = (it >> 1) & 1;
-                if (!mbar_wait(&acce[buf], aph ^ 1, abort_flag, p.err)) break;
-                tc_fence_after();
+                if (!mbar_test(&acce[buf], aph ^ 1) && !mbar_wait(&acce[buf], aph ^ 1, abort_flag, p.err)) break;
                 const uint32_t d = tmem + buf * BN;
                 int m0, n0, kb0, kb1;
                 U.decode(t, m0, n0, kb0, kb1, BN);
                 for (int kb = kb0; kb < kb1; ++kb) {
-                    if (!mbar_wait(&full[s], ph, abort_flag, p.err)) {
+                    if (!ready && !mbar_wait(&full[s], ph, abort_flag, p.err)) {
                         ok = false;
                         break;
                     }
                     tc_fence_after();
-                    const uint32_t a0 = smem_u32(sa + s * kAStage), b0 = smem_u32(sb + s * Cfg::kBStage);
+                    const int s_next = s + 1 == S ? 0 : s + 1;
+                    const uint32_t ph_next = s_next == 0 ? ph ^ 1 : ph;
+                    ready = mbar_test(&full[s_next], ph_next);  // read overlaps the MMAs below
+                    const uint64_t ad = a_desc0 + (uint64_t)s * (kAStage >> 4);
+                    const uint64_t bd = b_desc0 + (uint64_t)s * (Cfg::kBStage >> 4);
 #pragma unroll
                     for (int k = 0; k < kBK / 16; ++k)
-                        mma_bf16(d, make_sdesc(a0 + k * 32, 16, 1024, kSwizzle128),
-                                 make_sdesc(b0 + k * 32, 16, 1024, kSwizzle128), idesc, (kb != kb0) || (k != 0));
+                        mma_bf16(d, ad + 2 * k, bd + 2 * k, idesc, (kb != kb0) || (k != 0));
                     mma_commit(&empty[s]);
-                    if (++s == S) {
-                        s = 0;
-                        ph ^= 1;
-                    }
+                    s = s_next;
+                    ph = ph_next;
                 }
                 if (ok) mma_commit(&accf[buf]);
             }
@@ -336,17 +389,28 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
     } else {
         const int q = warp & 3;
         const int row = q * 32 + lane;
+        OutStage o{so, &tmo, row, 0};
         int it = 0;
         for (int t = blockIdx.x; t < total; t += gridDim.x, ++it) {
             const int buf = it & 1;
             const uint32_t aph = (it >> 1) & 1;
-            if (!mbar_wait(&accf[buf], aph, abort_flag, p.err)) break;
+            // the four epilogue warps meet at named barriers inside the tile,
+            // so they take the wait's outcome together (a timeout seen by one
+            // warp ends the loop for all)
+            const uint32_t got = mbar_wait(&accf[buf], aph, abort_flag, p.err) ? 1u : 0u;
+            uint32_t all;
+            asm volatile("{\n .reg .pred p, q;\n setp.ne.u32 p, %1, 0;\n bar.red.and.pred q, 3, 128, p;\n"
+                         " selp.u32 %0, 1, 0, q;\n}\n"
+                         : "=r"(all)
+                         : "r"(got)
+                         : "memory");
+            if (!all) break;
             tc_fence_after();
             int m0, n0, kb0, kb1;
             U.decode(t, m0, n0, kb0, kb1, BN);
             const TmemSrc tsrc{tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(buf * BN)};
             if (U.splits == 1) {
-                epilogue_tile<BN, EPI>(p, tsrc, m0 + row, n0);
+                epilogue_tile<BN, EPI>(p, tsrc, o, m0, n0);
                 tc_fence_before();
                 __syncwarp();
                 if (lane == 0) mbar_arrive(&acce[buf]);
@@ -380,11 +444,12 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
             if (*split_flag) {
                 __threadfence();
                 const WsSrc<BN> wsrc{p.ws, tile, U.tiles, U.splits, row};
-                epilogue_tile<BN, EPI>(p, wsrc, m0 + row, n0);
+                epilogue_tile<BN, EPI>(p, wsrc, o, m0, n0);
             }
             asm volatile("bar.sync 2, 128;" ::: "memory");
         }
-
+        // this CTA's output stores complete before it ends
+        if (threadIdx.x == 64) bulk_wait_all();
     }
     __syncthreads();
     if (*abort_flag) {
@@ -403,7 +468,8 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
 }
 
 template <int BN, int EPI>
-cudaError_t launch_one(const CUtensorMap *ta, const CUtensorMap *tb, const GemmParams &p, int grid, cudaStream_t s)
+cudaError_t launch_one(const CUtensorMap *ta, const CUtensorMap *tb, const CUtensorMap *to, const GemmParams &p,
+                       int grid, cudaStream_t s)
 {
     static bool attr_set = false;
     const size_t smem = GemmCfg<BN>::kSmem;
@@ -412,21 +478,54 @@ cudaError_t launch_one(const CUtensorMap *ta, const CUtensorMap *tb, const GemmP
         if (e != cudaSuccess) return e;
         attr_set = true;
     }
-    k_gemm<BN, EPI><<<grid, kGemmThreads, smem, s>>>(*ta, *tb, p);
+    k_gemm<BN, EPI><<<grid, kGemmThreads, smem, s>>>(*ta, *tb, *to, p);
     return cudaGetLastError();
 }
 
 template <int BN>
-cudaError_t launch_bn(const CUtensorMap *ta, const CUtensorMap *tb, const GemmParams &p, int epi, int grid,
-                      cudaStream_t s)
+cudaError_t launch_bn(const CUtensorMap *ta, const CUtensorMap *tb, const CUtensorMap *to, const GemmParams &p,
+                      int epi, int grid, cudaStream_t s)
 {
     switch (epi) {
-    case kEpiBias: return launch_one<BN, kEpiBias>(ta, tb, p, grid, s);
-    case kEpiGelu: return launch_one<BN, kEpiGelu>(ta, tb, p, grid, s);
-    case kEpiResid: return launch_one<BN, kEpiResid>(ta, tb, p, grid, s);
-    case kEpiQKNorm: return launch_one<BN, kEpiQKNorm>(ta, tb, p, grid, s);
+    case kEpiBias: return launch_one<BN, kEpiBias>(ta, tb, to, p, grid, s);
+    case kEpiGelu: return launch_one<BN, kEpiGelu>(ta, tb, to, p, grid, s);
+    case kEpiResid: return launch_one<BN, kEpiResid>(ta, tb, to, p, grid, s);
+    case kEpiQKNorm: return launch_one<BN, kEpiQKNorm>(ta, tb, to, p, grid, s);
     default: return cudaErrorInvalidValue;
     }
+}
+
+PFN_cuTensorMapEncodeTiled_v12000 tmap_encoder()
+{
+    static PFN_cuTensorMapEncodeTiled_v12000 encode = nullptr;
+    if (!encode) {
+        cudaDriverEntryPointQueryResult q;
+        void *fn = nullptr;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000, cudaEnableDefault, &q) !=
+                cudaSuccess ||
+            q != cudaDriverEntryPointSuccess || !fn)
+            return nullptr;
+        encode = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(fn);
+    }
+    return encode;
+}
+
+// The epilogue's output tensor: rows [0, M), columns [0, N), row stride ldo
+// elements; boxes of 128 rows x 64 bytes (32 bf16 or 16 fp32 columns), 64B
+// swizzle, matching OutStage.
+bool make_tmap_out(CUtensorMap *map, void *base, uint64_t rows, uint64_t cols, uint64_t ld, bool f32)
+{
+    PFN_cuTensorMapEncodeTiled_v12000 encode = tmap_encoder();
+    const uint64_t esz = f32 ? 4 : 2;
+    if (!encode || ((uintptr_t)base & 15) != 0 || (ld * esz) % 16 != 0) return false;
+    cuuint64_t dims[2] = {cols, rows};
+    cuuint64_t strides[1] = {ld * esz};
+    cuuint32_t box[2] = {(cuuint32_t)(64 / esz), 128};
+    cuuint32_t estr[2] = {1, 1};
+    CUresult r = encode(map, f32 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT32 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, base, dims,
+                        strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_64B,
+                        CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    return r == CUDA_SUCCESS;
 }
 
 }  // namespace
@@ -445,10 +544,13 @@ cudaError_t launch_gemm(const CUtensorMap *ta, const CUtensorMap *tb, const Gemm
                         int grid, cudaStream_t s)
 {
     if (p.K % kBK != 0 || p.N % bn != 0 || grid < 1) return cudaErrorInvalidValue;
+    CUtensorMap to;
+    if (!make_tmap_out(&to, p.out, (uint64_t)p.M, (uint64_t)p.N, (uint64_t)p.ldo, epi == kEpiResid))
+        return cudaErrorInvalidValue;
     switch (bn) {
-    case 64: return launch_bn<64>(ta, tb, p, epi, grid, s);
-    case 128: return launch_bn<128>(ta, tb, p, epi, grid, s);
-    case 256: return launch_bn<256>(ta, tb, p, epi, grid, s);
+    case 64: return launch_bn<64>(ta, tb, &to, p, epi, grid, s);
+    case 128: return launch_bn<128>(ta, tb, &to, p, epi, grid, s);
+    case 256: return launch_bn<256>(ta, tb, &to, p, epi, grid, s);
     default: return cudaErrorInvalidValue;
     }
 }
@@ -456,17 +558,8 @@ cudaError_t launch_gemm(const CUtensorMap *ta, const CUtensorMap *tb, const Gemm
 bool make_tmap_bf16(CUtensorMap *map, const void *base, uint64_t rows, uint64_t cols, uint64_t ld,
                     uint32_t box_rows, uint32_t box_cols)
 {
-    static PFN_cuTensorMapEncodeTiled_v12000 encode = nullptr;
-    if (!encode) {
-        cudaDriverEntryPointQueryResult q;
-        void *fn = nullptr;
-        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000, cudaEnableDefault, &q) !=
-                cudaSuccess ||
-            q != cudaDriverEntryPointSuccess || !fn)
-            return false;
-        encode = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(fn);
-    }
-    if (((uintptr_t)base & 15) != 0 || (ld * 2) % 16 != 0) return false;
+    PFN_cuTensorMapEncodeTiled_v12000 encode = tmap_encoder();
+    if (!encode || ((uintptr_t)base & 15) != 0 || (ld * 2) % 16 != 0) return false;
     CUtensorMapSwizzle swz;
     switch (box_cols * 2) {
     case 128: swz = CU_TENSOR_MAP_SWIZZLE_128B; break;
