@@ -162,6 +162,17 @@ F3DC_DEV void bulk_wait_read()
 // every committed bulk group complete (writes performed)
 F3DC_DEV void bulk_wait_all() { asm volatile("cp.async.bulk.wait_group 0;" ::: "memory"); }
 
+// Programmatic dependent launch.  A kernel launched with programmatic stream
+// serialization may start (and run its prologue) while the previous kernel
+// in the stream is still running.  griddep_wait() blocks until that kernel
+// has completed and its memory operations are visible; without the launch
+// attribute it returns at once.  Every kernel of this library calls it
+// before its first global-memory access (read or write), which also keeps
+// completion ordered along a chain of such kernels.  griddep_launch() lets
+// the next kernel be scheduled early; its CTAs still wait in griddep_wait().
+F3DC_DEV void griddep_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+F3DC_DEV void griddep_launch() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
+
 // Orders this thread's generic-proxy shared-memory writes before later
 // async-proxy (tensor core / TMA) reads of the same memory.
 F3DC_DEV void fence_proxy_async_smem() { asm volatile("fence.proxy.async.shared::cta;" ::: "memory"); }

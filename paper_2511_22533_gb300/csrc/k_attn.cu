@@ -127,8 +127,7 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
     volatile int *abort_flag = reinterpret_cast<volatile int *>(tmem_holder + 1);
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int n_tiles = p.n_tiles_dev ? *p.n_tiles_dev : p.n_tiles;
-    const int total = n_tiles * p.heads;
+    griddep_launch();
 
     if (threadIdx.x == 0) {
         mbar_init(q_full, 1);
@@ -154,6 +153,10 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
     __syncthreads();
     tc_fence_after();
     const uint32_t tmem = *tmem_holder;
+    // the previous kernel's outputs (Q / K / V, the row plan) are complete
+    griddep_wait();
+    const int n_tiles = p.n_tiles_dev ? *p.n_tiles_dev : p.n_tiles;
+    const int total = n_tiles * p.heads;
 
     if (warp == 0) {
         // ------------------------------------------------ TMA producer
@@ -496,7 +499,7 @@ cudaError_t launch_dh(const CUtensorMap *tq, const CUtensorMap *tk, const CUtens
         if (e != cudaSuccess) return e;
         attr_set = true;
     }
-    k_attn<DH><<<grid, kAttnThreads, smem, s>>>(*tq, *tk, *tv, p);
+    launch_k(k_attn<DH>, dim3(grid), dim3(kAttnThreads), smem, s, *tq, *tk, *tv, p);
     return cudaGetLastError();
 }
 

@@ -287,14 +287,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
     volatile int *split_flag = reinterpret_cast<volatile int *>(tmem_holder + 2);
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    Units U;
-    U.m_tiles = p.m_tiles_dev ? *p.m_tiles_dev : p.m_tiles;
-    U.tiles = U.m_tiles * (p.N / BN);
-    U.kb_n = p.K / kBK;
-    U.splits = gemm_split_count(U.tiles, (int)gridDim.x, U.kb_n, p.ws_units, p.ws != nullptr);
-    U.kb_per = (U.kb_n + U.splits - 1) / U.splits;
-    U.total = U.tiles * U.splits;
-    const int total = U.total;
+    griddep_launch();
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < S; ++s) {
@@ -317,6 +310,16 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
     __syncthreads();
     tc_fence_after();
     const uint32_t tmem = *tmem_holder;
+    // the previous kernel's outputs (A, the row plan, x) are complete
+    griddep_wait();
+    Units U;
+    U.m_tiles = p.m_tiles_dev ? *p.m_tiles_dev : p.m_tiles;
+    U.tiles = U.m_tiles * (p.N / BN);
+    U.kb_n = p.K / kBK;
+    U.splits = gemm_split_count(U.tiles, (int)gridDim.x, U.kb_n, p.ws_units, p.ws != nullptr);
+    U.kb_per = (U.kb_n + U.splits - 1) / U.splits;
+    U.total = U.tiles * U.splits;
+    const int total = U.total;
 
     if (warp == 0) {
         if (lane == 0) {
@@ -478,7 +481,7 @@ cudaError_t launch_one(const CUtensorMap *ta, const CUtensorMap *tb, const CUten
         if (e != cudaSuccess) return e;
         attr_set = true;
     }
-    k_gemm<BN, EPI><<<grid, kGemmThreads, smem, s>>>(*ta, *tb, *to, p);
+    launch_k(k_gemm<BN, EPI>, dim3(grid), dim3(kGemmThreads), smem, s, *ta, *tb, *to, p);
     return cudaGetLastError();
 }
 

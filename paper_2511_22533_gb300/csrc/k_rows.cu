@@ -42,6 +42,8 @@ __global__ void __launch_bounds__(kRowThreads) k_gather_embed(const float *S, in
                                                               const bf16 *in_b, const float *pos, float *x,
                                                               uint32_t *err)
 {
+    griddep_launch();
+    griddep_wait();
     const int m_rows = plan->m_rows;
     const int lane = threadIdx.x & 31, wpb = blockDim.x >> 5;
     for (int r = blockIdx.x * wpb + (threadIdx.x >> 5); r < m_rows; r += gridDim.x * wpb) {
@@ -107,6 +109,8 @@ __global__ void __launch_bounds__(kRowThreads) k_layernorm(const float *x, int W
                                                            const float *shift, const float *scale, const bf16 *g,
                                                            const bf16 *bb, bf16 *out)
 {
+    griddep_launch();
+    griddep_wait();
     const int m_rows = plan->m_rows;
     const int lane = threadIdx.x & 31, wpb = blockDim.x >> 5;
     for (int r = blockIdx.x * wpb + (threadIdx.x >> 5); r < m_rows; r += gridDim.x * wpb) {
@@ -149,6 +153,8 @@ __global__ void __launch_bounds__(kRowThreads) k_final_layer(const float *x, int
                                                              const float *shift, const float *scale,
                                                              const bf16 *out_w, const bf16 *out_b, float *v_active)
 {
+    griddep_launch();
+    griddep_wait();
     const int m_rows = plan->m_rows;
     const int lane = threadIdx.x & 31, wpb = blockDim.x >> 5;
     for (int r = blockIdx.x * wpb + (threadIdx.x >> 5); r < m_rows; r += gridDim.x * wpb) {
@@ -193,6 +199,8 @@ constexpr int kMaxG = 512;
 
 __global__ void __launch_bounds__(kMergeThreads) k_merge_euler(const MergeArgs a)
 {
+    griddep_launch();
+    griddep_wait();
     __shared__ float dec[8 * kMaxG];
     const bool count = a.dyn != nullptr;
     if (count) {
@@ -263,6 +271,8 @@ __global__ void __launch_bounds__(kMergeThreads) k_merge_euler(const MergeArgs a
 
 __global__ void k_scatter_rows(const float *v_active, const Plan *plan, int N, float *v_out)
 {
+    griddep_launch();
+    griddep_wait();
     const int b = blockIdx.y;
     const int na = plan->n_active[b], off = plan->row_off[b];
     for (int j = blockIdx.x * blockDim.x + threadIdx.x; j < na; j += gridDim.x * blockDim.x) {
@@ -276,6 +286,8 @@ __global__ void k_scatter_rows(const float *v_active, const Plan *plan, int N, f
 // ------------------------------------------------------------------ K9
 __global__ void k_time_freq(float t, float *freq)
 {
+    griddep_launch();
+    griddep_wait();
     const int f = threadIdx.x;  // 128 threads
     const float w = expf(-9.210340371976184f * (float)f / 128.0f);  // ln(10000)
     const float arg = 1000.0f * t * w;
@@ -291,6 +303,8 @@ constexpr int kGemvMaxK = 4096;
 __global__ void __launch_bounds__(kGemvThreads) k_gemv(const float *x, int K, const bf16 *w, const bf16 *bias,
                                                        float *y, int rows, int silu_in, int silu_out)
 {
+    griddep_launch();
+    griddep_wait();
     __shared__ float xs[kGemvMaxK];
     for (int k = threadIdx.x; k < K; k += blockDim.x) xs[k] = silu_in ? silu(x[k]) : x[k];
     __syncthreads();
@@ -341,7 +355,7 @@ cudaError_t launch_gather_embed(const float *S, int N, int W, const int32_t *act
                                 const float *pos, float *x, int max_rows, int num_sms, uint32_t *err,
                                 cudaStream_t s)
 {
-    k_gather_embed<<<row_grid(num_sms, max_rows), kRowThreads, 0, s>>>(S, N, W, active_idx, plan, tile_sample,
+    launch_k(k_gather_embed, dim3(row_grid(num_sms, max_rows)), dim3(kRowThreads), 0, s, S, N, W, active_idx, plan, tile_sample,
                                                                        in_w, in_b, pos, x, err);
     return cudaGetLastError();
 }
@@ -352,11 +366,11 @@ cudaError_t launch_layernorm(const float *x, int W, const Plan *plan, int mode, 
 {
     const int grid = row_grid(num_sms, max_rows);
     switch (W / 128) {
-    case 1: k_layernorm<1><<<grid, kRowThreads, 0, s>>>(x, W, plan, mode, shift, scale, g, b, out); break;
-    case 2: k_layernorm<2><<<grid, kRowThreads, 0, s>>>(x, W, plan, mode, shift, scale, g, b, out); break;
-    case 4: k_layernorm<4><<<grid, kRowThreads, 0, s>>>(x, W, plan, mode, shift, scale, g, b, out); break;
-    case 8: k_layernorm<8><<<grid, kRowThreads, 0, s>>>(x, W, plan, mode, shift, scale, g, b, out); break;
-    case 16: k_layernorm<16><<<grid, kRowThreads, 0, s>>>(x, W, plan, mode, shift, scale, g, b, out); break;
+    case 1: launch_k(k_layernorm<1>, dim3(grid), dim3(kRowThreads), 0, s, x, W, plan, mode, shift, scale, g, b, out); break;
+    case 2: launch_k(k_layernorm<2>, dim3(grid), dim3(kRowThreads), 0, s, x, W, plan, mode, shift, scale, g, b, out); break;
+    case 4: launch_k(k_layernorm<4>, dim3(grid), dim3(kRowThreads), 0, s, x, W, plan, mode, shift, scale, g, b, out); break;
+    case 8: launch_k(k_layernorm<8>, dim3(grid), dim3(kRowThreads), 0, s, x, W, plan, mode, shift, scale, g, b, out); break;
+    case 16: launch_k(k_layernorm<16>, dim3(grid), dim3(kRowThreads), 0, s, x, W, plan, mode, shift, scale, g, b, out); break;
     default: return cudaErrorInvalidValue;
     }
     return cudaGetLastError();
@@ -368,11 +382,11 @@ cudaError_t launch_final_layer(const float *x, int W, const Plan *plan, const fl
 {
     const int grid = row_grid(num_sms, max_rows);
     switch (W / 128) {
-    case 1: k_final_layer<1><<<grid, kRowThreads, 0, s>>>(x, W, plan, shift, scale, out_w, out_b, v_active); break;
-    case 2: k_final_layer<2><<<grid, kRowThreads, 0, s>>>(x, W, plan, shift, scale, out_w, out_b, v_active); break;
-    case 4: k_final_layer<4><<<grid, kRowThreads, 0, s>>>(x, W, plan, shift, scale, out_w, out_b, v_active); break;
-    case 8: k_final_layer<8><<<grid, kRowThreads, 0, s>>>(x, W, plan, shift, scale, out_w, out_b, v_active); break;
-    case 16: k_final_layer<16><<<grid, kRowThreads, 0, s>>>(x, W, plan, shift, scale, out_w, out_b, v_active); break;
+    case 1: launch_k(k_final_layer<1>, dim3(grid), dim3(kRowThreads), 0, s, x, W, plan, shift, scale, out_w, out_b, v_active); break;
+    case 2: launch_k(k_final_layer<2>, dim3(grid), dim3(kRowThreads), 0, s, x, W, plan, shift, scale, out_w, out_b, v_active); break;
+    case 4: launch_k(k_final_layer<4>, dim3(grid), dim3(kRowThreads), 0, s, x, W, plan, shift, scale, out_w, out_b, v_active); break;
+    case 8: launch_k(k_final_layer<8>, dim3(grid), dim3(kRowThreads), 0, s, x, W, plan, shift, scale, out_w, out_b, v_active); break;
+    case 16: launch_k(k_final_layer<16>, dim3(grid), dim3(kRowThreads), 0, s, x, W, plan, shift, scale, out_w, out_b, v_active); break;
     default: return cudaErrorInvalidValue;
     }
     return cudaGetLastError();
@@ -383,7 +397,7 @@ cudaError_t launch_merge_euler(const MergeArgs &a, cudaStream_t s)
     if (a.dyn && (a.G > kMaxG || a.N % 32 != 0)) return cudaErrorInvalidValue;
     const size_t total = (size_t)a.B * a.N;
     const int grid = (int)((total + kMergeThreads - 1) / kMergeThreads);
-    k_merge_euler<<<grid, kMergeThreads, 0, s>>>(a);
+    launch_k(k_merge_euler, dim3(grid), dim3(kMergeThreads), 0, s, a);
     return cudaGetLastError();
 }
 
@@ -391,13 +405,13 @@ cudaError_t launch_scatter_rows(const float *v_active, const Plan *plan, int B, 
                                 cudaStream_t s)
 {
     dim3 grid((N + 255) / 256, B);
-    k_scatter_rows<<<grid, 256, 0, s>>>(v_active, plan, N, v_out);
+    launch_k(k_scatter_rows, dim3(grid), dim3(256), 0, s, v_active, plan, N, v_out);
     return cudaGetLastError();
 }
 
 cudaError_t launch_time_freq(float t, float *freq, cudaStream_t s)
 {
-    k_time_freq<<<1, 128, 0, s>>>(t, freq);
+    launch_k(k_time_freq, dim3(1), dim3(128), 0, s, t, freq);
     return cudaGetLastError();
 }
 
@@ -408,7 +422,7 @@ cudaError_t launch_gemv(const float *x, int K, const bf16 *w, const bf16 *b, flo
     const int wpb = kGemvThreads / 32;
     int grid = (rows + 2 * wpb - 1) / (2 * wpb);
     if (grid > num_sms * 4) grid = num_sms * 4;
-    k_gemv<<<grid, kGemvThreads, 0, s>>>(x, K, w, b, y, rows, silu_in, silu_out);
+    launch_k(k_gemv, dim3(grid), dim3(kGemvThreads), 0, s, x, K, w, b, y, rows, silu_in, silu_out);
     return cudaGetLastError();
 }
 

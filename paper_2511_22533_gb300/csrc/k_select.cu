@@ -94,6 +94,8 @@ F3DC_DEV void write_plan(const SelectArgs &a, int b, int na, int &off)
 
 __global__ void __launch_bounds__(kSelThreads, 1) k_ssc_select(const SelectArgs a)
 {
+    griddep_launch();
+    griddep_wait();
     extern __shared__ uint32_t keys[];
     __shared__ uint32_t hist[256];
     __shared__ float red[4][kSelWarps];
@@ -272,6 +274,8 @@ __global__ void __launch_bounds__(kSelThreads, 1) k_ssc_select(const SelectArgs 
 __global__ void k_plan_from_counts(const int32_t *n_active, int B, int N, Plan *plan, int32_t *tile_sample,
                                    uint32_t *err)
 {
+    griddep_launch();
+    griddep_wait();
     __shared__ int offs[kMaxBatch + 1];
     if (threadIdx.x == 0) {
         int o = 0;
@@ -307,7 +311,7 @@ cudaError_t launch_ssc_select(const SelectArgs &a, cudaStream_t s)
     const size_t smem = (size_t)a.N * sizeof(uint32_t);
     cudaError_t e = cudaFuncSetAttribute(k_ssc_select, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
-    k_ssc_select<<<a.B, kSelThreads, smem, s>>>(a);
+    launch_k(k_ssc_select, dim3(a.B), dim3(kSelThreads), smem, s, a);
     return cudaGetLastError();
 }
 
@@ -318,7 +322,7 @@ cudaError_t launch_plan_from_counts(const int32_t *n_active, const int32_t *acti
     (void)active_idx;
     (void)row_of_token;
     if (B < 1 || B > kMaxBatch) return cudaErrorInvalidValue;
-    k_plan_from_counts<<<1, 256, 0, s>>>(n_active, B, N, plan, tile_sample, err);
+    launch_k(k_plan_from_counts, dim3(1), dim3(256), 0, s, n_active, B, N, plan, tile_sample, err);
     return cudaGetLastError();
 }
 

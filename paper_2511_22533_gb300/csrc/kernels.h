@@ -125,6 +125,25 @@ cudaError_t launch_gemm(const CUtensorMap *ta, const CUtensorMap *tb, const Gemm
                         int grid, cudaStream_t s);
 size_t gemm_smem_bytes(int bn);
 // bytes of split-K workspace for `units` partial tiles of width bn
+// Launches a kernel of this library with programmatic stream serialization
+// (programmatic dependent launch): the kernel may start while the previous
+// kernel in the stream finishes and waits for it in griddep_wait().
+template <typename... KArgs, typename... Args>
+cudaError_t launch_k(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t s, Args... args)
+{
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = grid;
+    cfg.blockDim = block;
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = s;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, kernel, args...);
+}
+
 inline size_t gemm_ws_bytes(int bn, int units) { return (size_t)units * 128 * bn * sizeof(float); }
 constexpr int kGemmMaxCounterTiles = 1024;
 
