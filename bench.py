@@ -232,6 +232,69 @@ def quota_log_host():
     return np.array(q, np.int32)[:, None]
 
 
+def hbm_kernels_b64(f3dc, torch, blob_d, pk):
+    """The HBM-bound kernels of the step at batch 64 (16^3 x 8 latents, half
+    of each sample's tokens cached), L2 flushed before each measurement: the
+    SSC selection alone through f3dc_ssc_select (median of 20 calls, CUDA
+    events around each call), and the gather/embed and merge/Euler kernels
+    from one profiled f3dc_step.  Bytes are the algorithmic ones (selection:
+    33 B per token + 4 B per active index; gather: 36 + 4W B per active token;
+    merge: 96 B per token + 32 B per active token)."""
+    shape = synth.SHAPES[WORKLOAD]
+    B, N = 64, shape.tokens
+    cfg = f3dc.config_for(shape, B)
+    h = f3dc.Handle(cfg, blob_d)
+    flush = torch.empty(64 * 1024 * 1024, dtype=torch.float32, device="cuda")  # 256 MB > L2
+    hist = synth.velocity_history(shape.grid, shape.channels, B, seed=11)
+    ring = torch.from_numpy(hist.view(np.int16)).cuda()
+    quota = torch.full((B,), N // 2, dtype=torch.int32, device="cuda")
+    idx = torch.empty((B, N), dtype=torch.int32, device="cuda")
+    nact = torch.empty((B,), dtype=torch.int32, device="cuda")
+    mask = torch.empty((B, N), dtype=torch.uint8, device="cuda")
+    times = []
+    for i in range(23):
+        flush.zero_()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record()
+        h.ssc_select(ring[2], ring[1], B, quota, idx, nact, mask)
+        e1.record()
+        torch.cuda.synchronize()
+        if i >= 3:
+            times.append(e0.elapsed_time(e1))
+    ms = float(np.median(times))
+    sel_bytes = B * N * 33 + B * (N - N // 2) * 4
+    out = {"workload": f"batch {B} x 4096 tokens (16^3 x 8), {N // 2} cached per sample, L2 flushed",
+           "ssc_select": {"us": ms * 1000.0, "bytes": sel_bytes, "gbs": sel_bytes / (ms / 1000.0) / 1e9}}
+    out["ssc_select"]["frac_hbm"] = out["ssc_select"]["gbs"] / pk["hbm_gbs"]
+    # one profiled step: gather/embed and merge/Euler at batch 64
+    cond = torch.from_numpy(np.ascontiguousarray(np.broadcast_to(
+        synth.cond_tokens(shape, 1, 3), (B, shape.cond_tokens, shape.cond_dim))).view(np.int16)).cuda()
+    h.set_cond(cond, B)
+    S = torch.from_numpy(synth.latents(shape, B, 5)).cuda()
+    k = 8  # a cached step: history slots k-1, k-2 hold the drift history
+    ring_k = torch.empty_like(ring)
+    ring_k[(k - 1) % 3] = ring[2]
+    ring_k[(k - 2) % 3] = ring[1]
+    ring_k[k % 3] = ring[0]
+    torch.cuda.synchronize()
+    flush.zero_()
+    h.profile(True)
+    h.step(k, B, S, ring_k, quota)
+    torch.cuda.synchronize()
+    stats = {st["name"]: st for st in h.profile_read()}
+    h.profile(False)
+    for name in ("gather_embed", "merge_euler"):
+        st = stats.get(name)
+        if st and st["total_ms"] > 0:
+            out[name] = {"us": st["total_ms"] * 1000.0 / max(st["launches"], 1), "bytes": st["bytes"],
+                         "gbs": st["bytes"] / (st["total_ms"] / 1000.0) / 1e9}
+            out[name]["frac_hbm"] = out[name]["gbs"] / pk["hbm_gbs"]
+    assert h.device_status() == 0
+    h.close()
+    del flush
+    return out
+
+
 def run_reference(args):
     rank = int(os.environ.get("RANK", "0"))
     if rank != 0:
@@ -307,7 +370,6 @@ def run_gpu(args):
     blob_d = torch.from_numpy(blob.view(np.int16)).cuda()
     cfg = f3dc.config_for(shape, 1)
     h = f3dc.Handle(cfg, blob_d)
-    del blob_d
     noise = synth.latents(shape, 1, rank_seed(rank))
     cond_np = synth.cond_tokens(shape, 1, rank_seed(rank))
     noise_d = torch.from_numpy(noise).cuda()
@@ -385,6 +447,10 @@ def run_gpu(args):
     e2e_value = whole_job_throughput(shape.steps, args.steps, world, ms_e2e)
     assert h.device_status() == 0
 
+    # ---- the HBM-bound kernels at batch 64 (secondary; not part of `value`)
+    hbm64 = hbm_kernels_b64(f3dc, torch, blob_d, pk) if rank == 0 else None
+    del blob_d
+
     # ---- CPU baseline (oracle on the host cores), rank 0 at N = 1 only
     cpu = None
     if world == 1 and rank == 0:
@@ -439,7 +505,7 @@ def run_gpu(args):
                      "tensor_tflops_per_gpu": mm_unc / (ms_unc / 1000.0) / 1e12},
         "active_tokens_per_step": [shape.tokens - int(c) for c in qlog[:, 0]],
         "sigma_measured_by_stand_in_decoder": float(sigma_meas[0]),
-        "roofline": roof, "kernels": kernels,
+        "roofline": roof, "kernels": kernels, "hbm_kernels_b64": hbm64,
         "cpu_baseline": cpu,
         "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": int(noise.nbytes + cond_np.nbytes),
                 "d2h_bytes_per_step": int(noise.nbytes)},
