@@ -104,47 +104,71 @@ F3DC_DEV void row_stats(const float4 (&v)[NV], int W, float &mean, float &rstd)
     rstd = rsqrtf(var + 1e-6f);
 }
 
+// One warp per row, lane l owning float4 columns q * 32 + l.  The per-column
+// modulation (adaLN scale / shift, or LN gain / bias) is staged in shared
+// memory once per CTA, and each warp loads its next row while it normalises
+// the current one, so the kernel streams rows at a persistent grid of two
+// CTAs per SM instead of paying two dependent memory round trips per row.
 template <int NV>
-__global__ void __launch_bounds__(kRowThreads) k_layernorm(const float *x, int W, const Plan *plan, int mode,
-                                                           const float *shift, const float *scale, const bf16 *g,
-                                                           const bf16 *bb, bf16 *out)
+__global__ void __launch_bounds__(kRowThreads, 2) k_layernorm(const float *x, int W, const Plan *plan, int mode,
+                                                              const float *shift, const float *scale,
+                                                              const bf16 *g, const bf16 *bb, bf16 *out)
 {
     griddep_launch();
     griddep_wait();
+    __shared__ float4 s_mul[NV * 32], s_add[NV * 32];  // y = xhat * mul + add per column
     const int m_rows = plan->m_rows;
     const int lane = threadIdx.x & 31, wpb = blockDim.x >> 5;
-    for (int r = blockIdx.x * wpb + (threadIdx.x >> 5); r < m_rows; r += gridDim.x * wpb) {
-        const float *xr = x + (size_t)r * W;
-        float4 v[NV];
+    const int stride = gridDim.x * wpb;
+    int r = blockIdx.x * wpb + (threadIdx.x >> 5);
+    if (blockIdx.x * wpb >= m_rows) return;  // the whole CTA is idle
+    for (int c4 = threadIdx.x; c4 < NV * 32; c4 += blockDim.x) {
+        const int n0 = 4 * c4;
+        if (mode == 0) {
+            const float4 sc = ld_f4(scale + n0);
+            s_mul[c4] = make_float4(1.f + sc.x, 1.f + sc.y, 1.f + sc.z, 1.f + sc.w);
+            s_add[c4] = ld_f4(shift + n0);
+        } else {
+            const uint2 gw = __ldg(reinterpret_cast<const uint2 *>(reinterpret_cast<const uint16_t *>(g) + n0));
+            const uint2 bw = __ldg(reinterpret_cast<const uint2 *>(reinterpret_cast<const uint16_t *>(bb) + n0));
+            s_mul[c4] = make_float4(bf16_bits_to_f32(gw.x & 0xFFFFu), bf16_bits_to_f32(gw.x >> 16),
+                                    bf16_bits_to_f32(gw.y & 0xFFFFu), bf16_bits_to_f32(gw.y >> 16));
+            s_add[c4] = make_float4(bf16_bits_to_f32(bw.x & 0xFFFFu), bf16_bits_to_f32(bw.x >> 16),
+                                    bf16_bits_to_f32(bw.y & 0xFFFFu), bf16_bits_to_f32(bw.y >> 16));
+        }
+    }
+    __syncthreads();
+    if (r >= m_rows) return;
+    float4 v[NV];
 #pragma unroll
-        for (int q = 0; q < NV; ++q) v[q] = ld_f4(xr + 4 * (q * 32 + lane));
+    for (int q = 0; q < NV; ++q) v[q] = ld_f4(x + (size_t)r * W + 4 * (q * 32 + lane));
+    for (;;) {
+        const int rn = r + stride;
+        float4 vn[NV];
+        if (rn < m_rows) {
+#pragma unroll
+            for (int q = 0; q < NV; ++q) vn[q] = ld_f4(x + (size_t)rn * W + 4 * (q * 32 + lane));
+        }
         float mean, rstd;
         row_stats<NV>(v, W, mean, rstd);
         uint16_t *orow = reinterpret_cast<uint16_t *>(out) + (size_t)r * W;
 #pragma unroll
         for (int q = 0; q < NV; ++q) {
             const int n0 = 4 * (q * 32 + lane);
-            float y[4] = {(v[q].x - mean) * rstd, (v[q].y - mean) * rstd, (v[q].z - mean) * rstd,
-                          (v[q].w - mean) * rstd};
-            if (mode == 0) {
-                const float4 sc = ld_f4(scale + n0), sh = ld_f4(shift + n0);
-                y[0] = y[0] * (1.f + sc.x) + sh.x;
-                y[1] = y[1] * (1.f + sc.y) + sh.y;
-                y[2] = y[2] * (1.f + sc.z) + sh.z;
-                y[3] = y[3] * (1.f + sc.w) + sh.w;
-            } else {
-                const uint2 gw = __ldg(reinterpret_cast<const uint2 *>(reinterpret_cast<const uint16_t *>(g) + n0));
-                const uint2 bw = __ldg(reinterpret_cast<const uint2 *>(reinterpret_cast<const uint16_t *>(bb) + n0));
-                y[0] = y[0] * bf16_bits_to_f32(gw.x & 0xFFFFu) + bf16_bits_to_f32(bw.x & 0xFFFFu);
-                y[1] = y[1] * bf16_bits_to_f32(gw.x >> 16) + bf16_bits_to_f32(bw.x >> 16);
-                y[2] = y[2] * bf16_bits_to_f32(gw.y & 0xFFFFu) + bf16_bits_to_f32(bw.y & 0xFFFFu);
-                y[3] = y[3] * bf16_bits_to_f32(gw.y >> 16) + bf16_bits_to_f32(bw.y >> 16);
-            }
+            const float4 mu = s_mul[q * 32 + lane], ad = s_add[q * 32 + lane];
+            const float y0 = (v[q].x - mean) * rstd * mu.x + ad.x;
+            const float y1 = (v[q].y - mean) * rstd * mu.y + ad.y;
+            const float y2 = (v[q].z - mean) * rstd * mu.z + ad.z;
+            const float y3 = (v[q].w - mean) * rstd * mu.w + ad.w;
             uint2 pk;
-            pk.x = pack_bf16x2(y[0], y[1]);
-            pk.y = pack_bf16x2(y[2], y[3]);
+            pk.x = pack_bf16x2(y0, y1);
+            pk.y = pack_bf16x2(y2, y3);
             *reinterpret_cast<uint2 *>(orow + n0) = pk;
         }
+        if (rn >= m_rows) break;
+        r = rn;
+#pragma unroll
+        for (int q = 0; q < NV; ++q) v[q] = vn[q];
     }
 }
 
@@ -364,7 +388,8 @@ cudaError_t launch_layernorm(const float *x, int W, const Plan *plan, int mode, 
                              const float *scale, const bf16 *g, const bf16 *b, bf16 *out, int max_rows,
                              int num_sms, cudaStream_t s)
 {
-    const int grid = row_grid(num_sms, max_rows);
+    const int need = (max_rows + kRowThreads / 32 - 1) / (kRowThreads / 32);
+    const int grid = need < 2 * num_sms ? (need > 0 ? need : 1) : 2 * num_sms;
     switch (W / 128) {
     case 1: launch_k(k_layernorm<1>, dim3(grid), dim3(kRowThreads), 0, s, x, W, plan, mode, shift, scale, g, b, out); break;
     case 2: launch_k(k_layernorm<2>, dim3(grid), dim3(kRowThreads), 0, s, x, W, plan, mode, shift, scale, g, b, out); break;
