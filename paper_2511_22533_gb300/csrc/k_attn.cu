@@ -54,7 +54,7 @@ struct AttnCfg {
     static constexpr uint32_t kAtom = 8 * kRowBytes;    // 8-row swizzle atom
     static constexpr uint32_t kSwz = DH == 64 ? kSwizzle128 : kSwizzle64;
     static constexpr int kCombineBytes = 128 * DH * 4;  // parity-1 O, one row per softmax row
-    static constexpr size_t kSmem = 1024 + kTileBytes * (1 + 2 * kKVStages) + kCombineBytes + 512 + 128 * 8;
+    static constexpr size_t kSmem = 1024 + kTileBytes * (2 + 2 * kKVStages) + kCombineBytes + 512 + 128 * 8;
     // TMEM columns: S_0 S_1 (fp32, 128 each) | O_0 O_1 (fp32, DH each) |
     // P_0 P_1 (bf16 pairs, 64 each)
     static constexpr uint32_t kColO = 256, kColP = 256 + 2 * DH;
@@ -105,15 +105,17 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
     using Cfg = AttnCfg<DH>;
     extern __shared__ uint8_t smem_raw[];
     uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+    // Q is double-buffered per item (item i in buffer i % 2), so the next
+    // item's Q arrives while the current item's last key tiles run
     uint8_t *sQ = smem;
-    uint8_t *sK = sQ + Cfg::kTileBytes;
+    uint8_t *sK = sQ + 2 * Cfg::kTileBytes;
     uint8_t *sV = sK + kKVStages * Cfg::kTileBytes;
     // the end-of-item combine hands parity 1's O and (m, l) to parity 0
     float *sComb = reinterpret_cast<float *>(sV + kKVStages * Cfg::kTileBytes);
     uint64_t *bars = reinterpret_cast<uint64_t *>(reinterpret_cast<uint8_t *>(sComb) + Cfg::kCombineBytes);
     float2 *sML = reinterpret_cast<float2 *>(reinterpret_cast<uint8_t *>(bars) + 512);
-    uint64_t *q_full = bars, *q_empty = bars + 1;
-    uint64_t *kv_full = bars + 2, *kv_empty = kv_full + kKVStages;
+    uint64_t *q_full = bars, *q_empty = bars + 2;
+    uint64_t *kv_full = bars + 4, *kv_empty = kv_full + kKVStages;
     // Key tile g (counted over the CTA's whole run) always sits in K/V stage
     // g % kKVStages, so kv_empty[g % kKVStages] completes exactly when P V of
     // tile g does: the producer reuses the stage on it, and the softmax takes
@@ -130,8 +132,10 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
     griddep_launch();
 
     if (threadIdx.x == 0) {
-        mbar_init(q_full, 1);
-        mbar_init(q_empty, 1);
+        for (int b = 0; b < 2; ++b) {
+            mbar_init(&q_full[b], 1);
+            mbar_init(&q_empty[b], 1);
+        }
         for (int s = 0; s < kKVStages; ++s) {
             mbar_init(&kv_full[s], 1);
             mbar_init(&kv_empty[s], 1);
@@ -168,9 +172,11 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
             bool ok = true;
             for (int w = blockIdx.x; w < total && ok; w += gridDim.x, ++item_it) {
                 const Item it = decode_item(p, w);
-                if (!mbar_wait(q_empty, (item_it & 1) ^ 1, abort_flag, p.err)) break;
-                mbar_arrive_expect_tx(q_full, Cfg::kTileBytes);
-                tma_load_2d(sQ, &tmq, p.q_col0 + it.h * DH, it.q_row0, q_full);
+                // buffer qb holds items qb, qb + 2, ...: its (item_it / 2)-th use
+                const uint32_t qb = item_it & 1, qph = (item_it >> 1) & 1;
+                if (!mbar_wait(&q_empty[qb], qph ^ 1, abort_flag, p.err)) break;
+                mbar_arrive_expect_tx(&q_full[qb], Cfg::kTileBytes);
+                tma_load_2d(sQ + qb * Cfg::kTileBytes, &tmq, p.q_col0 + it.h * DH, it.q_row0, &q_full[qb]);
                 const int nkt = (it.nk + 127) / 128;
                 for (int j = 0; j < nkt; ++j, ++kv_it) {
                     const int s = kv_it % kKVStages;
@@ -199,7 +205,8 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
             // descriptors of the stage bases; a K step of 16 elements inside a
             // 128B / 64B swizzle atom advances the start address by 32 bytes,
             // i.e. the descriptor by 2
-            const uint64_t q_desc = make_sdesc(smem_u32(sQ), 16, Cfg::kAtom, Cfg::kSwz);
+            const uint64_t q_desc0 = make_sdesc(smem_u32(sQ), 16, Cfg::kAtom, Cfg::kSwz);
+            uint64_t q_desc = q_desc0;  // this item's Q buffer
             const uint64_t k_desc0 = make_sdesc(smem_u32(sK), 16, Cfg::kAtom, Cfg::kSwz);
             const uint64_t v_desc0 = make_sdesc(smem_u32(sV), Cfg::kAtom, Cfg::kAtom, Cfg::kSwz);
             constexpr uint64_t kStageStep = Cfg::kTileBytes >> 4, kVRowStep = (16 * Cfg::kRowBytes) >> 4;
@@ -237,7 +244,9 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
                 const uint32_t nkt = (uint32_t)((it.nk + 127) / 128);
                 // S of the first two tiles: their S buffers were freed by the
                 // previous item's P (waited on before its P V)
-                if (!mbar_wait(q_full, item_it & 1, abort_flag, p.err)) break;
+                const uint32_t qb = item_it & 1;
+                if (!mbar_wait(&q_full[qb], (item_it >> 1) & 1, abort_flag, p.err)) break;
+                q_desc = q_desc0 + qb * (Cfg::kTileBytes >> 4);
                 if (!kv_wait(g)) break;
                 tc_fence_after();
                 s_mmas(g);
@@ -263,7 +272,7 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
                     pv_mmas(gt, j < 2);
                 }
                 if (!ok) break;
-                mma_commit(q_empty);  // every S of the item issued: Q may be replaced
+                mma_commit(&q_empty[qb]);  // every S of the item issued: its Q buffer may be refilled
                 for (; j < nkt; ++j) {
                     const uint32_t gt = g + j;
                     if (!p_ready(gt) && !p_wait(gt)) {
