@@ -105,33 +105,38 @@ struct TmemSrc {
 
 template <int BN>
 struct WsSrc {
-    const float *ws;  // partial tile of split s of this tile at ws + (tile + s*tiles)*128*BN
+    const float *ws;  // partials of split s of this tile: unit (s * tiles + tile), chunk-major
     int tile, tiles, splits, row;
-    // 4 columns at a time: the loads of every split are issued before the
-    // in-order sum, so the reduction costs one L2 latency per 4 columns
+    // A chunk's 32 columns of two splits are loaded at once (16 float4 loads
+    // in flight per thread), then summed in split order from 0, so the
+    // reduction costs one L2 latency per chunk and two splits
     F3DC_DEV void operator()(int c0, float *v) const
     {
+        // chunk-major workspace (see the partial store): unit u = s * tiles + tile
         const size_t split_stride4 = (size_t)tiles * 128 * BN / 4;
-        const float4 *base = reinterpret_cast<const float4 *>(ws + ((size_t)tile * 128 + row) * BN + c0);
+        const float4 *base =
+            reinterpret_cast<const float4 *>(ws + (((size_t)tile * (BN / 32) + c0 / 32) * 128 + row) * 32);
 #pragma unroll
-        for (int c4 = 0; c4 < 8; ++c4) {
-            float4 part[kGemmMaxSplits];
+        for (int j = 0; j < 32; ++j) v[j] = 0.f;
+#pragma unroll 1
+        for (int s0 = 0; s0 < splits; s0 += 2) {
+            float4 part[2][8];
 #pragma unroll
-            for (int s = 0; s < kGemmMaxSplits; ++s)
-                if (s < splits) part[s] = __ldcg(base + s * split_stride4 + c4);
-            float4 a = make_float4(0.f, 0.f, 0.f, 0.f);
+            for (int u = 0; u < 2; ++u)
 #pragma unroll
-            for (int s = 0; s < kGemmMaxSplits; ++s)
-                if (s < splits) {
-                    a.x += part[s].x;
-                    a.y += part[s].y;
-                    a.z += part[s].z;
-                    a.w += part[s].w;
+                for (int c4 = 0; c4 < 8; ++c4)
+                    if (s0 + u < splits) part[u][c4] = __ldcg(base + (s0 + u) * split_stride4 + c4);
+#pragma unroll
+            for (int u = 0; u < 2; ++u)
+                if (s0 + u < splits) {
+#pragma unroll
+                    for (int c4 = 0; c4 < 8; ++c4) {
+                        v[4 * c4 + 0] += part[u][c4].x;
+                        v[4 * c4 + 1] += part[u][c4].y;
+                        v[4 * c4 + 2] += part[u][c4].z;
+                        v[4 * c4 + 3] += part[u][c4].w;
+                    }
                 }
-            v[4 * c4 + 0] = a.x;
-            v[4 * c4 + 1] = a.y;
-            v[4 * c4 + 2] = a.z;
-            v[4 * c4 + 3] = a.w;
         }
     }
 };
@@ -152,16 +157,18 @@ struct OutStage {
         *reinterpret_cast<uint4 *>(slot() + row * 64 + ((c ^ ((row >> 1) & 3)) << 4)) = u;
     }
     // publish the chunk just written and send it to (x, y) of the output
+    // (or of the tensor `to`, e.g. the split-K workspace)
     template <bool kReduce>
-    F3DC_DEV void emit(int x, int y)
+    F3DC_DEV void emit(int x, int y, const CUtensorMap *to = nullptr)
     {
         fence_proxy_async_smem();
         asm volatile("bar.sync 3, 128;" ::: "memory");
         if (threadIdx.x == 64) {
+            const CUtensorMap *m = to ? to : map;
             if (kReduce)
-                tma_reduce_add_2d(map, slot(), x, y);
+                tma_reduce_add_2d(m, slot(), x, y);
             else
-                tma_store_2d(map, slot(), x, y);
+                tma_store_2d(m, slot(), x, y);
             bulk_commit();
             // the chunk before this one has been read: its buffer, and every
             // older one, may be rewritten after the next barrier
@@ -184,12 +191,15 @@ F3DC_DEV void put_bf16x32(OutStage &o, const float *v)
     }
 }
 
+// Applies the epilogue to this tile's column chunks k0, k0 + kstep, ...
+// (chunks of 64 columns for QKNORM, whose RMSNorm groups span 64, else 32).
 template <int BN, int EPI, typename Src>
-F3DC_DEV void epilogue_tile(const GemmParams &p, const Src &src, OutStage &o, int m0, int n0)
+F3DC_DEV void epilogue_tile(const GemmParams &p, const Src &src, OutStage &o, int m0, int n0, int k0 = 0,
+                            int kstep = 1)
 {
     if constexpr (EPI == kEpiQKNorm) {
 #pragma unroll 1
-        for (int c0 = 0; c0 < BN; c0 += 64) {
+        for (int c0 = 64 * k0; c0 < BN; c0 += 64 * kstep) {
             float v[64];
             src(c0, v);
             src(c0 + 32, v + 32);
@@ -220,7 +230,7 @@ F3DC_DEV void epilogue_tile(const GemmParams &p, const Src &src, OutStage &o, in
         }
     } else {
 #pragma unroll 1
-        for (int c0 = 0; c0 < BN; c0 += 32) {
+        for (int c0 = 32 * k0; c0 < BN; c0 += 32 * kstep) {
             float v[32];
             src(c0, v);
             const int col = n0 + c0;
@@ -271,7 +281,7 @@ struct Units {
 template <int BN, int EPI>
 __global__ void __launch_bounds__(kGemmThreads, 1)
     k_gemm(const __grid_constant__ CUtensorMap tma, const __grid_constant__ CUtensorMap tmb,
-           const __grid_constant__ CUtensorMap tmo, const GemmParams p)
+           const __grid_constant__ CUtensorMap tmo, const __grid_constant__ CUtensorMap tmw, const GemmParams p)
 {
     using Cfg = GemmCfg<BN>;
     constexpr int S = Cfg::kStages;
@@ -419,37 +429,68 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
                 if (lane == 0) mbar_arrive(&acce[buf]);
                 continue;
             }
-            // split K: store this split's fp32 partial row, free TMEM, and let
-            // the last CTA to finish the tile reduce the splits in order
-            float *wrow = p.ws + ((size_t)t * 128 + row) * BN;
+            // split K.  Each split stores its fp32 partial tile in the
+            // workspace, chunk-major (unit u's 32-column chunk k: 128 rows of
+            // 32 floats at row (u * BN / 32 + k) * 128 of the workspace
+            // tensor), through the staged TMA stores; frees TMEM; and arrives
+            // on the tile's counter.  Once every split has arrived, split s
+            // reduces chunks s, s + S, ... of the tile -- all partials summed
+            // in split order, so results do not depend on timing -- and
+            // applies the epilogue to them.  When splitting, a CTA holds at
+            // most one unit (tiles * splits <= grid <= SMs, one CTA per SM),
+            // so the wait below never waits on work queued behind itself.
+            const int tile = t % U.tiles, split = t / U.tiles;
 #pragma unroll 1
             for (int c0 = 0; c0 < BN; c0 += 32) {
                 float v[32];
                 tsrc(c0, v);
+                const int y = (t * (BN / 32) + c0 / 32) * 128;
 #pragma unroll
-                for (int q4 = 0; q4 < 8; ++q4)
-                    __stcg(reinterpret_cast<float4 *>(wrow + c0) + q4,
-                           make_float4(v[4 * q4], v[4 * q4 + 1], v[4 * q4 + 2], v[4 * q4 + 3]));
+                for (int h = 0; h < 2; ++h) {
+#pragma unroll
+                    for (int q4 = 0; q4 < 4; ++q4) {
+                        const float *w = v + 16 * h + 4 * q4;
+                        o.put16(q4, make_uint4(__float_as_uint(w[0]), __float_as_uint(w[1]), __float_as_uint(w[2]),
+                                               __float_as_uint(w[3])));
+                    }
+                    o.template emit<false>(16 * h, y, &tmw);
+                }
             }
             tc_fence_before();
             __syncwarp();
             if (lane == 0) mbar_arrive(&acce[buf]);
-            const int tile = t % U.tiles;
-            __threadfence();
             asm volatile("bar.sync 2, 128;" ::: "memory");
             if (threadIdx.x == 64) {
-                const int prev = atomicAdd(p.counters + tile, 1);
-                const int last = prev == U.splits - 1;
-                if (last) p.counters[tile] = 0;  // ready for the next launch
-                *split_flag = last;
-            }
-            asm volatile("bar.sync 2, 128;" ::: "memory");
-            if (*split_flag) {
+                // the partial's TMA stores are complete and visible before
+                // the arrival
+                bulk_wait_all();
+                asm volatile("fence.proxy.async.global;" ::: "memory");
                 __threadfence();
-                const WsSrc<BN> wsrc{p.ws, tile, U.tiles, U.splits, row};
-                epilogue_tile<BN, EPI>(p, wsrc, o, m0, n0);
+                atomicAdd(p.counters + tile, 1);
+                int ok = 1;
+                const uint64_t t0 = globaltimer();
+                while (*reinterpret_cast<volatile int32_t *>(p.counters + tile) < U.splits) {
+                    if (*abort_flag || globaltimer() - t0 > kWaitLimitNs) {
+                        *abort_flag = 1;
+                        raise_error(p.err, kDevTimeout);
+                        ok = 0;
+                        break;
+                    }
+                }
+                __threadfence();
+                *split_flag = ok;
             }
             asm volatile("bar.sync 2, 128;" ::: "memory");
+            if (!*split_flag) break;
+            __threadfence();
+            const WsSrc<BN> wsrc{p.ws, tile, U.tiles, U.splits, row};
+            epilogue_tile<BN, EPI>(p, wsrc, o, m0, n0, split, U.splits);
+            asm volatile("bar.sync 2, 128;" ::: "memory");
+            if (threadIdx.x == 64) {
+                // every split has read what it needs: the last one to get here
+                // returns the counter to 0 for the next launch
+                if (atomicAdd(p.counters + tile, 1) == 2 * U.splits - 1) p.counters[tile] = 0;
+            }
         }
         // this CTA's output stores complete before it ends
         if (threadIdx.x == 64) bulk_wait_all();
@@ -471,8 +512,8 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
 }
 
 template <int BN, int EPI>
-cudaError_t launch_one(const CUtensorMap *ta, const CUtensorMap *tb, const CUtensorMap *to, const GemmParams &p,
-                       int grid, cudaStream_t s)
+cudaError_t launch_one(const CUtensorMap *ta, const CUtensorMap *tb, const CUtensorMap *to, const CUtensorMap *tw,
+                       const GemmParams &p, int grid, cudaStream_t s)
 {
     static bool attr_set = false;
     const size_t smem = GemmCfg<BN>::kSmem;
@@ -481,19 +522,19 @@ cudaError_t launch_one(const CUtensorMap *ta, const CUtensorMap *tb, const CUten
         if (e != cudaSuccess) return e;
         attr_set = true;
     }
-    launch_k(k_gemm<BN, EPI>, dim3(grid), dim3(kGemmThreads), smem, s, *ta, *tb, *to, p);
+    launch_k(k_gemm<BN, EPI>, dim3(grid), dim3(kGemmThreads), smem, s, *ta, *tb, *to, *tw, p);
     return cudaGetLastError();
 }
 
 template <int BN>
-cudaError_t launch_bn(const CUtensorMap *ta, const CUtensorMap *tb, const CUtensorMap *to, const GemmParams &p,
-                      int epi, int grid, cudaStream_t s)
+cudaError_t launch_bn(const CUtensorMap *ta, const CUtensorMap *tb, const CUtensorMap *to, const CUtensorMap *tw,
+                      const GemmParams &p, int epi, int grid, cudaStream_t s)
 {
     switch (epi) {
-    case kEpiBias: return launch_one<BN, kEpiBias>(ta, tb, to, p, grid, s);
-    case kEpiGelu: return launch_one<BN, kEpiGelu>(ta, tb, to, p, grid, s);
-    case kEpiResid: return launch_one<BN, kEpiResid>(ta, tb, to, p, grid, s);
-    case kEpiQKNorm: return launch_one<BN, kEpiQKNorm>(ta, tb, to, p, grid, s);
+    case kEpiBias: return launch_one<BN, kEpiBias>(ta, tb, to, tw, p, grid, s);
+    case kEpiGelu: return launch_one<BN, kEpiGelu>(ta, tb, to, tw, p, grid, s);
+    case kEpiResid: return launch_one<BN, kEpiResid>(ta, tb, to, tw, p, grid, s);
+    case kEpiQKNorm: return launch_one<BN, kEpiQKNorm>(ta, tb, to, tw, p, grid, s);
     default: return cudaErrorInvalidValue;
     }
 }
@@ -547,13 +588,21 @@ cudaError_t launch_gemm(const CUtensorMap *ta, const CUtensorMap *tb, const Gemm
                         int grid, cudaStream_t s)
 {
     if (p.K % kBK != 0 || p.N % bn != 0 || grid < 1) return cudaErrorInvalidValue;
-    CUtensorMap to;
+    CUtensorMap to, tw;
     if (!make_tmap_out(&to, p.out, (uint64_t)p.M, (uint64_t)p.N, (uint64_t)p.ldo, epi == kEpiResid))
         return cudaErrorInvalidValue;
+    // split-K workspace as a [ws_units * bn / 32 * 128, 32] fp32 tensor
+    // (chunk-major partial tiles); without a workspace the output map stands in
+    if (p.ws) {
+        if (!make_tmap_out(&tw, p.ws, (uint64_t)p.ws_units * (bn / 32) * 128, 32, 32, true))
+            return cudaErrorInvalidValue;
+    } else {
+        tw = to;
+    }
     switch (bn) {
-    case 64: return launch_bn<64>(ta, tb, &to, p, epi, grid, s);
-    case 128: return launch_bn<128>(ta, tb, &to, p, epi, grid, s);
-    case 256: return launch_bn<256>(ta, tb, &to, p, epi, grid, s);
+    case 64: return launch_bn<64>(ta, tb, &to, &tw, p, epi, grid, s);
+    case 128: return launch_bn<128>(ta, tb, &to, &tw, p, epi, grid, s);
+    case 256: return launch_bn<256>(ta, tb, &to, &tw, p, epi, grid, s);
     default: return cudaErrorInvalidValue;
     }
 }

@@ -124,7 +124,7 @@ struct GemmParams {
 cudaError_t launch_gemm(const CUtensorMap *ta, const CUtensorMap *tb, const GemmParams &p, int epi, int bn,
                         int grid, cudaStream_t s);
 size_t gemm_smem_bytes(int bn);
-// bytes of split-K workspace for `units` partial tiles of width bn
+
 // Launches a kernel of this library with programmatic stream serialization
 // (programmatic dependent launch): the kernel may start while the previous
 // kernel in the stream finishes and waits for it in griddep_wait().
@@ -144,6 +144,7 @@ cudaError_t launch_k(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t sme
     return cudaLaunchKernelEx(&cfg, kernel, args...);
 }
 
+// bytes of split-K workspace for `units` partial tiles of width bn
 inline size_t gemm_ws_bytes(int bn, int units) { return (size_t)units * 128 * bn * sizeof(float); }
 constexpr int kGemmMaxCounterTiles = 1024;
 
@@ -155,7 +156,9 @@ constexpr int kGemmMaxCounterTiles = 1024;
 constexpr int kGemmMaxSplits = 16;
 __host__ __device__ inline int gemm_split_count(int tiles, int grid, int kb_n, int ws_units, bool have_ws)
 {
-    if (!have_ws || tiles <= 0 || 2 * tiles > grid || tiles > kGemmMaxCounterTiles) return 1;
+    // only a long K loop (K >= 2048) saves more than the partials' round trip
+    // through L2 and the in-order reduction cost
+    if (!have_ws || tiles <= 0 || 2 * tiles > grid || tiles > kGemmMaxCounterTiles || kb_n < 32) return 1;
     int sp = grid / tiles;
     if (sp > kb_n / 4) sp = kb_n / 4;
     if (sp > ws_units / tiles) sp = ws_units / tiles;
