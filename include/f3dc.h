@@ -274,11 +274,13 @@ f3dc_status f3dc_forward(f3dc_handle *h, float t, int32_t B, const float *S,
 #define F3DC_EPI_RESID 2  /* out fp32 += gate * (acc + bias), gate nullable (1) */
 
 /* out[m, n] = epi(sum_k A[m, k] B[n, k]) -- the tcgen05 GEMM of the
- * transformer (nn.Linear convention: B is [N, K] row-major).  When there are
- * few 128-row tiles the K range is split over several CTAs whose fp32 partials
- * go to a split-K workspace that this call allocates once per device and keeps
- * for the life of the process; results do not depend on the split (partials
- * are summed in a fixed order), and calls on one device must not overlap.
+ * transformer (nn.Linear convention: B is [N, K] row-major).  When the output
+ * tiles (128 rows x 64/128/256 columns) would leave at least half of the SMs
+ * idle and K >= 2048, the K range is split over several CTAs whose fp32
+ * partials go to a split-K workspace that this call allocates once per device
+ * and keeps for the life of the process; results do not depend on the split
+ * (partials are summed in a fixed order), and calls on one device must not
+ * overlap.
  *   A: device bf16 [M, K] row-major; B: device bf16 [N, K] row-major;
  *   bias: device bf16 [N], nullable; gate: device fp32 [N], nullable;
  *   out: device bf16 [M, N] (BIAS, GELU) or fp32 [M, N] (RESID).
