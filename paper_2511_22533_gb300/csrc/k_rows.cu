@@ -36,53 +36,92 @@ F3DC_DEV float bf16_at(const bf16 *p, size_t i)
 }
 
 // ------------------------------------------------------------------ K2
-__global__ void __launch_bounds__(kRowThreads) k_gather_embed(const float *S, int N, int W,
-                                                              const int32_t *active_idx, const Plan *plan,
-                                                              const int32_t *tile_sample, const bf16 *in_w,
-                                                              const bf16 *in_b, const float *pos, float *x,
-                                                              uint32_t *err)
+// Work unit: 32 consecutive packed rows (a quarter of a 128-row tile, so one
+// sample).  Threads 0..31 resolve the unit's rows to tokens (tile -> sample
+// -> active index -> latent) once and stage index and latent in shared
+// memory; then every thread owns one float4 of columns (its 4 x 8 input
+// weights and 4 biases held in registers for the whole kernel) and streams
+// the rows, issuing the position-embedding loads of 8 rows before using any.
+// Per column: acc = b_n, acc = fma(S_c, W_nc, acc) for c = 0..7, x = pos + acc.
+constexpr int kGatherUnit = 32;
+template <int NV>
+struct GatherCfg {
+    static constexpr int kT = 32 * NV;                        // threads per row
+    static constexpr int kThreads = kT < 256 ? 256 : kT;
+    static constexpr int kRPI = kThreads / kT;                 // rows per pass
+    static constexpr int kU = kRPI >= 8 ? 1 : (NV == 16 ? 4 : 8 / kRPI);  // passes unrolled
+};
+
+template <int NV>
+__global__ void __launch_bounds__(GatherCfg<NV>::kThreads, GatherCfg<NV>::kThreads >= 512 ? 1 : 2)
+    k_gather_embed(const float *S, int N, const int32_t *active_idx, const Plan *plan, const int32_t *tile_sample,
+                   const bf16 *in_w, const bf16 *in_b, const float *pos, float *x, uint32_t *err)
 {
+    using Cfg = GatherCfg<NV>;
+    constexpr int W = 128 * NV;
+    __shared__ int s_idx[kGatherUnit];
+    __shared__ float4 s_lat[kGatherUnit][2];
+    const int t = threadIdx.x, q = t % Cfg::kT, rsub = t / Cfg::kT;
+    // this thread's columns 4q .. 4q+3: weights and biases
+    float wv[4][8], bv[4];
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+        bf16x8_to_f32(__ldg(reinterpret_cast<const uint4 *>(in_w) + 4 * q + u), wv[u]);
+        bv[u] = bf16_at(in_b, 4 * q + u);
+    }
     griddep_launch();
     griddep_wait();
-    const int m_rows = plan->m_rows;
-    const int lane = threadIdx.x & 31, wpb = blockDim.x >> 5;
-    for (int r = blockIdx.x * wpb + (threadIdx.x >> 5); r < m_rows; r += gridDim.x * wpb) {
-        const int b = tile_sample[r / kTileRows];
-        const int j = r - plan->row_off[b];
-        float *xr = x + (size_t)r * W;
-        int i = -1;
-        if (j < plan->n_active[b]) {
-            i = active_idx[(size_t)b * N + j];
-            if ((unsigned)i >= (unsigned)N) {
-                raise_error(err, kDevBadIndex);
-                i = -1;
+    const int units = plan->m_rows / kGatherUnit;
+    for (int unit = blockIdx.x; unit < units; unit += gridDim.x) {
+        const int r0 = unit * kGatherUnit;
+        if (t < kGatherUnit) {
+            const int b = tile_sample[r0 / kTileRows];
+            const int j = r0 + t - plan->row_off[b];
+            int i = -1;
+            if (j < plan->n_active[b]) {
+                i = active_idx[(size_t)b * N + j];
+                if ((unsigned)i >= (unsigned)N) {
+                    raise_error(err, kDevBadIndex);
+                    i = -1;
+                }
+            }
+            s_idx[t] = i;
+            if (i >= 0) {
+                const float *Si = S + ((size_t)b * N + i) * kChannels;
+                s_lat[t][0] = ld_f4(Si);
+                s_lat[t][1] = ld_f4(Si + 4);
             }
         }
-        if (i < 0) {  // padding row: zeros keep every downstream value finite
-            for (int q = lane; q < W / 4; q += 32) st_f4(xr + 4 * q, make_float4(0.f, 0.f, 0.f, 0.f));
-            continue;
-        }
-        const float *Si = S + ((size_t)b * N + i) * kChannels;
-        float s[8];
-        const float4 s0 = ld_f4(Si), s1 = ld_f4(Si + 4);
-        s[0] = s0.x; s[1] = s0.y; s[2] = s0.z; s[3] = s0.w;
-        s[4] = s1.x; s[5] = s1.y; s[6] = s1.z; s[7] = s1.w;
-        const float *pi = pos + (size_t)i * W;
-        for (int q = lane; q < W / 4; q += 32) {
-            const float4 pe = ld_f4(pi + 4 * q);
-            float o[4] = {pe.x, pe.y, pe.z, pe.w};
+        __syncthreads();
+#pragma unroll 1
+        for (int p0 = 0; p0 < kGatherUnit; p0 += Cfg::kRPI * Cfg::kU) {
+            float4 pe[Cfg::kU];
 #pragma unroll
-            for (int u = 0; u < 4; ++u) {
-                const int n = 4 * q + u;
-                float wv[8];
-                bf16x8_to_f32(__ldg(reinterpret_cast<const uint4 *>(in_w) + n), wv);
-                float acc = bf16_at(in_b, n);
-#pragma unroll
-                for (int c = 0; c < 8; ++c) acc = fmaf(s[c], wv[c], acc);
-                o[u] += acc;
+            for (int u = 0; u < Cfg::kU; ++u) {
+                const int i = s_idx[p0 + u * Cfg::kRPI + rsub];
+                pe[u] = i >= 0 ? __ldg(reinterpret_cast<const float4 *>(pos + (size_t)i * W) + q)
+                               : make_float4(0.f, 0.f, 0.f, 0.f);
             }
-            st_f4(xr + 4 * q, make_float4(o[0], o[1], o[2], o[3]));
+#pragma unroll
+            for (int u = 0; u < Cfg::kU; ++u) {
+                const int rr = p0 + u * Cfg::kRPI + rsub;
+                float4 o = make_float4(0.f, 0.f, 0.f, 0.f);
+                if (s_idx[rr] >= 0) {  // padding rows stay zero: every downstream value finite
+                    const float4 l0 = s_lat[rr][0], l1 = s_lat[rr][1];
+                    const float sl[8] = {l0.x, l0.y, l0.z, l0.w, l1.x, l1.y, l1.z, l1.w};
+                    float acc[4];
+#pragma unroll
+                    for (int c4 = 0; c4 < 4; ++c4) {
+                        acc[c4] = bv[c4];
+#pragma unroll
+                        for (int c = 0; c < 8; ++c) acc[c4] = fmaf(sl[c], wv[c4][c], acc[c4]);
+                    }
+                    o = make_float4(pe[u].x + acc[0], pe[u].y + acc[1], pe[u].z + acc[2], pe[u].w + acc[3]);
+                }
+                st_f4(x + (size_t)(r0 + rr) * W + 4 * q, o);
+            }
         }
+        __syncthreads();
     }
 }
 
@@ -374,13 +413,30 @@ int row_grid(int num_sms, int max_rows)
 
 }  // namespace
 
+template <int NV>
+void launch_gather_nv(const float *S, int N, const int32_t *active_idx, const Plan *plan, const int32_t *tile_sample,
+                      const bf16 *in_w, const bf16 *in_b, const float *pos, float *x, int max_rows, int num_sms,
+                      uint32_t *err, cudaStream_t s)
+{
+    const int units = max_rows / kGatherUnit;
+    const int grid = units < 2 * num_sms ? (units > 0 ? units : 1) : 2 * num_sms;
+    launch_k(k_gather_embed<NV>, dim3(grid), dim3(GatherCfg<NV>::kThreads), 0, s, S, N, active_idx, plan, tile_sample,
+             in_w, in_b, pos, x, err);
+}
+
 cudaError_t launch_gather_embed(const float *S, int N, int W, const int32_t *active_idx, const Plan *plan,
                                 const int32_t *tile_sample, const bf16 *in_w, const bf16 *in_b,
                                 const float *pos, float *x, int max_rows, int num_sms, uint32_t *err,
                                 cudaStream_t s)
 {
-    launch_k(k_gather_embed, dim3(row_grid(num_sms, max_rows)), dim3(kRowThreads), 0, s, S, N, W, active_idx, plan, tile_sample,
-                                                                       in_w, in_b, pos, x, err);
+    switch (W / 128) {
+    case 1: launch_gather_nv<1>(S, N, active_idx, plan, tile_sample, in_w, in_b, pos, x, max_rows, num_sms, err, s); break;
+    case 2: launch_gather_nv<2>(S, N, active_idx, plan, tile_sample, in_w, in_b, pos, x, max_rows, num_sms, err, s); break;
+    case 4: launch_gather_nv<4>(S, N, active_idx, plan, tile_sample, in_w, in_b, pos, x, max_rows, num_sms, err, s); break;
+    case 8: launch_gather_nv<8>(S, N, active_idx, plan, tile_sample, in_w, in_b, pos, x, max_rows, num_sms, err, s); break;
+    case 16: launch_gather_nv<16>(S, N, active_idx, plan, tile_sample, in_w, in_b, pos, x, max_rows, num_sms, err, s); break;
+    default: return cudaErrorInvalidValue;
+    }
     return cudaGetLastError();
 }
 

@@ -4,13 +4,14 @@
 // step (Sec. 4.2 index-based token compaction).
 //
 // One CTA of 1024 threads per sample.  Pass 1 streams the two newest
-// velocity slots (16 B + 16 B per token, coalesced uint4 loads) and reduces
-// min / max of V and A; pass 2 re-reads them (L2-resident), forms the score
-// in the same fp32 operation order as the definition and stores an order-
-// preserving 32-bit key per token in shared memory.  A 4 x 8-bit radix
-// select finds the c-th smallest key; an index-ordered scan then caches
-// every key below it plus the lowest-index ties, and compacts the active
-// tokens in ascending order.
+// velocity slots (16 B + 16 B per token, coalesced uint4 loads, a thread's
+// first four tokens in one round of loads) and reduces min / max of V and A;
+// pass 2 takes V and A from registers (re-reading tokens beyond the first
+// 4096 from L2), forms the score in the same fp32 operation order as the
+// definition and stores an order-preserving 32-bit key per token in shared
+// memory.  A 4 x 8-bit radix select finds the c-th smallest key; an
+// index-ordered scan then caches every key below it plus the lowest-index
+// ties, and compacts the active tokens in ascending order.
 #include "common.cuh"
 #include "kernels.h"
 
@@ -20,7 +21,8 @@ namespace {
 
 constexpr int kSelThreads = 1024;
 constexpr int kSelWarps = kSelThreads / 32;
-constexpr int kSelMaxTokens = 49152;  // 4-byte keys in shared memory
+constexpr int kSelMaxTokens = 49152;  // 4-byte keys in shared memory (192 KB + 16 KB of histograms)
+constexpr int kRegTok = 4;            // tokens per thread held in registers between passes 1 and 2
 
 F3DC_DEV void load_token(const uint16_t *v1, const uint16_t *v2, size_t tok, float &V, float &A)
 {
@@ -65,22 +67,32 @@ F3DC_DEV int pad_tile(int a) { return (a + kTileRows - 1) / kTileRows * kTileRow
 
 F3DC_DEV int clamp_quota(int q, int N) { return q < 0 ? 0 : (q > N ? N : q); }
 
-// Row offset of sample b, total padded rows, and the sample's tiles.
+// Row offset of sample b, total padded rows, and the sample's tiles.  The
+// first warp sums the padded row counts of all samples (B <= 64: two per
+// lane) in one round of loads.
+static_assert(kMaxBatch <= 64, "write_plan covers two samples per lane");
 F3DC_DEV void write_plan(const SelectArgs &a, int b, int na, int &off)
 {
     __shared__ int s_off;
-    if (threadIdx.x == 0) {
-        int o = 0;
-        for (int bb = 0; bb < b; ++bb) o += pad_tile(a.N - clamp_quota(a.quota[bb], a.N));
-        s_off = o;
-        if (a.plan) {
-            a.plan->n_active[b] = na;
-            a.plan->row_off[b] = o;
-            if (b == 0) {
-                int tot = 0;
-                for (int bb = 0; bb < a.B; ++bb) tot += pad_tile(a.N - clamp_quota(a.quota[bb], a.N));
-                a.plan->m_rows = tot;
-                a.plan->n_tiles = tot / kTileRows;
+    if (threadIdx.x < 32) {
+        const int lane = threadIdx.x;
+        const int r0 = lane < a.B ? pad_tile(a.N - clamp_quota(a.quota[lane], a.N)) : 0;
+        const int r1 = lane + 32 < a.B ? pad_tile(a.N - clamp_quota(a.quota[lane + 32], a.N)) : 0;
+        int before = (lane < b ? r0 : 0) + (lane + 32 < b ? r1 : 0), tot = r0 + r1;
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) {
+            before += __shfl_xor_sync(0xffffffffu, before, o);
+            tot += __shfl_xor_sync(0xffffffffu, tot, o);
+        }
+        if (lane == 0) {
+            s_off = before;
+            if (a.plan) {
+                a.plan->n_active[b] = na;
+                a.plan->row_off[b] = before;
+                if (b == 0) {
+                    a.plan->m_rows = tot;
+                    a.plan->n_tiles = tot / kTileRows;
+                }
             }
         }
     }
@@ -97,10 +109,10 @@ __global__ void __launch_bounds__(kSelThreads, 1) k_ssc_select(const SelectArgs 
     griddep_launch();
     griddep_wait();
     extern __shared__ uint32_t keys[];
-    __shared__ uint32_t hist[256];
+    __shared__ uint32_t whist[16][256];
     __shared__ float red[4][kSelWarps];
-    __shared__ uint32_t wsum_lt[kSelWarps], wsum_eq[kSelWarps];
-    __shared__ uint32_t s_digit, s_rank;
+    __shared__ uint32_t wsum[kSelWarps], wpre[kSelWarps];
+    __shared__ uint32_t s_digit, s_rank, s_tot;
 
     const int b = blockIdx.x, tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     const int N = a.N;
@@ -128,9 +140,27 @@ __global__ void __launch_bounds__(kSelThreads, 1) k_ssc_select(const SelectArgs 
         return;
     }
 
-    // ---- pass 1: min / max of V and A (NaN never wins a comparison)
+    // ---- pass 1: min / max of V and A (NaN never wins a comparison).  The
+    // first kRegTok tokens of each thread are loaded together and kept in
+    // registers for pass 2; tokens beyond them are re-read there.
     float mnV = INFINITY, mxV = -INFINITY, mnA = INFINITY, mxA = -INFINITY;
-    for (int i = tid; i < N; i += kSelThreads) {
+    float Vr[kRegTok], Ar[kRegTok];
+#pragma unroll
+    for (int r = 0; r < kRegTok; ++r) {
+        const int i = tid + r * kSelThreads;
+        Vr[r] = Ar[r] = 0.0f;
+        if (i < N) load_token(a.v1, a.v2, base + i, Vr[r], Ar[r]);
+    }
+#pragma unroll
+    for (int r = 0; r < kRegTok; ++r) {
+        if (tid + r * kSelThreads < N) {
+            if (Vr[r] < mnV) mnV = Vr[r];
+            if (Vr[r] > mxV) mxV = Vr[r];
+            if (Ar[r] < mnA) mnA = Ar[r];
+            if (Ar[r] > mxA) mxA = Ar[r];
+        }
+    }
+    for (int i = tid + kRegTok * kSelThreads; i < N; i += kSelThreads) {
         float V, A;
         load_token(a.v1, a.v2, base + i, V, A);
         if (V < mnV) mnV = V;
@@ -165,107 +195,136 @@ __global__ void __launch_bounds__(kSelThreads, 1) k_ssc_select(const SelectArgs 
     }
 
     // ---- pass 2: C_i = w_a norm(A_i) + w_v norm(V_i) -> ordered keys
-    for (int i = tid; i < N; i += kSelThreads) {
+    auto score = [&](float V, float A) {
+        return __fadd_rn(__fmul_rn(a.wa, norm1(A, mnA, mxA)), __fmul_rn(a.wv, norm1(V, mnV, mxV)));
+    };
+#pragma unroll
+    for (int r = 0; r < kRegTok; ++r) {
+        const int i = tid + r * kSelThreads;
+        if (i < N) keys[i] = score_key(score(Vr[r], Ar[r]));
+    }
+    for (int i = tid + kRegTok * kSelThreads; i < N; i += kSelThreads) {
         float V, A;
         load_token(a.v1, a.v2, base + i, V, A);
-        const float s = __fadd_rn(__fmul_rn(a.wa, norm1(A, mnA, mxA)), __fmul_rn(a.wv, norm1(V, mnV, mxV)));
-        keys[i] = score_key(s);
+        keys[i] = score_key(score(V, A));
     }
     __syncthreads();
 
-    // ---- radix select: the c-th smallest key (1-based rank c)
+    // ---- radix select: the c-th smallest key (1-based rank c).  Each pair of
+    // warps counts digits into its own 256-bin histogram with plain shared-
+    // memory atomics; threads 0..255 then sum the 16 histograms bin by bin
+    // and scan them, and the one bin holding rank `rank` fixes the digit.
     uint32_t prefix = 0, hi_mask = 0;
     uint32_t rank = (uint32_t)c;
     for (int shift = 24; shift >= 0; shift -= 8) {
-        if (tid < 256) hist[tid] = 0;
+        for (int q = tid; q < 16 * 256; q += kSelThreads) (&whist[0][0])[q] = 0;
         __syncthreads();
-        for (int i0 = 0; i0 < N; i0 += kSelThreads) {
-            const int i = i0 + tid;
-            const bool in = i < N && (keys[i] & hi_mask) == prefix;
-            const uint32_t digit = in ? (keys[i] >> shift) & 255u : 256u;
-            const uint32_t peers = __match_any_sync(0xffffffffu, digit);
-            if (in && (__ffs(peers) - 1) == lane) atomicAdd(&hist[digit], (uint32_t)__popc(peers));
+        uint32_t *mine = whist[warp >> 1];
+        for (int i = tid; i < N; i += kSelThreads) {
+            const uint32_t k = keys[i];
+            if ((k & hi_mask) == prefix) atomicAdd(&mine[(k >> shift) & 255u], 1u);
         }
         __syncthreads();
-        if (warp == 0) {
-            uint32_t loc[8], sum = 0;
+        uint32_t v = 0, incl = 0;
+        if (tid < 256) {
 #pragma unroll
-            for (int j = 0; j < 8; ++j) {
-                loc[j] = hist[lane * 8 + j];
-                sum += loc[j];
-            }
-            uint32_t incl = sum;
+            for (int w = 0; w < 16; ++w) v += whist[w][tid];
+            incl = v;
 #pragma unroll
             for (int o = 1; o < 32; o <<= 1) {
                 const uint32_t n = __shfl_up_sync(0xffffffffu, incl, o);
                 if (lane >= o) incl += n;
             }
-            const uint32_t excl = incl - sum;
+            if (lane == 31) wsum[warp] = incl;
+        }
+        __syncthreads();
+        if (tid < 256) {
+            for (int w = 0; w < warp; ++w) incl += wsum[w];
+            const uint32_t excl = incl - v;
             if (excl < rank && rank <= incl) {
-                uint32_t cum = excl;
-#pragma unroll
-                for (int j = 0; j < 8; ++j) {
-                    if (cum + loc[j] >= rank) {
-                        s_digit = (uint32_t)(lane * 8 + j);
-                        s_rank = rank - cum;
-                        break;
-                    }
-                    cum += loc[j];
-                }
+                s_digit = (uint32_t)tid;
+                s_rank = rank - excl;
             }
         }
         __syncthreads();
         prefix |= s_digit << shift;
         hi_mask |= 255u << shift;
         rank = s_rank;
-        __syncthreads();
     }
     const uint32_t thr = prefix;  // keys below thr are cached, plus the first `rank` ties
 
     // ---- index-ordered compaction.  For token i with L(i) smaller keys and
     // E(i) ties before it, the tie is cached iff E(i) < rank, and an active
-    // token lands at position i - L(i) - min(E(i), rank).
+    // token lands at position i - L(i) - min(E(i), rank).  Each thread takes
+    // four consecutive tokens; one block-wide scan of the packed counts
+    // (L in the low, E in the high 16 bits) per 4096 tokens.
     uint32_t run_lt = 0, run_eq = 0;
-    const uint32_t lt_mask = (1u << lane) - 1u;
-    for (int i0 = 0; i0 < N; i0 += kSelThreads) {
-        const int i = i0 + tid;
-        const bool valid = i < N;
-        const uint32_t k = valid ? keys[i] : 0xFFFFFFFFu;
-        const bool lt = valid && k < thr;
-        const bool eq = valid && k == thr;
-        const uint32_t blt = __ballot_sync(0xffffffffu, lt), beq = __ballot_sync(0xffffffffu, eq);
-        if (lane == 0) {
-            wsum_lt[warp] = __popc(blt);
-            wsum_eq[warp] = __popc(beq);
+    for (int i0 = 0; i0 < N; i0 += 4 * kSelThreads) {
+        const int i = i0 + 4 * tid;
+        uint32_t k[4];
+        if (i + 3 < N) {
+            const uint4 kk = *reinterpret_cast<const uint4 *>(keys + i);
+            k[0] = kk.x;
+            k[1] = kk.y;
+            k[2] = kk.z;
+            k[3] = kk.w;
+        } else {
+#pragma unroll
+            for (int r = 0; r < 4; ++r) k[r] = i + r < N ? keys[i + r] : 0u;
+        }
+        uint32_t ltb = 0, eqb = 0;
+#pragma unroll
+        for (int r = 0; r < 4; ++r) {
+            if (i + r < N) {
+                ltb |= (uint32_t)(k[r] < thr) << r;
+                eqb |= (uint32_t)(k[r] == thr) << r;
+            }
+        }
+        const uint32_t cnt = (uint32_t)__popc(ltb) | ((uint32_t)__popc(eqb) << 16);
+        uint32_t incl = cnt;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+            const uint32_t n = __shfl_up_sync(0xffffffffu, incl, o);
+            if (lane >= o) incl += n;
+        }
+        if (lane == 31) wsum[warp] = incl;
+        __syncthreads();
+        if (warp == 0) {
+            const uint32_t x = wsum[lane];
+            uint32_t wi = x;
+#pragma unroll
+            for (int o = 1; o < 32; o <<= 1) {
+                const uint32_t n = __shfl_up_sync(0xffffffffu, wi, o);
+                if (lane >= o) wi += n;
+            }
+            wpre[lane] = wi - x;
+            if (lane == 31) s_tot = wi;
         }
         __syncthreads();
-        uint32_t plt = run_lt + __popc(blt & lt_mask), peq = run_eq + __popc(beq & lt_mask);
-        uint32_t tot_lt = 0, tot_eq = 0;
-        for (int w = 0; w < kSelWarps; ++w) {
-            const uint32_t x = wsum_lt[w], y = wsum_eq[w];
-            if (w < warp) {
-                plt += x;
-                peq += y;
-            }
-            tot_lt += x;
-            tot_eq += y;
-        }
-        if (valid) {
+        const uint32_t pre = wpre[warp] + incl - cnt;
+        uint32_t plt = run_lt + (pre & 0xFFFFu), peq = run_eq + (pre >> 16);
+#pragma unroll
+        for (int r = 0; r < 4; ++r) {
+            if (i + r >= N) break;
+            const bool lt = (ltb >> r) & 1u, eq = (eqb >> r) & 1u;
             const bool cached = lt || (eq && peq < rank);
-            if (a.mask) a.mask[base + i] = cached ? 1 : 0;
+            if (a.mask) a.mask[base + i + r] = cached ? 1 : 0;
             if (!cached) {
-                const uint32_t pos = (uint32_t)i - plt - min(peq, rank);
+                const uint32_t pos = (uint32_t)(i + r) - plt - min(peq, rank);
                 if (pos >= (uint32_t)na) raise_error(a.err, kDevBadPlan);
                 else {
-                    a.active_idx[base + pos] = i;
-                    if (a.row_of_token) a.row_of_token[base + i] = off + (int)pos;
+                    a.active_idx[base + pos] = i + r;
+                    if (a.row_of_token) a.row_of_token[base + i + r] = off + (int)pos;
                 }
             } else if (a.row_of_token) {
-                a.row_of_token[base + i] = -1;
+                a.row_of_token[base + i + r] = -1;
             }
+            plt += lt;
+            peq += eq;
         }
-        run_lt += tot_lt;
-        run_eq += tot_eq;
+        const uint32_t tot = s_tot;
+        run_lt += tot & 0xFFFFu;
+        run_eq += tot >> 16;
         __syncthreads();
     }
     if (tid == 0 && (uint32_t)N - run_lt - min(run_eq, rank) != (uint32_t)na) raise_error(a.err, kDevBadPlan);
