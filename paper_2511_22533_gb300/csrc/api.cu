@@ -381,9 +381,14 @@ cudaError_t dalloc(T **p, size_t count)
     return cudaMalloc(reinterpret_cast<void **>(p), count * sizeof(T) + 256);
 }
 
+// Tile width of a step GEMM: the widest that divides N.  A 128 x 256 tile
+// needs 96 B of operands per clock of MMA against 128 B for 128 x 128, and
+// the operand stream from L2 into each SM is what bounds these GEMMs: at 4096
+// rows, width 1024 runs 9.1 us at 256 against 12.7 us at 128 (K = 1024) and
+// 22.8 against 38.4 us (K = 4096), CUDA-graph timed.
 int pick_bn(int N)
 {
-    if (N % 256 == 0 && N >= 2048) return 256;
+    if (N % 256 == 0) return 256;
     if (N % 128 == 0) return 128;
     return 64;
 }
@@ -413,8 +418,12 @@ cudaError_t run_gemm(f3dc_handle *h, const CUtensorMap &ta, const CUtensorMap &t
     p.counters = h->gemm_cnt;
     p.ws_units = h->num_sms;
     p.err = h->dev_err;
-    int tiles = h->max_tiles * (N / bn);
-    int grid = tiles < h->num_sms ? tiles : h->num_sms;
+    // 256-wide tiles that would leave more than half of the SMs idle (few
+    // active rows) run 128 wide: at 1229 rows, width 1024 takes 7.7 us at 128
+    // against 8.6 us at 256 (K = 1024), width 3072 at 640 rows 7.9 against 8.5
+    p.narrow_below = bn == 256 ? h->num_sms / 2 : 0;
+    const int tiles = h->max_tiles * (N / (bn == 256 ? 128 : bn));
+    const int grid = tiles < h->num_sms ? tiles : h->num_sms;
     return launch_gemm(&ta, &tb, p, epi, bn, grid, s);
 }
 
@@ -569,13 +578,13 @@ bool build_maps(f3dc_handle *h)
     h->tm_kv_cross.resize(L);
     for (int l = 0; l < L; ++l) {
         const BlockOffsets &b = h->lay.blk[l];
-        ok = ok && make_tmap_bf16(&h->tm_qkv_w[l], h->wt(b.qkv_w), 3 * W, W, W, h->bn_qkv, 64);
-        ok = ok && make_tmap_bf16(&h->tm_o_w[l], h->wt(b.o_w), W, W, W, h->bn_w, 64);
-        ok = ok && make_tmap_bf16(&h->tm_cq_w[l], h->wt(b.cq_w), W, W, W, h->bn_w, 64);
-        ok = ok && make_tmap_bf16(&h->tm_co_w[l], h->wt(b.co_w), W, W, W, h->bn_w, 64);
-        ok = ok && make_tmap_bf16(&h->tm_fc1_w[l], h->wt(b.fc1_w), Wm, W, W, h->bn_fc1, 64);
-        ok = ok && make_tmap_bf16(&h->tm_fc2_w[l], h->wt(b.fc2_w), W, Wm, Wm, h->bn_w, 64);
-        ok = ok && make_tmap_bf16(&h->tm_ckv_w[l], h->wt(b.ckv_w), 2 * W, h->Dc, h->Dc, h->bn_ckv, 64);
+        ok = ok && make_tmap_bf16(&h->tm_qkv_w[l], h->wt(b.qkv_w), 3 * W, W, W, gemm_b_box_rows(h->bn_qkv), 64);
+        ok = ok && make_tmap_bf16(&h->tm_o_w[l], h->wt(b.o_w), W, W, W, gemm_b_box_rows(h->bn_w), 64);
+        ok = ok && make_tmap_bf16(&h->tm_cq_w[l], h->wt(b.cq_w), W, W, W, gemm_b_box_rows(h->bn_w), 64);
+        ok = ok && make_tmap_bf16(&h->tm_co_w[l], h->wt(b.co_w), W, W, W, gemm_b_box_rows(h->bn_w), 64);
+        ok = ok && make_tmap_bf16(&h->tm_fc1_w[l], h->wt(b.fc1_w), Wm, W, W, gemm_b_box_rows(h->bn_fc1), 64);
+        ok = ok && make_tmap_bf16(&h->tm_fc2_w[l], h->wt(b.fc2_w), W, Wm, Wm, gemm_b_box_rows(h->bn_w), 64);
+        ok = ok && make_tmap_bf16(&h->tm_ckv_w[l], h->wt(b.ckv_w), 2 * W, h->Dc, h->Dc, gemm_b_box_rows(h->bn_ckv), 64);
         ok = ok && make_tmap_bf16(&h->tm_kv_cross[l], h->ckv + (size_t)l * h->ckv_rows * 2 * W, h->ckv_rows, 2 * W,
                                   2 * W, 128, dh);
     }
@@ -1110,7 +1119,7 @@ f3dc_status f3dc_gemm(const void *A, const void *B, const void *bias, const floa
         return fail(nullptr, F3DC_ERR_INVALID_ARG, "pointers must be 16-byte aligned");
     const int bn = N % 256 == 0 ? 256 : (N % 128 == 0 ? 128 : 64);
     CUtensorMap ta, tb;
-    if (!make_tmap_bf16(&ta, A, M, K, K, 128, 64) || !make_tmap_bf16(&tb, B, N, K, K, bn, 64))
+    if (!make_tmap_bf16(&ta, A, M, K, K, 128, 64) || !make_tmap_bf16(&tb, B, N, K, K, gemm_b_box_rows(bn), 64))
         return fail(nullptr, F3DC_ERR_INVALID_ARG, "cuTensorMapEncodeTiled rejected A or B (alignment?)");
     GemmParams p;
     memset(&p, 0, sizeof(p));

@@ -191,15 +191,16 @@ F3DC_DEV void put_bf16x32(OutStage &o, const float *v)
     }
 }
 
-// Applies the epilogue to this tile's column chunks k0, k0 + kstep, ...
-// (chunks of 64 columns for QKNORM, whose RMSNorm groups span 64, else 32).
-template <int BN, int EPI, typename Src>
-F3DC_DEV void epilogue_tile(const GemmParams &p, const Src &src, OutStage &o, int m0, int n0, int k0 = 0,
+// Applies the epilogue to the column chunks k0, k0 + kstep, ... of a tile
+// bn columns wide (chunks of 64 columns for QKNORM, whose RMSNorm groups
+// span 64, else 32).
+template <int EPI, typename Src>
+F3DC_DEV void epilogue_tile(const GemmParams &p, const Src &src, OutStage &o, int m0, int n0, int bn, int k0 = 0,
                             int kstep = 1)
 {
     if constexpr (EPI == kEpiQKNorm) {
 #pragma unroll 1
-        for (int c0 = 64 * k0; c0 < BN; c0 += 64 * kstep) {
+        for (int c0 = 64 * k0; c0 < bn; c0 += 64 * kstep) {
             float v[64];
             src(c0, v);
             src(c0 + 32, v + 32);
@@ -230,7 +231,7 @@ F3DC_DEV void epilogue_tile(const GemmParams &p, const Src &src, OutStage &o, in
         }
     } else {
 #pragma unroll 1
-        for (int c0 = 32 * k0; c0 < BN; c0 += 32 * kstep) {
+        for (int c0 = 32 * k0; c0 < bn; c0 += 32 * kstep) {
             float v[32];
             src(c0, v);
             const int col = n0 + c0;
@@ -285,6 +286,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
 {
     using Cfg = GemmCfg<BN>;
     constexpr int S = Cfg::kStages;
+    constexpr int kBBox = BN < 128 ? BN : 128;  // rows of one B box (gemm_b_box_rows)
     extern __shared__ uint8_t smem_raw[];
     uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     uint8_t *sa = smem;
@@ -324,7 +326,12 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
     griddep_wait();
     Units U;
     U.m_tiles = p.m_tiles_dev ? *p.m_tiles_dev : p.m_tiles;
-    U.tiles = U.m_tiles * (p.N / BN);
+    // narrow mode: a 256-wide kernel whose tile count would leave too many SMs
+    // idle (the row count is only known here) runs 128-wide tiles instead,
+    // with the same stages (half of each B stage used) and TMEM buffers
+    const bool narrow = BN == 256 && p.ws == nullptr && U.m_tiles * (p.N / BN) < p.narrow_below;
+    const int bn = narrow ? BN / 2 : BN;
+    U.tiles = U.m_tiles * (p.N / bn);
     U.kb_n = p.K / kBK;
     U.splits = gemm_split_count(U.tiles, (int)gridDim.x, U.kb_n, p.ws_units, p.ws != nullptr);
     U.kb_per = (U.kb_n + U.splits - 1) / U.splits;
@@ -340,15 +347,18 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
             bool ok = true;
             for (int t = blockIdx.x; t < total && ok; t += gridDim.x) {
                 int m0, n0, kb0, kb1;
-                U.decode(t, m0, n0, kb0, kb1, BN);
+                U.decode(t, m0, n0, kb0, kb1, bn);
                 for (int kb = kb0; kb < kb1; ++kb) {
                     if (!mbar_wait(&empty[s], ph ^ 1, abort_flag, p.err)) {
                         ok = false;
                         break;
                     }
-                    mbar_arrive_expect_tx(&full[s], kAStage + Cfg::kBStage);
+                    mbar_arrive_expect_tx(&full[s], kAStage + bn * kBK * 2);
                     tma_load_2d(sa + s * kAStage, &tma, kb * kBK, m0, &full[s]);
-                    tma_load_2d(sb + s * Cfg::kBStage, &tmb, kb * kBK, n0, &full[s]);
+                    // B in boxes of kBBox rows, stacked in the stage (the
+                    // 8-row swizzle atoms continue across boxes)
+                    for (int hb = 0; hb < bn; hb += kBBox)
+                        tma_load_2d(sb + s * Cfg::kBStage + hb * (kBK * 2), &tmb, kb * kBK, n0 + hb, &full[s]);
                     if (++s == S) {
                         s = 0;
                         ph ^= 1;
@@ -362,7 +372,9 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
         // current stage's MMAs, so the read overlaps them, and takes the
         // bounded wait only when the test found the stage not yet loaded.
         if (lane == 0) {
-            constexpr uint32_t idesc = make_idesc_bf16(128, BN, 0, 0);
+            constexpr uint32_t idesc_w = make_idesc_bf16(128, BN, 0, 0);
+            constexpr uint32_t idesc_n = make_idesc_bf16(128, BN / 2 < 16 ? 16 : BN / 2, 0, 0);
+            const uint32_t idesc = narrow ? idesc_n : idesc_w;
             // stage-0 descriptors; stage s adds s * stage bytes / 16, a K
             // step of 16 elements inside the 128B swizzle atom adds 2
             const uint64_t a_desc0 = make_sdesc(smem_u32(sa), 16, 1024, kSwizzle128);
@@ -377,7 +389,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
                 if (!mbar_test(&acce[buf], aph ^ 1) && !mbar_wait(&acce[buf], aph ^ 1, abort_flag, p.err)) break;
                 const uint32_t d = tmem + buf * BN;
                 int m0, n0, kb0, kb1;
-                U.decode(t, m0, n0, kb0, kb1, BN);
+                U.decode(t, m0, n0, kb0, kb1, bn);
                 for (int kb = kb0; kb < kb1; ++kb) {
                     if (!ready && !mbar_wait(&full[s], ph, abort_flag, p.err)) {
                         ok = false;
@@ -420,10 +432,10 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
             if (!all) break;
             tc_fence_after();
             int m0, n0, kb0, kb1;
-            U.decode(t, m0, n0, kb0, kb1, BN);
+            U.decode(t, m0, n0, kb0, kb1, bn);
             const TmemSrc tsrc{tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(buf * BN)};
             if (U.splits == 1) {
-                epilogue_tile<BN, EPI>(p, tsrc, o, m0, n0);
+                epilogue_tile<EPI>(p, tsrc, o, m0, n0, bn);
                 tc_fence_before();
                 __syncwarp();
                 if (lane == 0) mbar_arrive(&acce[buf]);
@@ -484,7 +496,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
             if (!*split_flag) break;
             __threadfence();
             const WsSrc<BN> wsrc{p.ws, tile, U.tiles, U.splits, row};
-            epilogue_tile<BN, EPI>(p, wsrc, o, m0, n0, split, U.splits);
+            epilogue_tile<EPI>(p, wsrc, o, m0, n0, BN, split, U.splits);
             asm volatile("bar.sync 2, 128;" ::: "memory");
             if (threadIdx.x == 64) {
                 // every split has read what it needs: the last one to get here

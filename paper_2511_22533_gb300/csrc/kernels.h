@@ -118,11 +118,16 @@ struct GemmParams {
     float *ws;
     int32_t *counters;
     int ws_units;             // partial tiles the workspace holds
+    // bn = 256 without a workspace: when the device-side tile count of
+    // 256-wide tiles is below this, the kernel runs 128-wide tiles (0: never)
+    int narrow_below;
     uint32_t *err;
 };
-// bn in {64, 128, 256}
+// bn in {64, 128, 256}.  ta: A [M, K] in boxes of 128 rows x 64 columns; tb:
+// B [N, K] in boxes of gemm_b_box_rows(bn) rows x 64 columns.
 cudaError_t launch_gemm(const CUtensorMap *ta, const CUtensorMap *tb, const GemmParams &p, int epi, int bn,
                         int grid, cudaStream_t s);
+inline uint32_t gemm_b_box_rows(int bn) { return bn < 128 ? (uint32_t)bn : 128u; }
 size_t gemm_smem_bytes(int bn);
 
 // Launches a kernel of this library with programmatic stream serialization

@@ -85,7 +85,7 @@ extern "C" f3dc_status f3dc_gemm_noalloc(const void *A, const void *B, const voi
     }
 
     CUtensorMap ta, tb;
-    if (!make_tmap_bf16(&ta, A, M, K, K, 128, 64) || !make_tmap_bf16(&tb, B, N, K, K, bn, 64))
+    if (!make_tmap_bf16(&ta, A, M, K, K, 128, 64) || !make_tmap_bf16(&tb, B, N, K, K, gemm_b_box_rows(bn), 64))
         return fail(F3DC_ERR_INVALID_ARG, "cuTensorMapEncodeTiled rejected A or B (alignment?)");
     GemmParams p;
     memset(&p, 0, sizeof(p));
