@@ -381,6 +381,9 @@ cudaError_t dalloc(T **p, size_t count)
     return cudaMalloc(reinterpret_cast<void **>(p), count * sizeof(T) + 256);
 }
 
+// B-operand box rows of a step weight: 256-wide GEMMs run on CTA pairs.
+uint32_t wide_b_box(int bn) { return bn == 256 ? kGemmPairBBox : gemm_b_box_rows(bn); }
+
 // Tile width of a step GEMM: the widest that divides N.  A 128 x 256 tile
 // needs 96 B of operands per clock of MMA against 128 B for 128 x 128, and
 // the operand stream from L2 into each SM is what bounds these GEMMs: at 4096
@@ -418,11 +421,13 @@ cudaError_t run_gemm(f3dc_handle *h, const CUtensorMap &ta, const CUtensorMap &t
     p.counters = h->gemm_cnt;
     p.ws_units = h->num_sms;
     p.err = h->dev_err;
-    // 256-wide tiles that would leave more than half of the SMs idle (few
-    // active rows) run 128 wide: at 1229 rows, width 1024 takes 7.7 us at 128
-    // against 8.6 us at 256 (K = 1024), width 3072 at 640 rows 7.9 against 8.5
-    p.narrow_below = bn == 256 ? h->num_sms / 2 : 0;
-    const int tiles = h->max_tiles * (N / (bn == 256 ? 128 : bn));
+    // 256-wide tiles run on CTA pairs; those that would leave more than half
+    // of the SMs idle (few active rows) run 128 wide
+    if (bn == 256) {
+        p.narrow_below = h->num_sms / 2;
+        return launch_gemm_pair(&ta, &tb, p, epi, (h->max_tiles + 1) / 2 * (N / 128), s);
+    }
+    const int tiles = h->max_tiles * (N / bn);
     const int grid = tiles < h->num_sms ? tiles : h->num_sms;
     return launch_gemm(&ta, &tb, p, epi, bn, grid, s);
 }
@@ -578,13 +583,14 @@ bool build_maps(f3dc_handle *h)
     h->tm_kv_cross.resize(L);
     for (int l = 0; l < L; ++l) {
         const BlockOffsets &b = h->lay.blk[l];
-        ok = ok && make_tmap_bf16(&h->tm_qkv_w[l], h->wt(b.qkv_w), 3 * W, W, W, gemm_b_box_rows(h->bn_qkv), 64);
-        ok = ok && make_tmap_bf16(&h->tm_o_w[l], h->wt(b.o_w), W, W, W, gemm_b_box_rows(h->bn_w), 64);
-        ok = ok && make_tmap_bf16(&h->tm_cq_w[l], h->wt(b.cq_w), W, W, W, gemm_b_box_rows(h->bn_w), 64);
-        ok = ok && make_tmap_bf16(&h->tm_co_w[l], h->wt(b.co_w), W, W, W, gemm_b_box_rows(h->bn_w), 64);
-        ok = ok && make_tmap_bf16(&h->tm_fc1_w[l], h->wt(b.fc1_w), Wm, W, W, gemm_b_box_rows(h->bn_fc1), 64);
-        ok = ok && make_tmap_bf16(&h->tm_fc2_w[l], h->wt(b.fc2_w), W, Wm, Wm, gemm_b_box_rows(h->bn_w), 64);
-        ok = ok && make_tmap_bf16(&h->tm_ckv_w[l], h->wt(b.ckv_w), 2 * W, h->Dc, h->Dc, gemm_b_box_rows(h->bn_ckv), 64);
+        ok = ok && make_tmap_bf16(&h->tm_qkv_w[l], h->wt(b.qkv_w), 3 * W, W, W, wide_b_box(h->bn_qkv), 64);
+        ok = ok && make_tmap_bf16(&h->tm_o_w[l], h->wt(b.o_w), W, W, W, wide_b_box(h->bn_w), 64);
+        ok = ok && make_tmap_bf16(&h->tm_cq_w[l], h->wt(b.cq_w), W, W, W, wide_b_box(h->bn_w), 64);
+        ok = ok && make_tmap_bf16(&h->tm_co_w[l], h->wt(b.co_w), W, W, W, wide_b_box(h->bn_w), 64);
+        ok = ok && make_tmap_bf16(&h->tm_fc1_w[l], h->wt(b.fc1_w), Wm, W, W, wide_b_box(h->bn_fc1), 64);
+        ok = ok && make_tmap_bf16(&h->tm_fc2_w[l], h->wt(b.fc2_w), W, Wm, Wm, wide_b_box(h->bn_w), 64);
+        ok = ok && make_tmap_bf16(&h->tm_ckv_w[l], h->wt(b.ckv_w), 2 * W, h->Dc, h->Dc,
+                                  h->Dc % 128 == 0 ? wide_b_box(h->bn_ckv) : gemm_b_box_rows(h->bn_ckv), 64);
         ok = ok && make_tmap_bf16(&h->tm_kv_cross[l], h->ckv + (size_t)l * h->ckv_rows * 2 * W, h->ckv_rows, 2 * W,
                                   2 * W, 128, dh);
     }
@@ -884,9 +890,15 @@ f3dc_status f3dc_set_cond(f3dc_handle *h, const void *cond, int32_t B, void *str
         p.bias = h->wt(h->lay.blk[l].ckv_b);
         p.err = h->dev_err;
         const int tiles = p.m_tiles * (p.N / h->bn_ckv);
-        LAUNCH(KF_GEMM_COND, wfix(2.0 * rows * p.N * (double)p.K, true),
-               launch_gemm(&h->tm_cond, &h->tm_ckv_w[l], p, kEpiBias, h->bn_ckv,
-                           tiles < h->num_sms ? tiles : h->num_sms, s));
+        if (h->bn_ckv == 256 && h->Dc % 128 == 0) {
+            p.narrow_below = h->num_sms / 2;
+            LAUNCH(KF_GEMM_COND, wfix(2.0 * rows * p.N * (double)p.K, true),
+                   launch_gemm_pair(&h->tm_cond, &h->tm_ckv_w[l], p, kEpiBias, (p.m_tiles + 1) / 2 * (p.N / 128), s));
+        } else {
+            LAUNCH(KF_GEMM_COND, wfix(2.0 * rows * p.N * (double)p.K, true),
+                   launch_gemm(&h->tm_cond, &h->tm_ckv_w[l], p, kEpiBias, h->bn_ckv,
+                               tiles < h->num_sms ? tiles : h->num_sms, s));
+        }
     }
     h->cond_B = B;
     return F3DC_OK;
@@ -1118,8 +1130,16 @@ f3dc_status f3dc_gemm(const void *A, const void *B, const void *bias, const floa
     if (((uintptr_t)out & 15) || (bias && ((uintptr_t)bias & 15)) || (gate && ((uintptr_t)gate & 15)))
         return fail(nullptr, F3DC_ERR_INVALID_ARG, "pointers must be 16-byte aligned");
     const int bn = N % 256 == 0 ? 256 : (N % 128 == 0 ? 128 : 64);
+    int dev = 0, sms = 0;
+    CK(cudaGetDevice(&dev));
+    CK(cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev));
+    const int m_tiles = (M + kTileRows - 1) / kTileRows;
+    // 256-wide tiles without split K run on CTA pairs
+    const bool pair = bn == 256 && K % 128 == 0 && gemm_split_count(m_tiles * (N / bn), gemm_grid(m_tiles * (N / bn), sms), K / 64,
+                                                    sms, true) == 1;
     CUtensorMap ta, tb;
-    if (!make_tmap_bf16(&ta, A, M, K, K, 128, 64) || !make_tmap_bf16(&tb, B, N, K, K, gemm_b_box_rows(bn), 64))
+    if (!make_tmap_bf16(&ta, A, M, K, K, 128, 64) ||
+        !make_tmap_bf16(&tb, B, N, K, K, pair ? kGemmPairBBox : gemm_b_box_rows(bn), 64))
         return fail(nullptr, F3DC_ERR_INVALID_ARG, "cuTensorMapEncodeTiled rejected A or B (alignment?)");
     GemmParams p;
     memset(&p, 0, sizeof(p));
@@ -1131,12 +1151,14 @@ f3dc_status f3dc_gemm(const void *A, const void *B, const void *bias, const floa
     p.ldo = N;
     p.bias = reinterpret_cast<const bf16 *>(bias);
     p.gate = gate;
-    int dev = 0, sms = 0;
-    CK(cudaGetDevice(&dev));
-    CK(cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev));
     const int tiles = p.m_tiles * (N / bn);
     const int epi = epilogue == F3DC_EPI_BIAS ? kEpiBias : (epilogue == F3DC_EPI_GELU ? kEpiGelu : kEpiResid);
     cudaStream_t s = (cudaStream_t)stream;
+    if (pair) {
+        p.narrow_below = sms / 2;
+        CK(launch_gemm_pair(&ta, &tb, p, epi, (m_tiles + 1) / 2 * (N / 128), s));
+        return F3DC_OK;
+    }
     // split-K workspace: allocated once per device on first use and kept for
     // the life of the process (its counters return to 0 after every launch)
     static std::mutex ws_lock;

@@ -141,38 +141,48 @@ struct WsSrc {
     }
 };
 
-// Output staging shared by the epilogue warps: a chunk is one 128-row box of
-// 64-byte rows, 16-byte piece c of row r at 64 r + 16 (c ^ ((r / 2) % 4))
-// (the TMA 64B swizzle), which spreads a warp's row-per-lane stores over all
-// banks.  The box is written by thread 64 with a TMA store; before a buffer
-// is reused three chunks later its store has finished reading it.
+// Output staging shared by a group of four epilogue warps: a chunk is one
+// 128-row box of 64-byte rows, 16-byte piece c of row r at 64 r + 16 (c ^
+// ((r / 2) % 4)) (the TMA 64B swizzle), which spreads a warp's row-per-lane
+// stores over all banks.  The box is written out by the group's issuer thread
+// with a TMA store; before a buffer is reused nbufs chunks later its store
+// has finished reading it.
 struct OutStage {
-    uint8_t *buf;             // kOutBufs x kOutChunkBytes
+    uint8_t *buf;             // nbufs x kOutChunkBytes
     const CUtensorMap *map;   // output tensor: bf16 [M, N] or fp32 [M, N] (RESID, reduce-add)
     int row;                  // this thread's row of the tile
-    int ck;                   // chunks emitted so far by this CTA
-    F3DC_DEV uint8_t *slot() const { return buf + (ck % kOutBufs) * kOutChunkBytes; }
+    int ck;                   // chunks emitted so far by this group of four warps
+    int nbufs = kOutBufs;     // staging buffers (>= 2)
+    int bar = 3;              // named barrier of the four warps
+    int issuer = 64;          // thread that issues the group's TMA stores
+    F3DC_DEV uint8_t *slot() const { return buf + (ck % nbufs) * kOutChunkBytes; }
     F3DC_DEV void put16(int c, uint4 u) const
     {
         *reinterpret_cast<uint4 *>(slot() + row * 64 + ((c ^ ((row >> 1) & 3)) << 4)) = u;
     }
     // publish the chunk just written and send it to (x, y) of the output
-    // (or of the tensor `to`, e.g. the split-K workspace)
+    // (or of the tensor `to`, e.g. the split-K workspace).  After the
+    // barrier the warps write the next chunk into the buffer of chunk
+    // ck + 1 - nbufs, so the issuer first waits until that chunk's store has
+    // read it (at most nbufs - 2 stores still reading).
     template <bool kReduce>
     F3DC_DEV void emit(int x, int y, const CUtensorMap *to = nullptr)
     {
         fence_proxy_async_smem();
-        asm volatile("bar.sync 3, 128;" ::: "memory");
-        if (threadIdx.x == 64) {
+        if ((int)threadIdx.x == issuer) {
+            if (nbufs == 2)
+                bulk_wait_read<0>();
+            else
+                bulk_wait_read<1>();
+        }
+        asm volatile("bar.sync %0, 128;" ::"r"(bar) : "memory");
+        if ((int)threadIdx.x == issuer) {
             const CUtensorMap *m = to ? to : map;
             if (kReduce)
                 tma_reduce_add_2d(m, slot(), x, y);
             else
                 tma_store_2d(m, slot(), x, y);
             bulk_commit();
-            // the chunk before this one has been read: its buffer, and every
-            // older one, may be rewritten after the next barrier
-            bulk_wait_read<1>();
         }
         ++ck;
     }
@@ -523,6 +533,256 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
     }
 }
 
+// ------------------------------------------------------------ CTA pair
+// cta_group::2 GEMM for 256-wide tiles.  A cluster of two CTAs computes a
+// 256 x 256 tile (256 x 128 in narrow mode): each CTA loads its 128 rows of A
+// and its half of the tile's B rows into its own shared memory (128 K per stage), the even CTA
+// issues the 256-row MMAs for both, and each CTA's TMEM receives its own 128
+// rows of the accumulator, which its epilogue warps write out.  Per SM that
+// is 32 KB of operands per 512 MMA clocks instead of the 48 KB a 128 x 256
+// tile of one CTA needs, so the operand stream from L2 keeps up with the
+// tensor core.
+//   full[s]  (even CTA): both CTAs' TMA bytes of stage s (the even CTA's
+//            producer posts the expected count)
+//   empty[s] (both):     stage s consumed (multicast MMA commit)
+//   accf[b]  (both):     accumulator buffer b complete (multicast commit)
+//   acce[b]  (even CTA): buffer b read by the epilogue warps of both CTAs
+// A stage holds 128 K: two 64-column boxes per operand row block, each a
+// 128B-swizzled K-major region of its own ([half][rows][128 B]).
+constexpr int kPairBK = 128;
+constexpr int kPairHalf = 128 * 128;                // one 64-K box of 128 rows (16 KB)
+constexpr int kPairAStage = 2 * kPairHalf;          // this CTA's 128 A rows x 128 K
+constexpr int kPairBStage = 2 * kPairHalf;          // this CTA's (up to) 128 B rows x 128 K
+constexpr int kPairStages = 3;
+constexpr uint32_t kPairTmemCols = 512;             // two buffers of 256 columns
+// eight epilogue warps in two groups of four (one warp per TMEM lane quarter
+// in each), group g writing the tile's column chunks g, g + 2, ..., each
+// group through two staging buffers of its own
+constexpr int kPairThreads = 320;
+constexpr int kPairOutBufs = 2;
+constexpr size_t kPairSmem = 1024 + (size_t)kPairStages * (kPairAStage + kPairBStage) +
+                             2 * (size_t)kPairOutBufs * kOutChunkBytes + 256;
+
+template <int EPI>
+__global__ void __launch_bounds__(kPairThreads, 1)
+    k_gemm_pair(const __grid_constant__ CUtensorMap tma, const __grid_constant__ CUtensorMap tmb,
+                const __grid_constant__ CUtensorMap tmo, const GemmParams p)
+{
+    constexpr int S = kPairStages;
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+    uint8_t *sa = smem;
+    uint8_t *sb = smem + S * kPairAStage;
+    uint8_t *so = sb + S * kPairBStage;
+    uint64_t *bars = reinterpret_cast<uint64_t *>(so + 2 * kPairOutBufs * kOutChunkBytes);
+    uint64_t *full = bars, *empty = bars + S, *accf = bars + 2 * S, *acce = accf + 2, *drain = acce + 2;
+    uint32_t *tmem_holder = reinterpret_cast<uint32_t *>(drain + 1);
+    volatile int *abort_flag = reinterpret_cast<volatile int *>(tmem_holder + 1);
+
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const uint32_t rank = cluster_rank();
+    griddep_launch();
+
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < S; ++s) {
+            mbar_init(&full[s], 1);
+            mbar_init(&empty[s], 1);
+        }
+        mbar_init(&accf[0], 1);
+        mbar_init(&accf[1], 1);
+        mbar_init(&acce[0], 16);  // eight epilogue warps in each CTA
+        mbar_init(&acce[1], 16);
+        mbar_init(drain, 1);
+        *abort_flag = 0;
+        fence_mbar_init();
+    }
+    if (warp == 1) {
+        tmem_alloc_pair(tmem_holder, kPairTmemCols);
+        tmem_relinquish_pair();
+    }
+    tc_fence_before();
+    __syncthreads();
+    cluster_sync();  // both CTAs' barriers are initialised before any remote signal
+    tc_fence_after();
+    const uint32_t tmem = *tmem_holder;
+    griddep_wait();
+    const int m_tiles = p.m_tiles_dev ? *p.m_tiles_dev : p.m_tiles;
+    const bool narrow = m_tiles * (p.N / 256) < p.narrow_below;
+    const int bn = narrow ? 128 : 256;  // tile width; this CTA holds bn / 2 B rows
+    const int pm_tiles = (m_tiles + 1) / 2;
+    const int tiles = pm_tiles * (p.N / bn);
+    const int kb_n = p.K / kPairBK;
+    const int cl = blockIdx.x >> 1, ncl = gridDim.x >> 1;
+    const uint32_t full_c = mapa_shared(smem_u32(full), 0);  // the even CTA's full[0]
+    const uint32_t acce_c = mapa_shared(smem_u32(acce), 0);
+
+    if (warp == 0) {
+        if (lane == 0) {
+            tma_prefetch(&tma);
+            tma_prefetch(&tmb);
+            const uint32_t stage_bytes = 2u * (kPairAStage + (uint32_t)(bn / 2) * kPairBK * 2);  // both CTAs
+            int s = 0;
+            uint32_t ph = 0;
+            bool ok = true;
+            for (int t = cl; t < tiles && ok; t += ncl) {
+                const int arow = (t % pm_tiles) * 256 + (int)rank * 128;
+                const int brow = (t / pm_tiles) * bn + (int)rank * (bn / 2);
+                for (int kb = 0; kb < kb_n; ++kb) {
+                    if (!mbar_wait(&empty[s], ph ^ 1, abort_flag, p.err)) {
+                        ok = false;
+                        break;
+                    }
+                    if (rank == 0) mbar_arrive_expect_tx(&full[s], stage_bytes);
+                    const uint32_t fb = full_c + 8u * (uint32_t)s;
+#pragma unroll
+                    for (int h = 0; h < 2; ++h) {
+                        const int x = kb * kPairBK + h * 64;
+                        tma_load_2d_pair(sa + s * kPairAStage + h * kPairHalf, &tma, x, arow, fb);
+                        for (int hb = 0; hb < bn / 2; hb += (int)kGemmPairBBox)
+                            tma_load_2d_pair(sb + s * kPairBStage + h * kPairHalf + hb * 128, &tmb, x, brow + hb, fb);
+                    }
+                    if (++s == S) {
+                        s = 0;
+                        ph ^= 1;
+                    }
+                }
+            }
+        }
+    } else if (warp == 1) {
+        if (lane == 0 && rank == 0) {
+            constexpr uint32_t idesc_w = make_idesc_bf16(256, 256, 0, 0);
+            constexpr uint32_t idesc_n = make_idesc_bf16(256, 128, 0, 0);
+            const uint32_t idesc = narrow ? idesc_n : idesc_w;
+            const uint64_t a_desc0 = make_sdesc(smem_u32(sa), 16, 1024, kSwizzle128);
+            const uint64_t b_desc0 = make_sdesc(smem_u32(sb), 16, 1024, kSwizzle128);
+            int s = 0, it = 0;
+            uint32_t ph = 0;
+            bool ok = true;
+            bool ready = mbar_test(&full[0], 0);
+            for (int t = cl; t < tiles && ok; t += ncl, ++it) {
+                const int buf = it & 1;
+                const uint32_t aph = (it >> 1) & 1;
+                if (!mbar_test(&acce[buf], aph ^ 1) && !mbar_wait(&acce[buf], aph ^ 1, abort_flag, p.err)) break;
+                const uint32_t d = tmem + buf * 256;
+                for (int kb = 0; kb < kb_n; ++kb) {
+                    if (!ready && !mbar_wait(&full[s], ph, abort_flag, p.err)) {
+                        ok = false;
+                        break;
+                    }
+                    tc_fence_after();
+                    const int s_next = s + 1 == S ? 0 : s + 1;
+                    const uint32_t ph_next = s_next == 0 ? ph ^ 1 : ph;
+                    ready = mbar_test(&full[s_next], ph_next);
+                    const uint64_t ad = a_desc0 + (uint64_t)s * (kPairAStage >> 4);
+                    const uint64_t bd = b_desc0 + (uint64_t)s * (kPairBStage >> 4);
+#pragma unroll
+                    for (int k = 0; k < kPairBK / 16; ++k) {
+                        const uint64_t off = (uint64_t)(k >> 2) * (kPairHalf >> 4) + 2 * (k & 3);
+                        mma_bf16_pair(d, ad + off, bd + off, idesc, (kb != 0) || (k != 0));
+                    }
+                    mma_commit_pair_mc(&empty[s], 3);
+                    s = s_next;
+                    ph = ph_next;
+                }
+                if (ok) mma_commit_pair_mc(&accf[buf], 3);
+            }
+        }
+    } else {
+        const int q = warp & 3;
+        const int row = q * 32 + lane;
+        const int grp = (warp - 2) >> 2;
+        OutStage o{so + grp * kPairOutBufs * kOutChunkBytes, &tmo, row, 0, kPairOutBufs, 3 + grp, 64 + 128 * grp};
+        int it = 0;
+        for (int t = cl; t < tiles; t += ncl, ++it) {
+            const int buf = it & 1;
+            const uint32_t aph = (it >> 1) & 1;
+            const uint32_t got = mbar_wait(&accf[buf], aph, abort_flag, p.err) ? 1u : 0u;
+            uint32_t all;
+            asm volatile("{\n .reg .pred p, q;\n setp.ne.u32 p, %1, 0;\n bar.red.and.pred q, %2, 128, p;\n"
+                         " selp.u32 %0, 1, 0, q;\n}\n"
+                         : "=r"(all)
+                         : "r"(got), "r"(o.bar)
+                         : "memory");
+            if (!all) break;
+            tc_fence_after();
+            const int m0 = (t % pm_tiles) * 256 + (int)rank * 128;
+            const int n0 = (t / pm_tiles) * bn;
+            // the odd CTA's rows of the last pair lie beyond the plan when
+            // the tile count is odd: computed, not stored
+            if (m0 < m_tiles * 128) {
+                const TmemSrc tsrc{tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(buf * 256)};
+                epilogue_tile<EPI>(p, tsrc, o, m0, n0, bn, grp, 2);
+            }
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive_cluster(acce_c + 8u * (uint32_t)buf);
+        }
+        if ((int)threadIdx.x == o.issuer) bulk_wait_all();
+    }
+    __syncthreads();
+    if (*abort_flag) {
+        if (warp == 1 && lane == 0 && rank == 0) {
+            mma_commit_pair(drain);
+            mbar_wait_bounded(drain, 0, 100000000ull);
+        }
+        if (threadIdx.x == 0) spin_ns(200000);
+        __syncthreads();
+    }
+    // neither CTA leaves while the other may still signal its barriers or
+    // (the even CTA's MMAs) write its TMEM
+    cluster_sync();
+    if (warp == 1) {
+        tc_fence_after();
+        tmem_dealloc_pair(tmem, kPairTmemCols);
+    }
+}
+
+template <int EPI>
+cudaError_t launch_pair_one(const CUtensorMap *ta, const CUtensorMap *tb, const CUtensorMap *to, const GemmParams &p,
+                            int max_pair_tiles, cudaStream_t s)
+{
+    static int max_clusters = 0;
+    if (!max_clusters) {
+        cudaError_t e =
+            cudaFuncSetAttribute(k_gemm_pair<EPI>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kPairSmem);
+        if (e != cudaSuccess) return e;
+        cudaLaunchConfig_t cfg = {};
+        cfg.gridDim = dim3(2);
+        cfg.blockDim = dim3(kPairThreads);
+        cfg.dynamicSmemBytes = kPairSmem;
+        cudaLaunchAttribute at[1];
+        at[0].id = cudaLaunchAttributeClusterDimension;
+        at[0].val.clusterDim.x = 2;
+        at[0].val.clusterDim.y = 1;
+        at[0].val.clusterDim.z = 1;
+        cfg.attrs = at;
+        cfg.numAttrs = 1;
+        int n = 0;
+        e = cudaOccupancyMaxActiveClusters(&n, k_gemm_pair<EPI>, &cfg);
+        if (e != cudaSuccess) return e;
+        if (n < 1) return cudaErrorInvalidConfiguration;
+        max_clusters = n;
+    }
+    const int clusters = max_pair_tiles < max_clusters ? (max_pair_tiles > 0 ? max_pair_tiles : 1) : max_clusters;
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(2 * clusters);
+    cfg.blockDim = dim3(kPairThreads);
+    cfg.dynamicSmemBytes = kPairSmem;
+    cfg.stream = s;
+    cudaLaunchAttribute at[2];
+    at[0].id = cudaLaunchAttributeClusterDimension;
+    at[0].val.clusterDim.x = 2;
+    at[0].val.clusterDim.y = 1;
+    at[0].val.clusterDim.z = 1;
+    at[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    at[1].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = at;
+    cfg.numAttrs = 2;
+    cudaError_t e = cudaLaunchKernelEx(&cfg, k_gemm_pair<EPI>, *ta, *tb, *to, p);
+    if (e != cudaSuccess) return e;
+    return cudaGetLastError();
+}
+
 template <int BN, int EPI>
 cudaError_t launch_one(const CUtensorMap *ta, const CUtensorMap *tb, const CUtensorMap *to, const CUtensorMap *tw,
                        const GemmParams &p, int grid, cudaStream_t s)
@@ -615,6 +875,22 @@ cudaError_t launch_gemm(const CUtensorMap *ta, const CUtensorMap *tb, const Gemm
     case 64: return launch_bn<64>(ta, tb, &to, &tw, p, epi, grid, s);
     case 128: return launch_bn<128>(ta, tb, &to, &tw, p, epi, grid, s);
     case 256: return launch_bn<256>(ta, tb, &to, &tw, p, epi, grid, s);
+    default: return cudaErrorInvalidValue;
+    }
+}
+
+cudaError_t launch_gemm_pair(const CUtensorMap *ta, const CUtensorMap *tb, const GemmParams &p, int epi,
+                             int max_pair_tiles, cudaStream_t s)
+{
+    if (p.K % kPairBK != 0 || p.N % 256 != 0 || p.ws) return cudaErrorInvalidValue;
+    CUtensorMap to;
+    if (!make_tmap_out(&to, p.out, (uint64_t)p.M, (uint64_t)p.N, (uint64_t)p.ldo, epi == kEpiResid))
+        return cudaErrorInvalidValue;
+    switch (epi) {
+    case kEpiBias: return launch_pair_one<kEpiBias>(ta, tb, &to, p, max_pair_tiles, s);
+    case kEpiGelu: return launch_pair_one<kEpiGelu>(ta, tb, &to, p, max_pair_tiles, s);
+    case kEpiResid: return launch_pair_one<kEpiResid>(ta, tb, &to, p, max_pair_tiles, s);
+    case kEpiQKNorm: return launch_pair_one<kEpiQKNorm>(ta, tb, &to, p, max_pair_tiles, s);
     default: return cudaErrorInvalidValue;
     }
 }

@@ -128,6 +128,15 @@ struct GemmParams {
 cudaError_t launch_gemm(const CUtensorMap *ta, const CUtensorMap *tb, const GemmParams &p, int epi, int bn,
                         int grid, cudaStream_t s);
 inline uint32_t gemm_b_box_rows(int bn) { return bn < 128 ? (uint32_t)bn : 128u; }
+
+// 256-wide GEMM on CTA pairs (clusters of two, cta_group::2 MMAs of 256
+// rows): same parameters and epilogues as launch_gemm with bn = 256, K a
+// multiple of 128, no split K (p.ws null); tb in boxes of kGemmPairBBox rows
+// x 64 columns.  The
+// grid is min(max_pair_tiles, resident clusters) clusters.
+constexpr uint32_t kGemmPairBBox = 64;
+cudaError_t launch_gemm_pair(const CUtensorMap *ta, const CUtensorMap *tb, const GemmParams &p, int epi,
+                             int max_pair_tiles, cudaStream_t s);
 size_t gemm_smem_bytes(int bn);
 
 // Launches a kernel of this library with programmatic stream serialization
