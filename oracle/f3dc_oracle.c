@@ -17,6 +17,8 @@
  *                                                LayerNorm, cross-attention, MLP)
  *   - cache merge and rectified-flow Euler step (Algorithm 1 step 3; Sec. 3.1)
  *   - dynamic-voxel count                       (Sec. 4.1 Eq. 1)
+ *   - classifier-free guidance in its interval  (Sec. 4.3 Phase 3 "CFG-free";
+ *                                                Supp. Sec. D CFG interval t in [0.5, 1])
  *   - the whole sampler                         (Algorithm 1)
  *
  * Precision: the SSC score, the selection order, the Euler update and the
@@ -270,6 +272,33 @@ void orc_merge_euler(int N, int C, const int32_t *active_idx, int a, const float
     for (long long q = 0; q < (long long)N * C; ++q) {
         float step = dt * bf2f(v_t[q]);
         S[q] = S[q] - step;
+    }
+}
+
+/* ------------------------------------------------------------------------ */
+/* Classifier-free guidance.  The sampler guides the steps whose start time */
+/* lies in the CFG interval [t_lo, 1] (Supp. Sec. D: TRELLIS's flow         */
+/* sampler applies CFG for t in [0.5, 1]; Phase 3 is the CFG-free stage).   */
+/* The guided velocity moves from the unconditional prediction towards the  */
+/* conditional one by the strength s: v = v_u + s (v_c - v_u), in fp32:     */
+/* one subtraction, one multiplication by (float)s, one addition.           */
+/* ------------------------------------------------------------------------ */
+int orc_cfg_on(int T, double eta, double t_lo, int k)
+{
+    float *t = (float *)malloc(sizeof(float) * (size_t)(T + 1));
+    orc_time_schedule(T, eta, t);
+    const int on = (double)t[k - 1] >= t_lo;
+    free(t);
+    return on;
+}
+
+void orc_cfg_combine(long long n, const float *v_c, const float *v_u, double s, float *v)
+{
+    const float sf = (float)s;
+    for (long long q = 0; q < n; ++q) {
+        const float d = v_c[q] - v_u[q];
+        const float g = sf * d;
+        v[q] = v_u[q] + g;
     }
 }
 
@@ -647,12 +676,15 @@ void orc_dit_forward(const void *vm, const float *S, const int32_t *active_idx, 
  *   [T, B] active tokens, sigma_out [B] measured dynamic voxels at the
  *   anchor step (Eq. 1 between the grids before and after step k_a).
  * v_hist_out: nullable [2, B, N, C] bf16 -- (v_cache, v_prev_cache) at exit.
+ * cfg_on: guide the steps k with t_k >= cfg_t_lo with strength cfg_s; the
+ *   unconditional prediction sees the all-zero condition (reading: the paper
+ *   names no null condition) and the same active tokens.
  */
 int orc_sample(const void *vm, int T, double eta, double rho_a, double rho_off, double mu,
                double omega, double xi, int f_corr, int tau, int refresh_mode,
                float *S, const uint16_t *cond, int B, const double *sigma_override,
                const int32_t *quota_schedule, int32_t *quota_log, int32_t *nact_log,
-               double *sigma_out, uint16_t *v_hist_out)
+               double *sigma_out, uint16_t *v_hist_out, int cfg_on, double cfg_s, double cfg_t_lo)
 {
     const orc_model *m = (const orc_model *)vm;
     const int N = m->grid * m->grid * m->grid, C = m->C, G = m->G;
@@ -672,6 +704,15 @@ int orc_sample(const void *vm, int T, double eta, double rho_a, double rho_off, 
     float *Sold = (float *)malloc(sizeof(float) * NC);
     uint8_t *occ_a = (uint8_t *)malloc((size_t)N * G);
     uint8_t *occ_b = (uint8_t *)malloc((size_t)N * G);
+    float *kv_null = NULL, *va_c = NULL, *va_u = NULL;
+    if (cfg_on) {
+        uint16_t *zero = (uint16_t *)calloc((size_t)m->Nc * m->Dc, sizeof(uint16_t));
+        kv_null = (float *)malloc(sizeof(float) * (size_t)m->L * 2 * m->Nc * m->W);
+        orc_cond_kv(m, zero, kv_null);
+        free(zero);
+        va_c = (float *)malloc(sizeof(float) * NC);
+        va_u = (float *)malloc(sizeof(float) * NC);
+    }
 
     for (int b = 0; b < B; ++b) {
         float *Sb = S + (size_t)b * NC;
@@ -698,7 +739,15 @@ int orc_sample(const void *vm, int T, double eta, double rho_a, double rho_off, 
             }
             if (quota_log) quota_log[(size_t)(k - 1) * B + b] = c;
             if (nact_log) nact_log[(size_t)(k - 1) * B + b] = a;
-            if (a > 0) orc_dit_forward(m, Sb, idx, a, t[k - 1], kv, va);
+            if (a > 0) {
+                if (cfg_on && (double)t[k - 1] >= cfg_t_lo) {
+                    orc_dit_forward(m, Sb, idx, a, t[k - 1], kv, va_c);
+                    orc_dit_forward(m, Sb, idx, a, t[k - 1], kv_null, va_u);
+                    orc_cfg_combine((long long)a * C, va_c, va_u, cfg_s, va);
+                } else {
+                    orc_dit_forward(m, Sb, idx, a, t[k - 1], kv, va);
+                }
+            }
             if (k == ka) memcpy(Sold, Sb, sizeof(float) * NC);
             float dt = t[k - 1] - t[k];
             orc_merge_euler(N, C, idx, a, va, vc, dt, Sb, vt);
@@ -721,6 +770,6 @@ int orc_sample(const void *vm, int T, double eta, double rho_a, double rho_off, 
         }
     }
     free(t); free(kv); free(vc); free(vp); free(vt); free(score); free(cached); free(idx);
-    free(va); free(Sold); free(occ_a); free(occ_b);
+    free(va); free(Sold); free(occ_a); free(occ_b); free(kv_null); free(va_c); free(va_u);
     return 0;
 }

@@ -76,7 +76,10 @@ def lib():
             L.orc_dit_forward.argtypes = [C.c_void_p, _f32p, _i32p, C.c_int, C.c_float, _f32p, _f32p]
             L.orc_sample.argtypes = [C.c_void_p, C.c_int, C.c_double, C.c_double, C.c_double,
                                      C.c_double, C.c_double, C.c_double, C.c_int, C.c_int, C.c_int,
-                                     _f32p, _u16p, C.c_int, _f64p, _i32p, _i32p, _i32p, _f64p, _u16p]
+                                     _f32p, _u16p, C.c_int, _f64p, _i32p, _i32p, _i32p, _f64p, _u16p,
+                                     C.c_int, C.c_double, C.c_double]
+            L.orc_cfg_on.argtypes = [C.c_int, C.c_double, C.c_double, C.c_int]
+            L.orc_cfg_combine.argtypes = [C.c_longlong, _f32p, _f32p, C.c_double, _f32p]
             L.orc_f32_to_bf16.argtypes = [C.c_float]
             L.orc_f32_to_bf16.restype = C.c_uint16
             _lib = L
@@ -199,6 +202,19 @@ def dynamic_voxels(occ_a: np.ndarray, occ_b: np.ndarray) -> int:
     return int(lib().orc_dynamic_voxels(_p(a, _u8p), _p(b, _u8p), a.size))
 
 
+def cfg_on(T: int, eta: float, t_lo: float, k: int) -> bool:
+    """Whether step k (1-based) is guided: t_k in the CFG interval [t_lo, 1]."""
+    return bool(lib().orc_cfg_on(T, eta, t_lo, k))
+
+
+def cfg_combine(v_c, v_u, s: float) -> np.ndarray:
+    """Guided velocity v_u + s (v_c - v_u) in fp32 (subtract, multiply, add)."""
+    vc, vu = _f32(v_c), _f32(v_u)
+    out = np.empty_like(vc)
+    lib().orc_cfg_combine(vc.size, _p(vc, _f32p), _p(vu, _f32p), s, _p(out, _f32p))
+    return out
+
+
 def merge_euler(S, active_idx, v_active, v_cache_bits, dt: float):
     """Returns (S_new, v_t_bits); inputs are not modified."""
     S = _f32(S).copy()
@@ -268,8 +284,9 @@ class Model:
 
     def sample(self, S: np.ndarray, cond_bits: np.ndarray, *, T, eta=3.0, rho_a=0.2, rho_off=0.75,
                mu=-0.07, omega=0.7, xi=0.7, f_corr=3, tau=3, refresh_mode=0,
-               sigma_override=None, quota_schedule=None):
-        """Algorithm 1 for B samples.  Returns dict(S, quota, n_active, sigma, v_hist)."""
+               sigma_override=None, quota_schedule=None, cfg=None, cfg_t_lo=0.5):
+        """Algorithm 1 for B samples.  Returns dict(S, quota, n_active, sigma, v_hist).
+        cfg: guidance strength s (None: unguided) for the steps with t_k >= cfg_t_lo."""
         S = _f32(S).copy()
         B = S.shape[0]
         N = self.shape.tokens
@@ -284,5 +301,6 @@ class Model:
                          _p(S, _f32p), _p(cb, _u16p), B,
                          _p(sov, _f64p) if sov is not None else None,
                          _p(qs, _i32p) if qs is not None else None,
-                         _p(ql, _i32p), _p(nl, _i32p), _p(so, _f64p), _p(vh, _u16p))
+                         _p(ql, _i32p), _p(nl, _i32p), _p(so, _f64p), _p(vh, _u16p),
+                         0 if cfg is None else 1, 0.0 if cfg is None else float(cfg), float(cfg_t_lo))
         return dict(S=S, quota=ql, n_active=nl, sigma=so, v_hist=vh)
