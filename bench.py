@@ -42,6 +42,7 @@ from paper_2511_22533_gb300 import synth  # noqa: E402
 METRIC = "cached denoise steps/s at PCSC quota (1 GB300); tensor-pipe % of bf16 peak"
 UNIT = "steps/s"
 WORKLOAD = "trellis_l"
+CFG_STRENGTH = 5.0  # guidance strength of the secondary CFG measurement (the work does not depend on it)
 SIGMA = 65536.0
 FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
 
@@ -84,14 +85,17 @@ def paper_block_flops(a: int, W: int, Nc: int, H: int, B: int = 1) -> float:
     return mod + 3 * ln + sa + ca + mlp
 
 
-def sample_flops(quota_log, shape):
+def sample_flops(quota_log, shape, guided=None):
+    """Tensor-core and paper FLOPs of one sample; guided[k] marks the steps
+    that run the transformer twice (classifier-free guidance)."""
     N, W, L, Nc, H = shape.tokens, shape.width, shape.blocks, shape.cond_tokens, shape.heads
     mm = paper = 0.0
-    for c in quota_log[:, 0]:
+    for k, c in enumerate(quota_log[:, 0]):
         a = N - int(c)
+        reps = 2 if guided is not None and guided[k] else 1
         if a > 0:
-            mm += L * block_matmul_flops(a, W, Nc)
-            paper += L * paper_block_flops(a, W, Nc, H)
+            mm += reps * L * block_matmul_flops(a, W, Nc)
+            paper += reps * L * paper_block_flops(a, W, Nc, H)
     mm += L * 2.0 * Nc * (2 * W) * shape.cond_dim  # condition K / V, once per sample
     return mm, paper
 
@@ -447,6 +451,30 @@ def run_gpu(args):
     e2e_value = whole_job_throughput(shape.steps, args.steps, world, ms_e2e)
     assert h.device_status() == 0
 
+    # ---- classifier-free guidance over the interval [0.5, 1] (secondary; not
+    # part of `value`): the same workload with every step whose t_k >= 0.5 run
+    # for the condition and the zero condition on the same active tokens
+    cfg_g = f3dc.config_for(shape, 1, cfg_strength=CFG_STRENGTH, cfg_t_lo=0.5)
+    hg = f3dc.Handle(cfg_g, blob_d)
+
+    def guided_sample():
+        S.copy_(noise_d)
+        hg.sample(S, cond_d, 1, sigma_override=sig, want_log=False)
+
+    for _ in range(max(args.warmup, 1)):
+        guided_sample()
+    n_g = max(2, args.steps // 2)
+    ms_g = timed(n_g, guided_sample) / n_g
+    assert hg.device_status() == 0
+    hg.close()
+    t_sched = f3dc.time_schedule(cfg_g)
+    guided = [float(t_sched[k]) >= 0.5 for k in range(shape.steps)]
+    mm_g, paper_g = sample_flops(qlog, shape, guided)
+    cfg_line = {"strength": CFG_STRENGTH, "interval": [0.5, 1.0], "guided_steps": int(sum(guided)),
+                "ms_per_sample": ms_g, "steps_per_s": shape.steps * world / (ms_g / 1000.0),
+                "tensor_tflops_per_gpu": mm_g / (ms_g / 1000.0) / 1e12,
+                "paper_flops_per_sample_T": paper_g / 1e12}
+
     # ---- the HBM-bound kernels at batch 64 (secondary; not part of `value`)
     hbm64 = hbm_kernels_b64(f3dc, torch, blob_d, pk) if rank == 0 else None
     del blob_d
@@ -505,7 +533,7 @@ def run_gpu(args):
                      "tensor_tflops_per_gpu": mm_unc / (ms_unc / 1000.0) / 1e12},
         "active_tokens_per_step": [shape.tokens - int(c) for c in qlog[:, 0]],
         "sigma_measured_by_stand_in_decoder": float(sigma_meas[0]),
-        "roofline": roof, "kernels": kernels, "hbm_kernels_b64": hbm64,
+        "roofline": roof, "kernels": kernels, "hbm_kernels_b64": hbm64, "cfg": cfg_line,
         "cpu_baseline": cpu,
         "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": int(noise.nbytes + cond_np.nbytes),
                 "d2h_bytes_per_step": int(noise.nbytes)},

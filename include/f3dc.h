@@ -90,6 +90,12 @@ typedef struct f3dc_config {
     double omega;        /* SSC weight of the acceleration term */
     double xi;           /* Phase-3 cached fraction */
     double rho_cfg_off;  /* Phase-3 start, k_off = ceil(T rho_cfg_off) */
+    double cfg_strength; /* classifier-free guidance strength s (Supp. Sec. D): the steps
+                          * whose start time t_k >= cfg_t_lo use v = v_u + s (v_c - v_u),
+                          * v_u predicted for the all-zero condition on the same active
+                          * tokens; 0 disables guidance.  With s > 0, max_batch <= 32
+                          * (a guided step runs 2 B samples) */
+    double cfg_t_lo;     /* lower end of the CFG interval [cfg_t_lo, 1]; TRELLIS 0.5 */
 } f3dc_config;
 
 /* Weights: one bf16 device blob in layout version 1 -- every tensor

@@ -90,7 +90,8 @@ bool config_valid(const f3dc_config *c, std::string &why)
     if (c->grid < 1 || N % 32 != 0) why = "grid^3 must be a positive multiple of 32";
     else if (N > ssc_select_max_tokens()) why = "too many tokens for the selection kernel";
     else if (c->channels != kChannels) why = "channels must be 8";
-    else if (c->width < 128 || c->width % 128 != 0 || c->width > 2048) why = "width must be a multiple of 128 in [128, 2048]";
+    else if (c->width != 128 && c->width != 256 && c->width != 512 && c->width != 1024 && c->width != 2048)
+        why = "width must be 128, 256, 512, 1024 or 2048";
     else if (c->heads < 1 || c->width % c->heads != 0) why = "width must be divisible by heads";
     else if (c->width / c->heads != 32 && c->width / c->heads != 64) why = "head dim must be 32 or 64";
     else if (c->mlp_ratio != 4) why = "mlp_ratio must be 4";
@@ -105,6 +106,10 @@ bool config_valid(const f3dc_config *c, std::string &why)
     else if (!(c->eta > 0.0) || !std::isfinite(c->mu) || !(c->omega >= 0.0 && c->omega <= 1.0) ||
              !(c->xi >= 0.0 && c->xi <= 1.0) || !(c->rho_a >= 0.0) || !(c->rho_cfg_off >= 0.0))
         why = "hyperparameter out of range";
+    else if (!std::isfinite(c->cfg_strength) || c->cfg_strength < 0.0 || !std::isfinite(c->cfg_t_lo))
+        why = "cfg_strength must be finite and >= 0, cfg_t_lo finite";
+    else if (c->cfg_strength > 0.0 && 2 * c->max_batch > kMaxBatch)
+        why = "with classifier-free guidance max_batch must be <= 32";
     else
         return true;
     return false;
@@ -261,6 +266,7 @@ struct f3dc_handle {
     int32_t *gemm_cnt = nullptr;       // split-K per-tile arrival counters (kept at 0)
     cudaStream_t last_stream = nullptr;
     int cond_B = 0;
+    int cfg_B_now = 0;  // guided step in flight: samples >= cfg_B_now are the unguided copies
     // pinned per-step quota slots, two generations so one sampler call can
     // be enqueued while the previous one still copies from its slots
     int32_t *h_quota = nullptr;
@@ -447,6 +453,8 @@ cudaError_t run_attention(f3dc_handle *h, int mode, const CUtensorMap &tq, const
     p.tile_sample = h->tile_sample;
     p.plan = h->plan;
     p.nk_fixed = h->Nc;
+    p.kv_null_from = mode == 1 ? h->cfg_B_now : 0;
+    p.kv_null_sample = h->cfg.max_batch;
     p.out = h->att;
     p.ldo = h->W;
     p.scale_log2 = (float)(1.4426950408889634 / std::sqrt((double)h->dh));
@@ -473,7 +481,7 @@ f3dc_status run_dit(f3dc_handle *h, float t, const float *S, cudaStream_t s)
     // gather + embed the active tokens: 32 B latent + 4 B index in, 4W B out
     LAUNCH(KF_GATHER, wm(36.0 + 4.0 * dW),
            launch_gather_embed(S, h->N, W, h->active_idx, h->plan, h->tile_sample, h->wt(ly.in_w), h->wt(ly.in_b),
-                               h->pos, h->x, h->max_rows, h->num_sms, h->dev_err, s));
+                               h->pos, h->x, h->max_rows, h->num_sms, h->cfg_B_now, h->dev_err, s));
     const Work w_ln = wm(6.0 * dW);  // fp32 row in, bf16 row out
     Work w_self;
     w_self.c_sq = 4.0 * dW;          // Q K^T and P V among each sample's active tokens
@@ -647,6 +655,8 @@ f3dc_status f3dc_config_default(f3dc_config *cfg)
     cfg->omega = 0.7;
     cfg->xi = 0.7;
     cfg->rho_cfg_off = 0.75;
+    cfg->cfg_strength = 0.0;
+    cfg->cfg_t_lo = 0.5;
     return F3DC_OK;
 }
 
@@ -710,9 +720,12 @@ f3dc_status f3dc_create(const f3dc_config *cfg, const f3dc_weights *w, void *str
     h->G = cfg->gamma_up;
     h->T = cfg->steps;
     const int B = cfg->max_batch;
-    h->max_tiles = B * ((h->N + kTileRows - 1) / kTileRows);
+    // a guided step runs every sample twice (with its condition and with the
+    // zero condition, whose K/V rows sit in slot B of the condition cache)
+    const bool cfg_on = cfg->cfg_strength > 0.0;
+    h->max_tiles = (cfg_on ? 2 : 1) * B * ((h->N + kTileRows - 1) / kTileRows);
     h->max_rows = h->max_tiles * kTileRows;
-    h->ckv_rows = ((size_t)B * h->Nc + 2 * kTileRows - 1) / kTileRows * kTileRows;
+    h->ckv_rows = ((size_t)(B + (cfg_on ? 1 : 0)) * h->Nc + 2 * kTileRows - 1) / kTileRows * kTileRows;
     h->bn_qkv = pick_bn(3 * h->W);
     h->bn_w = pick_bn(h->W);
     h->bn_fc1 = pick_bn(h->Wm);
@@ -800,6 +813,14 @@ f3dc_status f3dc_create(const f3dc_config *cfg, const f3dc_weights *w, void *str
     CKC(cudaStreamCreateWithFlags(&h->exec_stream, cudaStreamNonBlocking));
     CKC(cudaEventCreateWithFlags(&h->ev_in, cudaEventDisableTiming));
     CKC(cudaEventCreateWithFlags(&h->ev_out, cudaEventDisableTiming));
+    if (cfg_on) {
+        // K/V of the zero condition: W_kv 0 + b_kv, i.e. the bias row in every
+        // one of the Nc rows of slot B (what the condition GEMM gives for a
+        // zero input, bf16 for bf16)
+        for (int l = 0; l < h->L; ++l)
+            CKC(launch_broadcast_row(h->ckv + ((size_t)l * h->ckv_rows + (size_t)B * h->Nc) * 2 * W, (size_t)2 * W,
+                                     h->wt(h->lay.blk[l].ckv_b), h->Nc, 2 * W, s));
+    }
 #undef CKC
     if (!build_maps(h)) {
         free_handle(h);
@@ -920,9 +941,16 @@ f3dc_status f3dc_step(f3dc_handle *h, int32_t k, int32_t B, float *S_inout, void
     const uint16_t *v1 = ring + (size_t)((k - 1) % 3) * slot;
     const uint16_t *v2 = ring + (size_t)(((k - 2) % 3 + 3) % 3) * slot;
 
-    // SSC selection + row plan (Algorithm 1 step 2, first line)
+    // classifier-free guidance when t_k lies in the CFG interval (Supp. Sec. D)
+    std::vector<float> t(h->T + 1);
+    time_schedule(h->cfg, t.data());
+    const bool guided = h->cfg.cfg_strength > 0.0 && (double)t[k - 1] >= h->cfg.cfg_t_lo;
+
+    // SSC selection + row plan (Algorithm 1 step 2, first line); a guided
+    // step's plan adds an unguided copy of every sample
     SelectArgs a;
     memset(&a, 0, sizeof(a));
+    a.cfg_dup = guided ? 1 : 0;
     a.v1 = v1;
     a.v2 = v2;
     a.quota = quota_dev;
@@ -944,9 +972,9 @@ f3dc_status f3dc_step(f3dc_handle *h, int32_t k, int32_t B, float *S_inout, void
     LAUNCH(KF_SELECT, w_sel, launch_ssc_select(a, s));
 
     // FlowTransformer on the active tokens at t_k
-    std::vector<float> t(h->T + 1);
-    time_schedule(h->cfg, t.data());
+    h->cfg_B_now = guided ? B : 0;
     f3dc_status st = run_dit(h, t[k - 1], S_inout, s);
+    h->cfg_B_now = 0;
     if (st != F3DC_OK) return st;
 
     // merge + Euler + history (Algorithm 1 step 3)
@@ -964,6 +992,8 @@ f3dc_status f3dc_step(f3dc_handle *h, int32_t k, int32_t B, float *S_inout, void
     m.G = h->G;
     m.dyn = dyn_voxels_dev;
     m.max_rows = h->max_rows;
+    m.cfg_s = guided ? (float)h->cfg.cfg_strength : 0.0f;
+    m.plan = h->plan;
     m.err = h->dev_err;
     Work w_merge;
     w_merge.c_tok = 96.0;  // S in/out (32 + 32 B), cached velocity in, v_t out (16 + 16 B)

@@ -79,7 +79,7 @@ F3DC_DEV Item decode_item(const AttnParams &p, int w)
         it.nk = p.plan->n_active[b];
     } else if (p.mode == 1) {
         const int b = p.tile_sample[t];
-        it.kv_row0 = b * p.nk_fixed;
+        it.kv_row0 = (p.kv_null_from > 0 && b >= p.kv_null_from ? p.kv_null_sample : b) * p.nk_fixed;
         it.nk = p.nk_fixed;
     } else {
         it.kv_row0 = 0;

@@ -55,7 +55,7 @@ struct GatherCfg {
 template <int NV>
 __global__ void __launch_bounds__(GatherCfg<NV>::kThreads, GatherCfg<NV>::kThreads >= 512 ? 1 : 2)
     k_gather_embed(const float *S, int N, const int32_t *active_idx, const Plan *plan, const int32_t *tile_sample,
-                   const bf16 *in_w, const bf16 *in_b, const float *pos, float *x, uint32_t *err)
+                   const bf16 *in_w, const bf16 *in_b, const float *pos, float *x, int cfg_B, uint32_t *err)
 {
     using Cfg = GatherCfg<NV>;
     constexpr int W = 128 * NV;
@@ -76,10 +76,11 @@ __global__ void __launch_bounds__(GatherCfg<NV>::kThreads, GatherCfg<NV>::kThrea
         const int r0 = unit * kGatherUnit;
         if (t < kGatherUnit) {
             const int b = tile_sample[r0 / kTileRows];
+            const int sb = cfg_B > 0 && b >= cfg_B ? b - cfg_B : b;  // guided step: unguided copy of sb
             const int j = r0 + t - plan->row_off[b];
             int i = -1;
             if (j < plan->n_active[b]) {
-                i = active_idx[(size_t)b * N + j];
+                i = active_idx[(size_t)sb * N + j];
                 if ((unsigned)i >= (unsigned)N) {
                     raise_error(err, kDevBadIndex);
                     i = -1;
@@ -87,7 +88,7 @@ __global__ void __launch_bounds__(GatherCfg<NV>::kThreads, GatherCfg<NV>::kThrea
             }
             s_idx[t] = i;
             if (i >= 0) {
-                const float *Si = S + ((size_t)b * N + i) * kChannels;
+                const float *Si = S + ((size_t)sb * N + i) * kChannels;
                 s_lat[t][0] = ld_f4(Si);
                 s_lat[t][1] = ld_f4(Si + 4);
             }
@@ -284,12 +285,21 @@ __global__ void __launch_bounds__(kMergeThreads) k_merge_euler(const MergeArgs a
         const int row = a.row_of_token[tok];
         uint32_t vb[8];
         if (row >= 0) {
-            if (row >= a.max_rows) {
+            const size_t ru = a.cfg_s != 0.0f ? (size_t)row + (size_t)(a.plan->m_rows / 2) : 0;
+            if (row >= a.max_rows || ru >= (size_t)a.max_rows) {
                 raise_error(a.err, kDevBadIndex);
                 for (int c = 0; c < 8; ++c) vb[c] = 0;
             } else {
                 const float4 v0 = ld_f4(a.v_active + (size_t)row * 8), v1 = ld_f4(a.v_active + (size_t)row * 8 + 4);
-                const float va[8] = {v0.x, v0.y, v0.z, v0.w, v1.x, v1.y, v1.z, v1.w};
+                float va[8] = {v0.x, v0.y, v0.z, v0.w, v1.x, v1.y, v1.z, v1.w};
+                if (a.cfg_s != 0.0f) {
+                    // guided step: v_u + s (v_c - v_u), the unguided copy's row
+                    // half the plan further (subtract, multiply, add)
+                    const float4 u0 = ld_f4(a.v_active + ru * 8), u1 = ld_f4(a.v_active + ru * 8 + 4);
+                    const float vu[8] = {u0.x, u0.y, u0.z, u0.w, u1.x, u1.y, u1.z, u1.w};
+#pragma unroll
+                    for (int c = 0; c < 8; ++c) va[c] = __fadd_rn(vu[c], __fmul_rn(a.cfg_s, __fsub_rn(va[c], vu[c])));
+                }
 #pragma unroll
                 for (int c = 0; c < 8; ++c) vb[c] = f32_to_bf16_bits(va[c]);
             }
@@ -416,27 +426,52 @@ int row_grid(int num_sms, int max_rows)
 template <int NV>
 void launch_gather_nv(const float *S, int N, const int32_t *active_idx, const Plan *plan, const int32_t *tile_sample,
                       const bf16 *in_w, const bf16 *in_b, const float *pos, float *x, int max_rows, int num_sms,
-                      uint32_t *err, cudaStream_t s)
+                      int cfg_B, uint32_t *err, cudaStream_t s)
 {
     const int units = max_rows / kGatherUnit;
     const int grid = units < 2 * num_sms ? (units > 0 ? units : 1) : 2 * num_sms;
     launch_k(k_gather_embed<NV>, dim3(grid), dim3(GatherCfg<NV>::kThreads), 0, s, S, N, active_idx, plan, tile_sample,
-             in_w, in_b, pos, x, err);
+             in_w, in_b, pos, x, cfg_B, err);
 }
 
 cudaError_t launch_gather_embed(const float *S, int N, int W, const int32_t *active_idx, const Plan *plan,
                                 const int32_t *tile_sample, const bf16 *in_w, const bf16 *in_b,
-                                const float *pos, float *x, int max_rows, int num_sms, uint32_t *err,
-                                cudaStream_t s)
+                                const float *pos, float *x, int max_rows, int num_sms, int cfg_B,
+                                uint32_t *err, cudaStream_t s)
 {
+#define F3DC_GATHER(NV)                                                                                        \
+    launch_gather_nv<NV>(S, N, active_idx, plan, tile_sample, in_w, in_b, pos, x, max_rows, num_sms, cfg_B, err, s)
     switch (W / 128) {
-    case 1: launch_gather_nv<1>(S, N, active_idx, plan, tile_sample, in_w, in_b, pos, x, max_rows, num_sms, err, s); break;
-    case 2: launch_gather_nv<2>(S, N, active_idx, plan, tile_sample, in_w, in_b, pos, x, max_rows, num_sms, err, s); break;
-    case 4: launch_gather_nv<4>(S, N, active_idx, plan, tile_sample, in_w, in_b, pos, x, max_rows, num_sms, err, s); break;
-    case 8: launch_gather_nv<8>(S, N, active_idx, plan, tile_sample, in_w, in_b, pos, x, max_rows, num_sms, err, s); break;
-    case 16: launch_gather_nv<16>(S, N, active_idx, plan, tile_sample, in_w, in_b, pos, x, max_rows, num_sms, err, s); break;
+    case 1: F3DC_GATHER(1); break;
+    case 2: F3DC_GATHER(2); break;
+    case 4: F3DC_GATHER(4); break;
+    case 8: F3DC_GATHER(8); break;
+    case 16: F3DC_GATHER(16); break;
     default: return cudaErrorInvalidValue;
     }
+#undef F3DC_GATHER
+    return cudaGetLastError();
+}
+
+__global__ void k_broadcast_row(bf16 *dst, size_t ld, const bf16 *src, int rows, int cols)
+{
+    griddep_launch();
+    griddep_wait();
+    const int c8 = cols / 8;
+    for (size_t q = (size_t)blockIdx.x * blockDim.x + threadIdx.x; q < (size_t)rows * c8;
+         q += (size_t)gridDim.x * blockDim.x) {
+        const size_t r = q / c8, c = q - r * c8;
+        reinterpret_cast<uint4 *>(dst + r * ld)[c] = reinterpret_cast<const uint4 *>(src)[c];
+    }
+}
+
+cudaError_t launch_broadcast_row(bf16 *dst, size_t ld, const bf16 *src, int rows, int cols, cudaStream_t s)
+{
+    if (cols % 8 != 0 || ld % 8 != 0 || rows < 0) return cudaErrorInvalidValue;
+    if (rows == 0) return cudaSuccess;
+    const size_t total = (size_t)rows * (cols / 8);
+    const int grid = (int)((total + 255) / 256 < 1024 ? (total + 255) / 256 : 1024);
+    launch_k(k_broadcast_row, dim3(grid), dim3(256), 0, s, dst, ld, src, rows, cols);
     return cudaGetLastError();
 }
 

@@ -73,7 +73,7 @@ F3DC_DEV int clamp_quota(int q, int N) { return q < 0 ? 0 : (q > N ? N : q); }
 static_assert(kMaxBatch <= 64, "write_plan covers two samples per lane");
 F3DC_DEV void write_plan(const SelectArgs &a, int b, int na, int &off)
 {
-    __shared__ int s_off;
+    __shared__ int s_off, s_tot_rows;
     if (threadIdx.x < 32) {
         const int lane = threadIdx.x;
         const int r0 = lane < a.B ? pad_tile(a.N - clamp_quota(a.quota[lane], a.N)) : 0;
@@ -86,12 +86,18 @@ F3DC_DEV void write_plan(const SelectArgs &a, int b, int na, int &off)
         }
         if (lane == 0) {
             s_off = before;
+            s_tot_rows = tot;
             if (a.plan) {
                 a.plan->n_active[b] = na;
                 a.plan->row_off[b] = before;
+                if (a.cfg_dup) {  // the unguided copy of sample b
+                    a.plan->n_active[a.B + b] = na;
+                    a.plan->row_off[a.B + b] = tot + before;
+                }
                 if (b == 0) {
-                    a.plan->m_rows = tot;
-                    a.plan->n_tiles = tot / kTileRows;
+                    const int all = a.cfg_dup ? 2 * tot : tot;
+                    a.plan->m_rows = all;
+                    a.plan->n_tiles = all / kTileRows;
                 }
             }
         }
@@ -101,6 +107,10 @@ F3DC_DEV void write_plan(const SelectArgs &a, int b, int na, int &off)
     if (a.tile_sample) {
         const int t0 = off / kTileRows, nt = pad_tile(na) / kTileRows;
         for (int t = threadIdx.x; t < nt; t += blockDim.x) a.tile_sample[t0 + t] = b;
+        if (a.cfg_dup) {
+            const int t1 = (s_tot_rows + off) / kTileRows;
+            for (int t = threadIdx.x; t < nt; t += blockDim.x) a.tile_sample[t1 + t] = a.B + b;
+        }
     }
 }
 
@@ -366,7 +376,8 @@ int ssc_select_max_tokens() { return kSelMaxTokens; }
 
 cudaError_t launch_ssc_select(const SelectArgs &a, cudaStream_t s)
 {
-    if (a.N > kSelMaxTokens || a.B < 1 || a.B > kMaxBatch) return cudaErrorInvalidValue;
+    if (a.N > kSelMaxTokens || a.B < 1 || a.B > kMaxBatch || (a.cfg_dup && 2 * a.B > kMaxBatch))
+        return cudaErrorInvalidValue;
     const size_t smem = (size_t)a.N * sizeof(uint32_t);
     cudaError_t e = cudaFuncSetAttribute(k_ssc_select, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;

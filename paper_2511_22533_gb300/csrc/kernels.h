@@ -40,6 +40,9 @@ struct SelectArgs {
     int32_t *row_of_token;     // [B, N], nullable: packed row or -1 if cached
     Plan *plan;                // nullable
     int32_t *tile_sample;      // nullable
+    // guided (CFG) step: the plan also lists samples B..2B-1, copies of
+    // samples 0..B-1 (same active counts, rows after all of 0..B-1's)
+    int cfg_dup;
     uint32_t *err;
 };
 cudaError_t launch_ssc_select(const SelectArgs &a, cudaStream_t s);
@@ -53,10 +56,14 @@ cudaError_t launch_plan_from_counts(const int32_t *n_active, const int32_t *acti
 
 // ------------------------------------------------------------ row kernels
 // x[r] = in_w S[b, i] + in_b + pos[i] for packed active row r; zero pad rows.
+// cfg_B > 0: plan samples b >= cfg_B read the tokens and latents of b - cfg_B.
 cudaError_t launch_gather_embed(const float *S, int N, int W, const int32_t *active_idx, const Plan *plan,
                                 const int32_t *tile_sample, const bf16 *in_w, const bf16 *in_b,
-                                const float *pos, float *x, int max_rows, int num_sms, uint32_t *err,
-                                cudaStream_t s);
+                                const float *pos, float *x, int max_rows, int num_sms, int cfg_B,
+                                uint32_t *err, cudaStream_t s);
+
+// Every one of `rows` rows of dst (leading dimension ld) = the bf16 row src.
+cudaError_t launch_broadcast_row(bf16 *dst, size_t ld, const bf16 *src, int rows, int cols, cudaStream_t s);
 
 // h = LN(x) (1 + scale) + shift (mode 0, fp32 mod vectors) or LN(x) g + b
 // (mode 1, bf16 affine).  rows from plan->m_rows.
@@ -82,6 +89,10 @@ struct MergeArgs {
     int G;
     int64_t *dyn;                 // nullable [B]
     int max_rows;
+    // guided step (cfg_s != 0): the active velocity is v_u + cfg_s (v_c - v_u)
+    // with v_c at the token's row and v_u plan->m_rows / 2 rows further
+    float cfg_s;
+    const Plan *plan;
     uint32_t *err;
 };
 cudaError_t launch_merge_euler(const MergeArgs &a, cudaStream_t s);
@@ -200,6 +211,9 @@ struct AttnParams {
     bf16 *out;
     int ldo;
     float scale_log2;              // log2(e) / sqrt(dh)
+    // mode 1: samples b >= kv_null_from (0: none) attend to the keys of
+    // sample slot kv_null_sample (the zero condition of a guided step)
+    int kv_null_from, kv_null_sample;
     uint32_t *err;
 };
 cudaError_t launch_attention(const CUtensorMap *tq, const CUtensorMap *tk, const CUtensorMap *tv,

@@ -120,7 +120,7 @@ def test_forward_trellis_width_two_blocks(orc):
 
 def test_forward_trellis_width_few_active(orc):
     # 300 and 77 active tokens at TRELLIS width: every projection (QKV with the
-    # QK norm, out, cross-Q, cross-out, fc1 + GELU, fc2) runs with split K
+    # QK norm, out, cross-Q, cross-out, fc1 + GELU, fc2) runs few, narrow tiles
     shape = synth.ModelShape(16, 8, 1024, 1, 16, 4, 1374, 1024, 25, 64)
     c = Ctx(orc, shape, 2, seed=8)
     g = np.random.default_rng(8)
