@@ -153,7 +153,15 @@ static float orc_norm1(float x, float mn, float mx)
     return num / den;
 }
 
-void orc_ssc_score(const uint16_t *v1, const uint16_t *v2, int N, int C, double omega, float *score)
+/*
+ * Variant (SSC with three predictions): v3 = v_i(t-3) non-NULL replaces the
+ * first difference by the second difference of the velocity,
+ *   A_i = ||(v_i(t-1) - v_i(t-2)) - (v_i(t-2) - v_i(t-3))||_2,
+ * the discrete rate of change of Sec. 4.1's acceleration; each channel's
+ * term is (x - y) - (y - z), two subtractions then one, in fp32.
+ */
+void orc_ssc_score3(const uint16_t *v1, const uint16_t *v2, const uint16_t *v3, int N, int C, double omega,
+                    float *score)
 {
     float *V = (float *)malloc(sizeof(float) * (size_t)(N > 0 ? N : 1));
     float *A = (float *)malloc(sizeof(float) * (size_t)(N > 0 ? N : 1));
@@ -164,6 +172,11 @@ void orc_ssc_score(const uint16_t *v1, const uint16_t *v2, int N, int C, double 
             float x = bf2f(v1[(size_t)i * C + c]);
             float y = bf2f(v2[(size_t)i * C + c]);
             float d = x - y;
+            if (v3) {
+                float z = bf2f(v3[(size_t)i * C + c]);
+                float e = y - z;
+                d = d - e;
+            }
             float xx = x * x;
             float dd = d * d;
             sv = sv + xx;
@@ -187,6 +200,11 @@ void orc_ssc_score(const uint16_t *v1, const uint16_t *v2, int N, int C, double 
     }
     free(V);
     free(A);
+}
+
+void orc_ssc_score(const uint16_t *v1, const uint16_t *v2, int N, int C, double omega, float *score)
+{
+    orc_ssc_score3(v1, v2, NULL, N, C, omega, score);
 }
 
 /* ------------------------------------------------------------------------ */
@@ -679,12 +697,15 @@ void orc_dit_forward(const void *vm, const float *S, const int32_t *active_idx, 
  * cfg_on: guide the steps k with t_k >= cfg_t_lo with strength cfg_s; the
  *   unconditional prediction sees the all-zero condition (reading: the paper
  *   names no null condition) and the same active tokens.
+ * ssc_accel: 1 scores with the second difference over the last three
+ *   velocities (orc_ssc_score3), 0 with the first difference of Sec. 4.1.
  */
 int orc_sample(const void *vm, int T, double eta, double rho_a, double rho_off, double mu,
                double omega, double xi, int f_corr, int tau, int refresh_mode,
                float *S, const uint16_t *cond, int B, const double *sigma_override,
                const int32_t *quota_schedule, int32_t *quota_log, int32_t *nact_log,
-               double *sigma_out, uint16_t *v_hist_out, int cfg_on, double cfg_s, double cfg_t_lo)
+               double *sigma_out, uint16_t *v_hist_out, int cfg_on, double cfg_s, double cfg_t_lo,
+               int ssc_accel)
 {
     const orc_model *m = (const orc_model *)vm;
     const int N = m->grid * m->grid * m->grid, C = m->C, G = m->G;
@@ -697,6 +718,7 @@ int orc_sample(const void *vm, int T, double eta, double rho_a, double rho_off, 
     uint16_t *vc = (uint16_t *)calloc(NC, sizeof(uint16_t)); /* v_cache <- 0 */
     uint16_t *vp = (uint16_t *)calloc(NC, sizeof(uint16_t)); /* v_prev_cache <- 0 */
     uint16_t *vt = (uint16_t *)malloc(sizeof(uint16_t) * NC);
+    uint16_t *vpp = (uint16_t *)calloc(NC, sizeof(uint16_t)); /* v(t-3) <- 0 */
     float *score = (float *)malloc(sizeof(float) * (size_t)N);
     uint8_t *cached = (uint8_t *)malloc((size_t)N);
     int32_t *idx = (int32_t *)malloc(sizeof(int32_t) * (size_t)N);
@@ -719,6 +741,7 @@ int orc_sample(const void *vm, int T, double eta, double rho_a, double rho_off, 
         orc_cond_kv(m, cond + (size_t)b * m->Nc * m->Dc, kv);
         memset(vc, 0, sizeof(uint16_t) * NC);
         memset(vp, 0, sizeof(uint16_t) * NC);
+        memset(vpp, 0, sizeof(uint16_t) * NC);
         int consec = 0;
         double sigma = sigma_override ? sigma_override[b] : 0.0;
         for (int k = 1; k <= T; ++k) {
@@ -731,7 +754,7 @@ int orc_sample(const void *vm, int T, double eta, double rho_a, double rho_off, 
             c = orc_tau_gate(c, tau, refresh_mode, &consec);
             int a;
             if (c > 0) {
-                orc_ssc_score(vc, vp, N, C, omega, score);
+                orc_ssc_score3(vc, vp, ssc_accel ? vpp : NULL, N, C, omega, score);
                 a = orc_select(score, N, c, cached, idx);
             } else {
                 for (int i = 0; i < N; ++i) idx[i] = i;
@@ -758,8 +781,9 @@ int orc_sample(const void *vm, int T, double eta, double rho_a, double rho_off, 
                 if (sigma_out) sigma_out[b] = meas;
                 if (!sigma_override) sigma = meas;
             }
-            /* v_prev_cache <- v_cache; v_cache <- v_t */
-            uint16_t *tmp = vp;
+            /* v(t-3) <- v_prev_cache <- v_cache <- v_t */
+            uint16_t *tmp = vpp;
+            vpp = vp;
             vp = vc;
             vc = vt;
             vt = tmp;
@@ -769,7 +793,7 @@ int orc_sample(const void *vm, int T, double eta, double rho_a, double rho_off, 
             memcpy(v_hist_out + (size_t)B * NC + (size_t)b * NC, vp, sizeof(uint16_t) * NC);
         }
     }
-    free(t); free(kv); free(vc); free(vp); free(vt); free(score); free(cached); free(idx);
+    free(t); free(kv); free(vc); free(vp); free(vt); free(vpp); free(score); free(cached); free(idx);
     free(va); free(Sold); free(occ_a); free(occ_b); free(kv_null); free(va_c); free(va_u);
     return 0;
 }

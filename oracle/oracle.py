@@ -77,7 +77,8 @@ def lib():
             L.orc_sample.argtypes = [C.c_void_p, C.c_int, C.c_double, C.c_double, C.c_double,
                                      C.c_double, C.c_double, C.c_double, C.c_int, C.c_int, C.c_int,
                                      _f32p, _u16p, C.c_int, _f64p, _i32p, _i32p, _i32p, _f64p, _u16p,
-                                     C.c_int, C.c_double, C.c_double]
+                                     C.c_int, C.c_double, C.c_double, C.c_int]
+            L.orc_ssc_score3.argtypes = [_u16p, _u16p, _u16p, C.c_int, C.c_int, C.c_double, _f32p]
             L.orc_cfg_on.argtypes = [C.c_int, C.c_double, C.c_double, C.c_int]
             L.orc_cfg_combine.argtypes = [C.c_longlong, _f32p, _f32p, C.c_double, _f32p]
             L.orc_f32_to_bf16.argtypes = [C.c_float]
@@ -131,6 +132,15 @@ def ssc_score(v1_bits: np.ndarray, v2_bits: np.ndarray, omega: float) -> np.ndar
     N, Cc = v1.shape
     out = np.empty(N, np.float32)
     lib().orc_ssc_score(_p(v1, _u16p), _p(v2, _u16p), N, Cc, omega, _p(out, _f32p))
+    return out
+
+
+def ssc_score3(v1_bits: np.ndarray, v2_bits: np.ndarray, v3_bits: np.ndarray, omega: float) -> np.ndarray:
+    """SSC score with the second-difference acceleration over v(t-1), v(t-2), v(t-3)."""
+    v1, v2, v3 = _u16(v1_bits), _u16(v2_bits), _u16(v3_bits)
+    N, Cc = v1.shape
+    out = np.empty(N, np.float32)
+    lib().orc_ssc_score3(_p(v1, _u16p), _p(v2, _u16p), _p(v3, _u16p), N, Cc, omega, _p(out, _f32p))
     return out
 
 
@@ -284,7 +294,7 @@ class Model:
 
     def sample(self, S: np.ndarray, cond_bits: np.ndarray, *, T, eta=3.0, rho_a=0.2, rho_off=0.75,
                mu=-0.07, omega=0.7, xi=0.7, f_corr=3, tau=3, refresh_mode=0,
-               sigma_override=None, quota_schedule=None, cfg=None, cfg_t_lo=0.5):
+               sigma_override=None, quota_schedule=None, cfg=None, cfg_t_lo=0.5, ssc_accel=0):
         """Algorithm 1 for B samples.  Returns dict(S, quota, n_active, sigma, v_hist).
         cfg: guidance strength s (None: unguided) for the steps with t_k >= cfg_t_lo."""
         S = _f32(S).copy()
@@ -302,5 +312,6 @@ class Model:
                          _p(sov, _f64p) if sov is not None else None,
                          _p(qs, _i32p) if qs is not None else None,
                          _p(ql, _i32p), _p(nl, _i32p), _p(so, _f64p), _p(vh, _u16p),
-                         0 if cfg is None else 1, 0.0 if cfg is None else float(cfg), float(cfg_t_lo))
+                         0 if cfg is None else 1, 0.0 if cfg is None else float(cfg), float(cfg_t_lo),
+                         int(ssc_accel))
         return dict(S=S, quota=ql, n_active=nl, sigma=so, v_hist=vh)

@@ -153,3 +153,44 @@ def test_selection_signed_zero_ties_by_index(orc):
     s = np.array([0.0, -0.0, 0.0, -0.0], np.float32)
     cached, _ = orc.select(s, 2)
     assert cached.tolist() == [1, 1, 0, 0]
+
+
+# ---- SSC with three predictions: the second difference of the velocity
+def _bf16(a):
+    return synth.f32_to_bf16_bits(np.asarray(a, np.float32))
+
+
+def test_ssc3_linear_history_has_zero_acceleration(orc):
+    # v(t-3), v(t-2), v(t-1) on a straight line (small integers: exact in
+    # bf16) have a zero second difference everywhere, so the score is the
+    # velocity term alone: (1 - w) norm(V)
+    rng = np.random.default_rng(0)
+    a = rng.integers(-8, 8, (64, 8)).astype(np.float32)
+    d = rng.integers(-4, 4, (64, 8)).astype(np.float32)
+    v3, v2, v1 = _bf16(a), _bf16(a + d), _bf16(a + 2 * d)
+    s3 = orc.ssc_score3(v1, v2, v3, 0.7)
+    nv = orc.ssc_score(v1, v2, 0.0)                 # w = 0: exactly norm(V)
+    np.testing.assert_array_equal(s3, (np.float32(1.0) - np.float32(0.7)) * nv)
+
+
+def test_ssc3_constant_previous_pair_is_the_first_difference(orc):
+    # v(t-3) = v(t-2): the second difference is the first difference exactly
+    v = synth.velocity_history(4, 8, 1, seed=2)
+    v1, v2 = v[2, 0], v[1, 0]
+    np.testing.assert_array_equal(orc.ssc_score3(v1, v2, v2, 0.7), orc.ssc_score(v1, v2, 0.7))
+
+
+def test_ssc3_quadratic_history_orders_by_curvature(orc):
+    # v = a + b t + c t^2 at t = 0, 1, 2: second difference 2c per token, so
+    # with w = 1 the order is that of |c|
+    rng = np.random.default_rng(1)
+    n = 27
+    a = rng.integers(-4, 4, (n, 8)).astype(np.float32)
+    b = rng.integers(-2, 2, (n, 8)).astype(np.float32)
+    c = np.zeros((n, 8), np.float32)
+    mags = rng.permutation(n).astype(np.float32) + 1
+    c[:, 0] = mags / 8.0                            # distinct |c|, exact in bf16
+    v3, v2, v1 = _bf16(a), _bf16(a + b + c), _bf16(a + 2 * b + 4 * c)
+    s = orc.ssc_score3(v1, v2, v3, 1.0)
+    np.testing.assert_array_equal(np.argsort(s, kind="stable"), np.argsort(mags, kind="stable"))
+    assert s[np.argmin(mags)] == 0.0 and s[np.argmax(mags)] == 1.0
