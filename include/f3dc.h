@@ -96,6 +96,10 @@ typedef struct f3dc_config {
                           * tokens; 0 disables guidance.  With s > 0, max_batch <= 32
                           * (a guided step runs 2 B samples) */
     double cfg_t_lo;     /* lower end of the CFG interval [cfg_t_lo, 1]; TRELLIS 0.5 */
+    int32_t ssc_accel;   /* SSC acceleration term: 0 the first difference |v(t-1) - v(t-2)|
+                          * (Sec. 4.1), 1 the second difference
+                          * |(v(t-1) - v(t-2)) - (v(t-2) - v(t-3))| over the ring's three slots */
+    int32_t reserved0;   /* must be 0 */
 } f3dc_config;
 
 /* Weights: one bf16 device blob in layout version 1 -- every tensor

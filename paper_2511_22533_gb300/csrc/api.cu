@@ -110,6 +110,8 @@ bool config_valid(const f3dc_config *c, std::string &why)
         why = "cfg_strength must be finite and >= 0, cfg_t_lo finite";
     else if (c->cfg_strength > 0.0 && 2 * c->max_batch > kMaxBatch)
         why = "with classifier-free guidance max_batch must be <= 32";
+    else if ((c->ssc_accel != 0 && c->ssc_accel != 1) || c->reserved0 != 0)
+        why = "ssc_accel must be 0 or 1 and reserved0 0";
     else
         return true;
     return false;
@@ -953,6 +955,8 @@ f3dc_status f3dc_step(f3dc_handle *h, int32_t k, int32_t B, float *S_inout, void
     a.cfg_dup = guided ? 1 : 0;
     a.v1 = v1;
     a.v2 = v2;
+    // v(t-3) still sits in the slot this step overwrites (zeros before step 3)
+    a.v3 = h->cfg.ssc_accel ? v_new : nullptr;
     a.quota = quota_dev;
     a.B = B;
     a.N = h->N;

@@ -11,7 +11,9 @@
 // definition and stores an order-preserving 32-bit key per token in shared
 // memory.  A 4 x 8-bit radix select finds the c-th smallest key; an
 // index-ordered scan then caches every key below it plus the lowest-index
-// ties, and compacts the active tokens in ascending order.
+// ties, and compacts the active tokens in ascending order.  With a third
+// history slot (SSC with three predictions) the acceleration term is the
+// second difference of the velocity and pass 1 reads 48 B per token.
 #include "common.cuh"
 #include "kernels.h"
 
@@ -24,12 +26,16 @@ constexpr int kSelWarps = kSelThreads / 32;
 constexpr int kSelMaxTokens = 49152;  // 4-byte keys in shared memory (192 KB + 16 KB of histograms)
 constexpr int kRegTok = 4;            // tokens per thread held in registers between passes 1 and 2
 
-F3DC_DEV void load_token(const uint16_t *v1, const uint16_t *v2, size_t tok, float &V, float &A)
+// V = |v1|, A = |v1 - v2| (Sec. 4.1), or with v3 the second difference
+// |(v1 - v2) - (v2 - v3)|, each channel term in that fp32 order.
+F3DC_DEV void load_token(const uint16_t *v1, const uint16_t *v2, const uint16_t *v3, size_t tok, float &V, float &A)
 {
     const uint4 p = __ldg(reinterpret_cast<const uint4 *>(v1) + tok);
     const uint4 q = __ldg(reinterpret_cast<const uint4 *>(v2) + tok);
+    const uint4 r = v3 ? __ldg(reinterpret_cast<const uint4 *>(v3) + tok) : make_uint4(0, 0, 0, 0);
     const uint32_t pw[4] = {p.x, p.y, p.z, p.w};
     const uint32_t qw[4] = {q.x, q.y, q.z, q.w};
+    const uint32_t rw[4] = {r.x, r.y, r.z, r.w};
     float sv = 0.0f, sa = 0.0f;
 #pragma unroll
     for (int c = 0; c < 8; ++c) {
@@ -37,7 +43,8 @@ F3DC_DEV void load_token(const uint16_t *v1, const uint16_t *v2, size_t tok, flo
         const uint32_t qu = (qw[c >> 1] >> ((c & 1) * 16)) & 0xFFFFu;
         const float x = bf16_bits_to_f32(pu);
         const float y = bf16_bits_to_f32(qu);
-        const float d = __fsub_rn(x, y);
+        float d = __fsub_rn(x, y);
+        if (v3) d = __fsub_rn(d, __fsub_rn(y, bf16_bits_to_f32((rw[c >> 1] >> ((c & 1) * 16)) & 0xFFFFu)));
         sv = __fadd_rn(sv, __fmul_rn(x, x));
         sa = __fadd_rn(sa, __fmul_rn(d, d));
     }
@@ -159,7 +166,7 @@ __global__ void __launch_bounds__(kSelThreads, 1) k_ssc_select(const SelectArgs 
     for (int r = 0; r < kRegTok; ++r) {
         const int i = tid + r * kSelThreads;
         Vr[r] = Ar[r] = 0.0f;
-        if (i < N) load_token(a.v1, a.v2, base + i, Vr[r], Ar[r]);
+        if (i < N) load_token(a.v1, a.v2, a.v3, base + i, Vr[r], Ar[r]);
     }
 #pragma unroll
     for (int r = 0; r < kRegTok; ++r) {
@@ -172,7 +179,7 @@ __global__ void __launch_bounds__(kSelThreads, 1) k_ssc_select(const SelectArgs 
     }
     for (int i = tid + kRegTok * kSelThreads; i < N; i += kSelThreads) {
         float V, A;
-        load_token(a.v1, a.v2, base + i, V, A);
+        load_token(a.v1, a.v2, a.v3, base + i, V, A);
         if (V < mnV) mnV = V;
         if (V > mxV) mxV = V;
         if (A < mnA) mnA = A;
@@ -215,7 +222,7 @@ __global__ void __launch_bounds__(kSelThreads, 1) k_ssc_select(const SelectArgs 
     }
     for (int i = tid + kRegTok * kSelThreads; i < N; i += kSelThreads) {
         float V, A;
-        load_token(a.v1, a.v2, base + i, V, A);
+        load_token(a.v1, a.v2, a.v3, base + i, V, A);
         keys[i] = score_key(score(V, A));
     }
     __syncthreads();

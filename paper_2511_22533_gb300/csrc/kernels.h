@@ -31,6 +31,7 @@ struct Plan {
 // ------------------------------------------------------------ selection
 struct SelectArgs {
     const uint16_t *v1, *v2;   // bf16 [B, N, 8]
+    const uint16_t *v3;        // nullable: second-difference acceleration with v(t-3)
     const int32_t *quota;      // [B]
     int B, N;
     float wa, wv;              // omega and 1 - omega, fp32

@@ -37,7 +37,8 @@ class Config(C.Structure):
                 ("gamma_up", C.c_int32), ("tau", C.c_int32), ("f_corr", C.c_int32),
                 ("refresh_mode", C.c_int32), ("eta", C.c_double), ("rho_a", C.c_double), ("mu", C.c_double),
                 ("omega", C.c_double), ("xi", C.c_double), ("rho_cfg_off", C.c_double),
-                ("cfg_strength", C.c_double), ("cfg_t_lo", C.c_double)]
+                ("cfg_strength", C.c_double), ("cfg_t_lo", C.c_double), ("ssc_accel", C.c_int32),
+                ("reserved0", C.c_int32)]
 
 
 class KernelStats(C.Structure):
