@@ -99,10 +99,13 @@ typedef struct f3dc_config {
     int32_t ssc_accel;   /* SSC acceleration term: 0 the first difference |v(t-1) - v(t-2)|
                           * (Sec. 4.1), 1 the second difference
                           * |(v(t-1) - v(t-2)) - (v(t-2) - v(t-3))| over the ring's three slots */
-    int32_t reserved0;   /* must be 0 */
+    int32_t decoder;     /* grid decoder O(S) of Eq. 1 at the anchor step: 0 the linear
+                          * stand-in (dec_w), 1 the convolutional stand-in (dc*_w: 3x3x3
+                          * convolutions C->16 at D^3, 2x up, 16->8, 2x up, 8->1 at (4D)^3,
+                          * ReLU between; needs gamma_up = 64) */
 } f3dc_config;
 
-/* Weights: one bf16 device blob in layout version 1 -- every tensor
+/* Weights: one bf16 device blob in layout version 2 -- every tensor
  * row-major ([out, in] for linear layers), concatenated in this order, each
  * starting at a multiple of 64 elements (W = width, C = channels,
  * Dc = cond_dim, Wm = 4 W, G = gamma_up):
@@ -111,11 +114,14 @@ typedef struct f3dc_config {
  *     qn_g [W], kn_g [W], o_w [W,W], o_b [W], ln2_g [W], ln2_b [W],
  *     cq_w [W,W], cq_b [W], ckv_w [2W,Dc], ckv_b [2W], co_w [W,W], co_b [W],
  *     fc1_w [Wm,W], fc1_b [Wm], fc2_w [W,Wm], fc2_b [W],
- *   fmod_w [2W,W], fmod_b [2W], out_w [C,W], out_b [C], dec_w [C,G].
+ *   fmod_w [2W,W], fmod_b [2W], out_w [C,W], out_b [C], dec_w [C,G],
+ *   dc1_w [16, C*27], dc1_b [16], dc2_w [8, 16*27], dc2_b [8], dc3_w [1, 8*27],
+ *   dc3_b [1] (the convolutional stand-in decoder, 3x3x3 taps k = 9 (dz+1) +
+ *   3 (dy+1) + (dx+1) innermost).
  * f3dc_create copies what it needs into library-owned memory; the caller
  * may free the blob when f3dc_create returns. */
 typedef struct f3dc_weights {
-    int32_t layout_version; /* must be 1 */
+    int32_t layout_version; /* must be 2 */
     const void *blob;       /* device pointer, bf16 */
     size_t blob_elems;      /* must equal f3dc_weights_elems(cfg) */
 } f3dc_weights;

@@ -331,6 +331,8 @@ typedef struct {
     /* per block */
     float **mod_w, **mod_b, **qkv_w, **qkv_b, **qn_g, **kn_g, **o_w, **o_b, **ln2_g, **ln2_b;
     float **cq_w, **cq_b, **ckv_w, **ckv_b, **co_w, **co_b, **fc1_w, **fc1_b, **fc2_w, **fc2_b;
+    /* convolutional stand-in decoder */
+    uint16_t *dc1_w, *dc1_b, *dc2_w, *dc2_b, *dc3_w, *dc3_b;
 } orc_model;
 
 static float *take(const uint16_t *blob, size_t *pos, size_t n)
@@ -341,7 +343,15 @@ static float *take(const uint16_t *blob, size_t *pos, size_t n)
     return t;
 }
 
-/* Weight blob layout version 1: bf16, nn.Linear [out, in] row-major, in the
+static uint16_t *take_bits(const uint16_t *blob, size_t *pos, size_t n)
+{
+    uint16_t *t = (uint16_t *)malloc(sizeof(uint16_t) * n);
+    memcpy(t, blob + *pos, sizeof(uint16_t) * n);
+    *pos += (n + ORC_ALIGN - 1) / ORC_ALIGN * ORC_ALIGN;
+    return t;
+}
+
+/* Weight blob layout version 2: bf16, nn.Linear [out, in] row-major, in the
  * order below, each tensor starting at a multiple of 64 elements. */
 void *orc_model_create(int grid, int C, int W, int L, int H, int mlp, int Nc, int Dc, int G,
                        const uint16_t *blob)
@@ -389,8 +399,13 @@ void *orc_model_create(int grid, int C, int W, int L, int H, int mlp, int Nc, in
     m->fmod_b = take(blob, &p, (size_t)2 * W);
     m->out_w = take(blob, &p, (size_t)C * W);
     m->out_b = take(blob, &p, C);
-    m->dec_w = (uint16_t *)malloc(sizeof(uint16_t) * (size_t)C * G);
-    memcpy(m->dec_w, blob + p, sizeof(uint16_t) * (size_t)C * G);
+    m->dec_w = take_bits(blob, &p, (size_t)C * G);
+    m->dc1_w = take_bits(blob, &p, (size_t)16 * C * 27);
+    m->dc1_b = take_bits(blob, &p, 16);
+    m->dc2_w = take_bits(blob, &p, (size_t)8 * 16 * 27);
+    m->dc2_b = take_bits(blob, &p, 8);
+    m->dc3_w = take_bits(blob, &p, (size_t)8 * 27);
+    m->dc3_b = take_bits(blob, &p, 1);
     return m;
 }
 
@@ -400,6 +415,7 @@ void orc_model_free(void *vm)
     if (!m) return;
     free(m->in_w); free(m->in_b); free(m->t_w1); free(m->t_b1); free(m->t_w2); free(m->t_b2);
     free(m->fmod_w); free(m->fmod_b); free(m->out_w); free(m->out_b); free(m->dec_w);
+    free(m->dc1_w); free(m->dc1_b); free(m->dc2_w); free(m->dc2_b); free(m->dc3_w); free(m->dc3_b);
     float **blk[] = {m->mod_w, m->mod_b, m->qkv_w, m->qkv_b, m->qn_g, m->kn_g, m->o_w, m->o_b,
                      m->ln2_g, m->ln2_b, m->cq_w, m->cq_b, m->ckv_w, m->ckv_b, m->co_w, m->co_b,
                      m->fc1_w, m->fc1_b, m->fc2_w, m->fc2_b};
@@ -680,6 +696,59 @@ void orc_dit_forward(const void *vm, const float *S, const int32_t *active_idx, 
     free(x); free(h); free(y); free(o); free(qkv); free(u); free(temb); free(mod); free(pe);
 }
 
+/* ------------------------------------------------------------------------ */
+/* Convolutional stand-in decoder (reading: TRELLIS's decoder and weights   */
+/* are not in the paper; Eq. 1 only needs a grid decoder O(S)).  The shape  */
+/* of an upsampling 3-D convolution stack: 3x3x3 convolutions with zero     */
+/* padding, ReLU, nearest-neighbour 2x upsampling in between:               */
+/*   C -> 16 at D^3, x2, 16 -> 8 at (2D)^3, x2, 8 -> 1 at (4D)^3,           */
+/* and sub-voxel v is occupied iff its logit > 0 ((4D)^3 = 64 N sub-voxels,  */
+/* gamma_up = 64).  Each output: acc = bias, then for tap k = 0..26         */
+/* ((dz, dy, dx) in {-1, 0, 1}^3, dx fastest) and input channel ci in order, */
+/* acc = acc + x w with one rounding per * and +; taps outside the grid are  */
+/* skipped.  Grid index (z D + y) D + x, as the tokens.                     */
+/* ------------------------------------------------------------------------ */
+static void orc_conv3d(const float *in, int cin, int din, int up, const uint16_t *w, const uint16_t *b, int cout,
+                       int relu, float *out)
+{
+    const int d = din * up;
+    const size_t vin = (size_t)din * din * din, vout = (size_t)d * d * d;
+    for (int co = 0; co < cout; ++co)
+        for (int z = 0; z < d; ++z)
+            for (int y = 0; y < d; ++y)
+                for (int x = 0; x < d; ++x) {
+                    float acc = bf2f(b[co]);
+                    for (int k = 0; k < 27; ++k) {
+                        const int zz = z + k / 9 - 1, yy = y + (k / 3) % 3 - 1, xx = x + k % 3 - 1;
+                        if (zz < 0 || zz >= d || yy < 0 || yy >= d || xx < 0 || xx >= d) continue;
+                        const size_t src = ((size_t)(zz / up) * din + (size_t)(yy / up)) * din + (size_t)(xx / up);
+                        for (int ci = 0; ci < cin; ++ci) {
+                            const float p = in[(size_t)ci * vin + src] * bf2f(w[((size_t)co * cin + ci) * 27 + k]);
+                            acc = acc + p;
+                        }
+                    }
+                    out[(size_t)co * vout + ((size_t)z * d + y) * d + x] = relu ? (acc > 0.0f ? acc : 0.0f) : acc;
+                }
+}
+
+void orc_decode_conv(const void *vm, const float *S, uint8_t *occ)
+{
+    const orc_model *m = (const orc_model *)vm;
+    const int D = m->grid, C = m->C;
+    const size_t N = (size_t)D * D * D;
+    float *x0 = (float *)malloc(sizeof(float) * N * C);
+    float *x1 = (float *)malloc(sizeof(float) * N * 16);
+    float *x2 = (float *)malloc(sizeof(float) * N * 8 * 8);
+    float *lg = (float *)malloc(sizeof(float) * N * 64);
+    for (size_t v = 0; v < N; ++v)
+        for (int c = 0; c < C; ++c) x0[(size_t)c * N + v] = S[v * C + c];
+    orc_conv3d(x0, C, D, 1, m->dc1_w, m->dc1_b, 16, 1, x1);
+    orc_conv3d(x1, 16, D, 2, m->dc2_w, m->dc2_b, 8, 1, x2);
+    orc_conv3d(x2, 8, 2 * D, 2, m->dc3_w, m->dc3_b, 1, 0, lg);
+    for (size_t q = 0; q < N * 64; ++q) occ[q] = (uint8_t)(lg[q] > 0.0f);
+    free(x0); free(x1); free(x2); free(lg);
+}
+
 /* ======================================================================== */
 /* Algorithm 1 end to end for B independent samples.                         */
 /* ======================================================================== */
@@ -699,13 +768,15 @@ void orc_dit_forward(const void *vm, const float *S, const int32_t *active_idx, 
  *   names no null condition) and the same active tokens.
  * ssc_accel: 1 scores with the second difference over the last three
  *   velocities (orc_ssc_score3), 0 with the first difference of Sec. 4.1.
+ * decoder: 1 decodes the grids of Eq. 1 with the convolutional stand-in
+ *   (orc_decode_conv, needs G = 64), 0 with the linear one (orc_occupancy).
  */
 int orc_sample(const void *vm, int T, double eta, double rho_a, double rho_off, double mu,
                double omega, double xi, int f_corr, int tau, int refresh_mode,
                float *S, const uint16_t *cond, int B, const double *sigma_override,
                const int32_t *quota_schedule, int32_t *quota_log, int32_t *nact_log,
                double *sigma_out, uint16_t *v_hist_out, int cfg_on, double cfg_s, double cfg_t_lo,
-               int ssc_accel)
+               int ssc_accel, int decoder)
 {
     const orc_model *m = (const orc_model *)vm;
     const int N = m->grid * m->grid * m->grid, C = m->C, G = m->G;
@@ -775,8 +846,13 @@ int orc_sample(const void *vm, int T, double eta, double rho_a, double rho_off, 
             float dt = t[k - 1] - t[k];
             orc_merge_euler(N, C, idx, a, va, vc, dt, Sb, vt);
             if (k == ka) {
-                orc_occupancy(Sold, N, C, m->dec_w, G, occ_a);
-                orc_occupancy(Sb, N, C, m->dec_w, G, occ_b);
+                if (decoder) {
+                    orc_decode_conv(m, Sold, occ_a);
+                    orc_decode_conv(m, Sb, occ_b);
+                } else {
+                    orc_occupancy(Sold, N, C, m->dec_w, G, occ_a);
+                    orc_occupancy(Sb, N, C, m->dec_w, G, occ_b);
+                }
                 double meas = (double)orc_dynamic_voxels(occ_a, occ_b, (long long)N * G);
                 if (sigma_out) sigma_out[b] = meas;
                 if (!sigma_override) sigma = meas;

@@ -77,7 +77,8 @@ def lib():
             L.orc_sample.argtypes = [C.c_void_p, C.c_int, C.c_double, C.c_double, C.c_double,
                                      C.c_double, C.c_double, C.c_double, C.c_int, C.c_int, C.c_int,
                                      _f32p, _u16p, C.c_int, _f64p, _i32p, _i32p, _i32p, _f64p, _u16p,
-                                     C.c_int, C.c_double, C.c_double, C.c_int]
+                                     C.c_int, C.c_double, C.c_double, C.c_int, C.c_int]
+            L.orc_decode_conv.argtypes = [C.c_void_p, _f32p, _u8p]
             L.orc_ssc_score3.argtypes = [_u16p, _u16p, _u16p, C.c_int, C.c_int, C.c_double, _f32p]
             L.orc_cfg_on.argtypes = [C.c_int, C.c_double, C.c_double, C.c_int]
             L.orc_cfg_combine.argtypes = [C.c_longlong, _f32p, _f32p, C.c_double, _f32p]
@@ -275,6 +276,13 @@ class Model:
         lib().orc_modulation(self.h, _p(te, _f32p), block, _p(out, _f32p))
         return out
 
+    def decode_conv(self, S: np.ndarray) -> np.ndarray:
+        """Occupancy of the convolutional stand-in decoder: uint8 [(4D)^3], index (z 4D + y) 4D + x."""
+        S = _f32(S)
+        out = np.empty(self.shape.tokens * 64, np.uint8)
+        lib().orc_decode_conv(self.h, _p(S, _f32p), _p(out, _u8p))
+        return out
+
     def cond_kv(self, cond_bits: np.ndarray) -> np.ndarray:
         s = self.shape
         cb = _u16(cond_bits)
@@ -294,7 +302,7 @@ class Model:
 
     def sample(self, S: np.ndarray, cond_bits: np.ndarray, *, T, eta=3.0, rho_a=0.2, rho_off=0.75,
                mu=-0.07, omega=0.7, xi=0.7, f_corr=3, tau=3, refresh_mode=0,
-               sigma_override=None, quota_schedule=None, cfg=None, cfg_t_lo=0.5, ssc_accel=0):
+               sigma_override=None, quota_schedule=None, cfg=None, cfg_t_lo=0.5, ssc_accel=0, decoder=0):
         """Algorithm 1 for B samples.  Returns dict(S, quota, n_active, sigma, v_hist).
         cfg: guidance strength s (None: unguided) for the steps with t_k >= cfg_t_lo."""
         S = _f32(S).copy()
@@ -313,5 +321,5 @@ class Model:
                          _p(qs, _i32p) if qs is not None else None,
                          _p(ql, _i32p), _p(nl, _i32p), _p(so, _f64p), _p(vh, _u16p),
                          0 if cfg is None else 1, 0.0 if cfg is None else float(cfg), float(cfg_t_lo),
-                         int(ssc_accel))
+                         int(ssc_accel), int(decoder))
         return dict(S=S, quota=ql, n_active=nl, sigma=so, v_hist=vh)

@@ -25,11 +25,12 @@ struct BlockOffsets {
 
 struct Layout {
     size_t in_w, in_b, t_w1, t_b1, t_w2, t_b2, fmod_w, fmod_b, out_w, out_b, dec_w;
+    size_t dc1_w, dc1_b, dc2_w, dc2_b, dc3_w, dc3_b;  // convolutional stand-in decoder
     std::vector<BlockOffsets> blk;
     size_t total;
 };
 
-// Walks the layout-v1 tensor order; each tensor starts on a 64-element
+// Walks the layout-v2 tensor order; each tensor starts on a 64-element
 // boundary.
 Layout weight_layout(const f3dc_config &c)
 {
@@ -76,6 +77,12 @@ Layout weight_layout(const f3dc_config &c)
     L.out_w = take(C * W);
     L.out_b = take(C);
     L.dec_w = take(C * G);
+    L.dc1_w = take(16 * C * 27);
+    L.dc1_b = take(16);
+    L.dc2_w = take(8 * 16 * 27);
+    L.dc2_b = take(8);
+    L.dc3_w = take(8 * 27);
+    L.dc3_b = take(1);
     L.total = pos;
     return L;
 }
@@ -110,8 +117,10 @@ bool config_valid(const f3dc_config *c, std::string &why)
         why = "cfg_strength must be finite and >= 0, cfg_t_lo finite";
     else if (c->cfg_strength > 0.0 && 2 * c->max_batch > kMaxBatch)
         why = "with classifier-free guidance max_batch must be <= 32";
-    else if ((c->ssc_accel != 0 && c->ssc_accel != 1) || c->reserved0 != 0)
-        why = "ssc_accel must be 0 or 1 and reserved0 0";
+    else if (c->ssc_accel != 0 && c->ssc_accel != 1)
+        why = "ssc_accel must be 0 or 1";
+    else if ((c->decoder != 0 && c->decoder != 1) || (c->decoder == 1 && c->gamma_up != 64))
+        why = "decoder must be 0, or 1 with gamma_up 64";
     else
         return true;
     return false;
@@ -701,7 +710,7 @@ f3dc_status f3dc_create(const f3dc_config *cfg, const f3dc_weights *w, void *str
     if (!out) return fail(nullptr, F3DC_ERR_INVALID_ARG, "null out");
     *out = nullptr;
     if (!config_valid(cfg, why)) return fail(nullptr, F3DC_ERR_INVALID_ARG, why);
-    if (!w || w->layout_version != 1 || !w->blob) return fail(nullptr, F3DC_ERR_INVALID_ARG, "weights: need layout_version 1 and a blob");
+    if (!w || w->layout_version != 2 || !w->blob) return fail(nullptr, F3DC_ERR_INVALID_ARG, "weights: need layout_version 2 and a blob");
     const Layout lay = weight_layout(*cfg);
     if (w->blob_elems != lay.total)
         return fail(nullptr, F3DC_ERR_INVALID_ARG,

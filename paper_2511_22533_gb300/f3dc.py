@@ -38,7 +38,7 @@ class Config(C.Structure):
                 ("refresh_mode", C.c_int32), ("eta", C.c_double), ("rho_a", C.c_double), ("mu", C.c_double),
                 ("omega", C.c_double), ("xi", C.c_double), ("rho_cfg_off", C.c_double),
                 ("cfg_strength", C.c_double), ("cfg_t_lo", C.c_double), ("ssc_accel", C.c_int32),
-                ("reserved0", C.c_int32)]
+                ("decoder", C.c_int32)]
 
 
 class KernelStats(C.Structure):
@@ -179,7 +179,7 @@ class Handle:
     def __init__(self, cfg: Config, blob, stream=None):
         self.cfg = cfg
         self.h = C.c_void_p()
-        w = Weights(1, blob.data_ptr(), blob.numel())
+        w = Weights(2, blob.data_ptr(), blob.numel())
         _check(lib().f3dc_create(C.byref(cfg), C.byref(w), _stream(stream), C.byref(self.h)))
 
     def close(self):

@@ -17,7 +17,7 @@ random-init):
                 16 heads, 1374 condition tokens of dim 1024, T = 25.
 * ``scaled``    32^3 x 8 latent (32768 tokens), same transformer, T = 50.
 
-Weight blob (layout version 1): every tensor is bf16, row-major
+Weight blob (layout version 2): every tensor is bf16, row-major
 ``[out_features, in_features]`` for linear layers, concatenated in the order
 returned by :func:`weight_layout`, each tensor starting at a multiple of 64
 elements (128 bytes).
@@ -136,6 +136,11 @@ def weight_layout(shape: ModelShape):
         ("fmod_w", -1, (2 * W, W), "w"), ("fmod_b", -1, (2 * W,), "b"),
         ("out_w", -1, (C, W), "w"), ("out_b", -1, (C,), "b"),
         ("dec_w", -1, (C, G), "dec"),
+        # the convolutional stand-in decoder: 3x3x3 convolutions C -> 16 at
+        # D^3, 16 -> 8 at (2D)^3, 8 -> 1 at (4D)^3, [out, in * 27]
+        ("dc1_w", -1, (16, C * 27), "w"), ("dc1_b", -1, (16,), "b"),
+        ("dc2_w", -1, (8, 16 * 27), "w"), ("dc2_b", -1, (8,), "b"),
+        ("dc3_w", -1, (1, 8 * 27), "w"), ("dc3_b", -1, (1,), "b"),
     ]
     return items
 
@@ -152,7 +157,7 @@ def weight_offsets(shape: ModelShape):
 
 
 def weights_blob(shape: ModelShape, seed: int) -> np.ndarray:
-    """Random-init bf16 weight blob (uint16 bits), layout version 1."""
+    """Random-init bf16 weight blob (uint16 bits), layout version 2."""
     offs, total = weight_offsets(shape)
     blob = np.zeros(total, np.uint16)
     g = _rng(seed + 3)
