@@ -475,6 +475,26 @@ def run_gpu(args):
                 "tensor_tflops_per_gpu": mm_g / (ms_g / 1000.0) / 1e12,
                 "paper_flops_per_sample_T": paper_g / 1e12}
 
+    # ---- the convolutional stand-in decoder of Eq. 1 (secondary): one sample
+    # measuring sigma at the anchor step, the decoder's launches timed
+    hd = f3dc.Handle(f3dc.config_for(shape, 1, decoder=1), blob_d)
+    S.copy_(noise_d)
+    hd.sample(S, cond_d, 1, want_log=False)
+    hd.profile(True)
+    S.copy_(noise_d)
+    _, sig_conv = hd.sample(S, cond_d, 1)
+    dstats = {st["name"]: st for st in hd.profile_read()}
+    hd.profile(False)
+    assert hd.device_status() == 0
+    hd.close()
+    dst = dstats.get("decode_conv")
+    dec_line = None
+    if dst and dst["launches"] > 0:
+        per_decode = dst["total_ms"] / dst["launches"]  # one profiled entry (three kernels) per decode
+        dec_line = {"grid_out": [4 * shape.grid] * 3, "decodes_per_sample": int(dst["launches"]),
+                    "ms_per_decode": per_decode, "gflops": dst["flops"] / (dst["total_ms"] / 1000.0) / 1e9,
+                    "sigma_measured": float(sig_conv[0])}
+
     # ---- the HBM-bound kernels at batch 64 (secondary; not part of `value`)
     hbm64 = hbm_kernels_b64(f3dc, torch, blob_d, pk) if rank == 0 else None
     del blob_d
@@ -533,7 +553,7 @@ def run_gpu(args):
                      "tensor_tflops_per_gpu": mm_unc / (ms_unc / 1000.0) / 1e12},
         "active_tokens_per_step": [shape.tokens - int(c) for c in qlog[:, 0]],
         "sigma_measured_by_stand_in_decoder": float(sigma_meas[0]),
-        "roofline": roof, "kernels": kernels, "hbm_kernels_b64": hbm64, "cfg": cfg_line,
+        "roofline": roof, "kernels": kernels, "hbm_kernels_b64": hbm64, "cfg": cfg_line, "decoder_conv": dec_line,
         "cpu_baseline": cpu,
         "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": int(noise.nbytes + cond_np.nbytes),
                 "d2h_bytes_per_step": int(noise.nbytes)},

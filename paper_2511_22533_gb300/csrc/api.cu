@@ -196,11 +196,12 @@ std::vector<float> position_table(int grid, int W)
 // ---------------------------------------------------------------- profiling
 enum KernelFamily {
     KF_SELECT, KF_GATHER, KF_LN, KF_GEMM, KF_ATTN_SELF, KF_ATTN_CROSS, KF_FINAL, KF_MERGE, KF_TEMB, KF_GEMM_COND,
-    KF_PLAN, KF_SCATTER, KF_COUNT
+    KF_PLAN, KF_SCATTER, KF_DECODE, KF_COUNT
 };
 const char *const kFamilyName[KF_COUNT] = {"ssc_select", "gather_embed", "layernorm",  "gemm",
                                            "attn_self",  "attn_cross",   "final_layer", "merge_euler",
-                                           "temb_gemv",  "gemm_cond",    "plan",        "scatter"};
+                                           "temb_gemv",  "gemm_cond",    "plan",        "scatter",
+                                           "decode_conv"};
 
 // Algorithmic work of one launch as a function of the step's plan:
 //   c_m * M + c_sq * sum_b a_b^2 + c_tok * B N + c_sel * (tokens of samples
@@ -277,6 +278,8 @@ struct f3dc_handle {
     int32_t *gemm_cnt = nullptr;       // split-K per-tile arrival counters (kept at 0)
     cudaStream_t last_stream = nullptr;
     int cond_B = 0;
+    float *dec_scratch = nullptr;  // convolutional decoder (cfg.decoder == 1)
+    uint32_t *dec_bits = nullptr;
     int cfg_B_now = 0;  // guided step in flight: samples >= cfg_B_now are the unguided copies
     // pinned per-step quota slots, two generations so one sampler call can
     // be enqueued while the previous one still copies from its slots
@@ -621,7 +624,7 @@ void free_handle(f3dc_handle *h)
     void *ptrs[] = {h->wblob, h->mod_w, h->mod_b, h->pos, h->x, h->v_active, h->freq, h->h1, h->temb, h->mod,
                     h->h, h->qkv, h->att, h->qc, h->u, h->ckv, h->ring, h->plan, h->tile_sample, h->active_idx,
                     h->row_of_token, h->n_active, h->mask, h->quota_dev, h->dyn, h->dev_err, h->gemm_ws,
-                    h->gemm_cnt};
+                    h->gemm_cnt, h->dec_scratch, h->dec_bits};
     for (void *p : ptrs)
         if (p) cudaFree(p);
     if (h->h_quota) cudaFreeHost(h->h_quota);
@@ -813,6 +816,10 @@ f3dc_status f3dc_create(const f3dc_config *cfg, const f3dc_weights *w, void *str
     CKC(dalloc(&h->mask, (size_t)B * N));
     CKC(dalloc(&h->quota_dev, (size_t)(h->T + 1) * B));
     CKC(dalloc(&h->dyn, (size_t)B));
+    if (cfg->decoder == 1) {
+        CKC(dalloc(&h->dec_scratch, decode_scratch_floats(B, cfg->grid)));
+        CKC(dalloc(&h->dec_bits, (size_t)B * 2 * N));
+    }
     CKC(dalloc(&h->dev_err, 1));
     CKC(cudaMemsetAsync(h->dev_err, 0, sizeof(uint32_t), s));
     CKC(dalloc(&h->gemm_ws, gemm_ws_bytes(256, h->num_sms) / sizeof(float)));
@@ -952,6 +959,31 @@ f3dc_status f3dc_step(f3dc_handle *h, int32_t k, int32_t B, float *S_inout, void
     const uint16_t *v1 = ring + (size_t)((k - 1) % 3) * slot;
     const uint16_t *v2 = ring + (size_t)(((k - 2) % 3 + 3) % 3) * slot;
 
+    // Eq. 1 with the convolutional decoder: the grid before the step, as bits
+    const bool conv_dec = dyn_voxels_dev && h->cfg.decoder == 1;
+    auto decode = [&](int compare) {
+        DecodeArgs d;
+        memset(&d, 0, sizeof(d));
+        d.S = S_inout;
+        d.B = B;
+        d.D = h->cfg.grid;
+        d.w1 = reinterpret_cast<const uint16_t *>(h->wt(h->lay.dc1_w));
+        d.b1 = reinterpret_cast<const uint16_t *>(h->wt(h->lay.dc1_b));
+        d.w2 = reinterpret_cast<const uint16_t *>(h->wt(h->lay.dc2_w));
+        d.b2 = reinterpret_cast<const uint16_t *>(h->wt(h->lay.dc2_b));
+        d.w3 = reinterpret_cast<const uint16_t *>(h->wt(h->lay.dc3_w));
+        d.b3 = reinterpret_cast<const uint16_t *>(h->wt(h->lay.dc3_b));
+        d.scratch = h->dec_scratch;
+        d.bits = h->dec_bits;
+        d.compare = compare;
+        d.dyn = dyn_voxels_dev;
+        d.num_sms = h->num_sms;
+        return launch_decode_conv(d, s);
+    };
+    // (4D)^3 outputs of the last layer plus (2D)^3 x 8 and D^3 x 16 before it
+    const Work w_dec = wfix(2.0 * 27 * (double)h->N * B * (8 * 16 + 64 * 16 * 8 / 8 + 64 * 8), true);
+    if (conv_dec) LAUNCH(KF_DECODE, w_dec, decode(0));
+
     // classifier-free guidance when t_k lies in the CFG interval (Supp. Sec. D)
     std::vector<float> t(h->T + 1);
     time_schedule(h->cfg, t.data());
@@ -1003,7 +1035,7 @@ f3dc_status f3dc_step(f3dc_handle *h, int32_t k, int32_t B, float *S_inout, void
     m.dt = t[k - 1] - t[k];
     m.dec_w = reinterpret_cast<const uint16_t *>(h->wt(h->lay.dec_w));
     m.G = h->G;
-    m.dyn = dyn_voxels_dev;
+    m.dyn = conv_dec ? nullptr : dyn_voxels_dev;  // the linear decoder is fused into the merge
     m.max_rows = h->max_rows;
     m.cfg_s = guided ? (float)h->cfg.cfg_strength : 0.0f;
     m.plan = h->plan;
@@ -1012,6 +1044,7 @@ f3dc_status f3dc_step(f3dc_handle *h, int32_t k, int32_t B, float *S_inout, void
     w_merge.c_tok = 96.0;  // S in/out (32 + 32 B), cached velocity in, v_t out (16 + 16 B)
     w_merge.c_m = 32.0;    // fresh fp32 velocity of each active token
     LAUNCH(KF_MERGE, w_merge, launch_merge_euler(m, s));
+    if (conv_dec) LAUNCH(KF_DECODE, w_dec, decode(1));  // the grid after the step, XOR-counted
     if (h->prof.on) return prof_drain(h, s);
     return F3DC_OK;
 }

@@ -98,6 +98,22 @@ struct MergeArgs {
 };
 cudaError_t launch_merge_euler(const MergeArgs &a, cudaStream_t s);
 
+// Convolutional stand-in decoder of Eq. 1 on B latent grids S [B, D^3, 8]:
+// occupancy bits of the (4D)^3 sub-voxels (2 D^3 words per sample) stored to
+// `bits` (compare = 0) or XOR-counted against them into dyn[b] (compare = 1).
+struct DecodeArgs {
+    const float *S;
+    int B, D;
+    const uint16_t *w1, *b1, *w2, *b2, *w3, *b3;   // bf16 dc1..dc3
+    float *scratch;                                // decode_scratch_floats(B, D)
+    uint32_t *bits;                                // [B, 2 D^3]
+    int compare;
+    int64_t *dyn;                                  // [B] when compare
+    int num_sms;
+};
+size_t decode_scratch_floats(int B, int D);
+cudaError_t launch_decode_conv(const DecodeArgs &a, cudaStream_t s);
+
 // Scatter packed rows back to sample-local positions (diagnostic forward).
 cudaError_t launch_scatter_rows(const float *v_active, const Plan *plan, int B, int N, float *v_out,
                                 cudaStream_t s);
