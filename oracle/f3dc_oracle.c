@@ -17,6 +17,7 @@
  *                                                LayerNorm, cross-attention, MLP)
  *   - cache merge and rectified-flow Euler step (Algorithm 1 step 3; Sec. 3.1)
  *   - dynamic-voxel count                       (Sec. 4.1 Eq. 1)
+ *   - data-driven PCSC slope (RANSAC, median)   (Supp. "Data-driven Parameter Selection")
  *   - classifier-free guidance in its interval  (Sec. 4.3 Phase 3 "CFG-free";
  *                                                Supp. Sec. D CFG interval t in [0.5, 1])
  *   - the whole sampler                         (Algorithm 1)
@@ -749,6 +750,101 @@ void orc_decode_conv(const void *vm, const float *S, uint8_t *occ)
     free(x0); free(x1); free(x2); free(lg);
 }
 
+/* ------------------------------------------------------------------------ */
+/* Data-driven PCSC slope (Supp. "Data-driven Parameter Selection"): per     */
+/* instance, a RANSAC line fit of ln(dS_k) against the step index k over the */
+/* intermediate steps k_lo..k_hi (8..18 in the paper), instances whose fit  */
+/* is poor filtered out, and mu = the median of the remaining slopes.       */
+/* Readings: the hypotheses are every pair of points (exhaustive, so the    */
+/* fit is deterministic); the best pair has the most inliers (|residual| <= */
+/* tol in ln units), ties to the smaller inlier sum of squared residuals,   */
+/* then to the earlier pair; the slope is then the least-squares slope over */
+/* its inliers; steps with dS_k = 0 carry no point; an instance is kept iff */
+/* it has >= 3 points and its inliers are >= min_frac of them; the median of */
+/* an even count is the mean of the middle two.                            */
+/* curves: [n][T] dynamic voxels per 1-based step k at index k - 1.         */
+/* slopes_out / kept_out: nullable [n].  Returns the number kept; mu_out is */
+/* NaN when none is.                                                        */
+/* ------------------------------------------------------------------------ */
+static int orc_cmp_double(const void *a, const void *b)
+{
+    const double x = *(const double *)a, y = *(const double *)b;
+    return (x > y) - (x < y);
+}
+
+int orc_fit_mu(const double *curves, int n, int T, int k_lo, int k_hi, double tol, double min_frac,
+               double *mu_out, double *slopes_out, int *kept_out)
+{
+    double *kept_slopes = (double *)malloc(sizeof(double) * (size_t)(n > 0 ? n : 1));
+    double xs[64], ys[64];
+    int nk = 0;
+    for (int i = 0; i < n; ++i) {
+        int m = 0;
+        for (int k = k_lo; k <= k_hi && k <= T && m < 64; ++k) {
+            const double d = curves[(size_t)i * T + (k - 1)];
+            if (d > 0.0) {
+                xs[m] = (double)k;
+                ys[m] = log(d);
+                ++m;
+            }
+        }
+        double slope = NAN;
+        int keep = 0;
+        if (m >= 3) {
+            int best_cnt = -1;
+            double best_sse = INFINITY;
+            double best_a = 0.0, best_b = 0.0;
+            for (int p = 0; p < m; ++p)
+                for (int q = p + 1; q < m; ++q) {
+                    const double b = (ys[q] - ys[p]) / (xs[q] - xs[p]);
+                    const double a = ys[p] - b * xs[p];
+                    int cnt = 0;
+                    double sse = 0.0;
+                    for (int j = 0; j < m; ++j) {
+                        const double r = ys[j] - (a + b * xs[j]);
+                        if (fabs(r) <= tol) {
+                            ++cnt;
+                            sse += r * r;
+                        }
+                    }
+                    if (cnt > best_cnt || (cnt == best_cnt && sse < best_sse)) {
+                        best_cnt = cnt;
+                        best_sse = sse;
+                        best_a = a;
+                        best_b = b;
+                    }
+                }
+            /* least squares over the best hypothesis' inliers */
+            double sx = 0.0, sy = 0.0, sxx = 0.0, sxy = 0.0;
+            int c = 0;
+            for (int j = 0; j < m; ++j) {
+                const double r = ys[j] - (best_a + best_b * xs[j]);
+                if (fabs(r) <= tol) {
+                    sx += xs[j];
+                    sy += ys[j];
+                    sxx += xs[j] * xs[j];
+                    sxy += xs[j] * ys[j];
+                    ++c;
+                }
+            }
+            const double den = c * sxx - sx * sx;
+            slope = den != 0.0 ? (c * sxy - sx * sy) / den : best_b;
+            keep = (double)best_cnt >= min_frac * (double)m;
+        }
+        if (slopes_out) slopes_out[i] = slope;
+        if (kept_out) kept_out[i] = keep;
+        if (keep) kept_slopes[nk++] = slope;
+    }
+    double mu = NAN;
+    if (nk > 0) {
+        qsort(kept_slopes, (size_t)nk, sizeof(double), orc_cmp_double);
+        mu = (nk % 2) ? kept_slopes[nk / 2] : 0.5 * (kept_slopes[nk / 2 - 1] + kept_slopes[nk / 2]);
+    }
+    if (mu_out) *mu_out = mu;
+    free(kept_slopes);
+    return nk;
+}
+
 /* ======================================================================== */
 /* Algorithm 1 end to end for B independent samples.                         */
 /* ======================================================================== */
@@ -770,13 +866,15 @@ void orc_decode_conv(const void *vm, const float *S, uint8_t *occ)
  *   velocities (orc_ssc_score3), 0 with the first difference of Sec. 4.1.
  * decoder: 1 decodes the grids of Eq. 1 with the convolutional stand-in
  *   (orc_decode_conv, needs G = 64), 0 with the linear one (orc_occupancy).
+ * dyn_log: nullable [T, B]; Eq. 1's dS between the grids before and after
+ *   every step (the curve the PCSC slope is fitted to).
  */
 int orc_sample(const void *vm, int T, double eta, double rho_a, double rho_off, double mu,
                double omega, double xi, int f_corr, int tau, int refresh_mode,
                float *S, const uint16_t *cond, int B, const double *sigma_override,
                const int32_t *quota_schedule, int32_t *quota_log, int32_t *nact_log,
                double *sigma_out, uint16_t *v_hist_out, int cfg_on, double cfg_s, double cfg_t_lo,
-               int ssc_accel, int decoder)
+               int ssc_accel, int decoder, int64_t *dyn_log)
 {
     const orc_model *m = (const orc_model *)vm;
     const int N = m->grid * m->grid * m->grid, C = m->C, G = m->G;
@@ -842,10 +940,10 @@ int orc_sample(const void *vm, int T, double eta, double rho_a, double rho_off, 
                     orc_dit_forward(m, Sb, idx, a, t[k - 1], kv, va);
                 }
             }
-            if (k == ka) memcpy(Sold, Sb, sizeof(float) * NC);
+            if (k == ka || dyn_log) memcpy(Sold, Sb, sizeof(float) * NC);
             float dt = t[k - 1] - t[k];
             orc_merge_euler(N, C, idx, a, va, vc, dt, Sb, vt);
-            if (k == ka) {
+            if (k == ka || dyn_log) {
                 if (decoder) {
                     orc_decode_conv(m, Sold, occ_a);
                     orc_decode_conv(m, Sb, occ_b);
@@ -854,8 +952,11 @@ int orc_sample(const void *vm, int T, double eta, double rho_a, double rho_off, 
                     orc_occupancy(Sb, N, C, m->dec_w, G, occ_b);
                 }
                 double meas = (double)orc_dynamic_voxels(occ_a, occ_b, (long long)N * G);
-                if (sigma_out) sigma_out[b] = meas;
-                if (!sigma_override) sigma = meas;
+                if (dyn_log) dyn_log[(size_t)(k - 1) * B + b] = (int64_t)meas;
+                if (k == ka) {
+                    if (sigma_out) sigma_out[b] = meas;
+                    if (!sigma_override) sigma = meas;
+                }
             }
             /* v(t-3) <- v_prev_cache <- v_cache <- v_t */
             uint16_t *tmp = vpp;

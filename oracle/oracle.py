@@ -77,8 +77,10 @@ def lib():
             L.orc_sample.argtypes = [C.c_void_p, C.c_int, C.c_double, C.c_double, C.c_double,
                                      C.c_double, C.c_double, C.c_double, C.c_int, C.c_int, C.c_int,
                                      _f32p, _u16p, C.c_int, _f64p, _i32p, _i32p, _i32p, _f64p, _u16p,
-                                     C.c_int, C.c_double, C.c_double, C.c_int, C.c_int]
+                                     C.c_int, C.c_double, C.c_double, C.c_int, C.c_int, C.POINTER(C.c_int64)]
             L.orc_decode_conv.argtypes = [C.c_void_p, _f32p, _u8p]
+            L.orc_fit_mu.argtypes = [_f64p, C.c_int, C.c_int, C.c_int, C.c_int, C.c_double, C.c_double,
+                                     _f64p, _f64p, C.POINTER(C.c_int)]
             L.orc_ssc_score3.argtypes = [_u16p, _u16p, _u16p, C.c_int, C.c_int, C.c_double, _f32p]
             L.orc_cfg_on.argtypes = [C.c_int, C.c_double, C.c_double, C.c_int]
             L.orc_cfg_combine.argtypes = [C.c_longlong, _f32p, _f32p, C.c_double, _f32p]
@@ -213,6 +215,18 @@ def dynamic_voxels(occ_a: np.ndarray, occ_b: np.ndarray) -> int:
     return int(lib().orc_dynamic_voxels(_p(a, _u8p), _p(b, _u8p), a.size))
 
 
+def fit_mu(curves, k_lo=8, k_hi=18, tol=0.1, min_frac=0.6):
+    """Data-driven PCSC slope from dynamic-voxel curves [n, T]: returns
+    (mu, slopes [n], kept [n] bool)."""
+    c = np.ascontiguousarray(curves, np.float64)
+    n, T = c.shape
+    mu = C.c_double(0.0)
+    slopes = np.empty(n, np.float64)
+    kept = (C.c_int * max(n, 1))()
+    lib().orc_fit_mu(_p(c, _f64p), n, T, k_lo, k_hi, tol, min_frac, C.byref(mu), _p(slopes, _f64p), kept)
+    return mu.value, slopes, np.array([bool(kept[i]) for i in range(n)])
+
+
 def cfg_on(T: int, eta: float, t_lo: float, k: int) -> bool:
     """Whether step k (1-based) is guided: t_k in the CFG interval [t_lo, 1]."""
     return bool(lib().orc_cfg_on(T, eta, t_lo, k))
@@ -302,7 +316,8 @@ class Model:
 
     def sample(self, S: np.ndarray, cond_bits: np.ndarray, *, T, eta=3.0, rho_a=0.2, rho_off=0.75,
                mu=-0.07, omega=0.7, xi=0.7, f_corr=3, tau=3, refresh_mode=0,
-               sigma_override=None, quota_schedule=None, cfg=None, cfg_t_lo=0.5, ssc_accel=0, decoder=0):
+               sigma_override=None, quota_schedule=None, cfg=None, cfg_t_lo=0.5, ssc_accel=0, decoder=0,
+               want_curve=False):
         """Algorithm 1 for B samples.  Returns dict(S, quota, n_active, sigma, v_hist).
         cfg: guidance strength s (None: unguided) for the steps with t_k >= cfg_t_lo."""
         S = _f32(S).copy()
@@ -315,11 +330,13 @@ class Model:
         vh = np.zeros((2, B, N, self.shape.channels), np.uint16)
         sov = np.ascontiguousarray(sigma_override, np.float64) if sigma_override is not None else None
         qs = np.ascontiguousarray(quota_schedule, np.int32) if quota_schedule is not None else None
+        dl = np.zeros((T, B), np.int64) if want_curve else None
         lib().orc_sample(self.h, T, eta, rho_a, rho_off, mu, omega, xi, f_corr, tau, refresh_mode,
                          _p(S, _f32p), _p(cb, _u16p), B,
                          _p(sov, _f64p) if sov is not None else None,
                          _p(qs, _i32p) if qs is not None else None,
                          _p(ql, _i32p), _p(nl, _i32p), _p(so, _f64p), _p(vh, _u16p),
                          0 if cfg is None else 1, 0.0 if cfg is None else float(cfg), float(cfg_t_lo),
-                         int(ssc_accel), int(decoder))
-        return dict(S=S, quota=ql, n_active=nl, sigma=so, v_hist=vh)
+                         int(ssc_accel), int(decoder),
+                         dl.ctypes.data_as(C.POINTER(C.c_int64)) if dl is not None else None)
+        return dict(S=S, quota=ql, n_active=nl, sigma=so, v_hist=vh, dyn=dl)
