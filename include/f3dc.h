@@ -231,6 +231,30 @@ f3dc_status f3dc_sample(f3dc_handle *h, float *S_inout, const void *cond, int32_
                         const double *sigma_override, const int32_t *quota_schedule,
                         int32_t *quota_log, double *sigma_out, void *stream);
 
+/* The dynamic-voxel curve of Sec. 4.1 (Eq. 1 at every step of a sampler
+ * run without caching -- the curve of the paper's Fig. 2 that the PCSC
+ * slope is fitted to), with the handle's decoder.
+ *   S_inout: device fp32 [B, N, C]: noise in, S_0 out
+ *   cond:    device bf16 [B, N_c, D_c]
+ *   curve_out: host int64 [T, B]: dS_k between the grids before and after
+ *            step k (1-based) at index (k - 1) B + b
+ * Runs the T steps with quota 0 and synchronizes the stream at the end. */
+f3dc_status f3dc_dynamic_voxel_curve(f3dc_handle *h, float *S_inout, const void *cond, int32_t B,
+                                     int64_t *curve_out, void *stream);
+
+/* Data-driven PCSC slope (Supp. "Data-driven Parameter Selection"): for each
+ * of n curves ([n, T] host doubles, dS of 1-based step k at index k - 1), a
+ * RANSAC line fit of ln dS_k against k over steps k_lo..k_hi (the paper uses
+ * 8..18), every pair of points a hypothesis (deterministic), the most
+ * inliers (|residual| <= tol in ln units; ties: smaller inlier sum of
+ * squares, then the earlier pair) refitted by least squares over its
+ * inliers; steps with dS_k = 0 carry no point; a curve is kept iff it has
+ * >= 3 points and inliers >= min_frac of them; *mu_out = the median of the
+ * kept slopes (mean of the middle two for an even count; NaN if none).
+ * slopes_out, kept_out: host [n], nullable.  Host only, pure. */
+f3dc_status f3dc_fit_mu(const double *curves, int32_t n, int32_t T, int32_t k_lo, int32_t k_hi, double tol,
+                        double min_frac, double *mu_out, double *slopes_out, int32_t *kept_out);
+
 /* ---------------------------------------------------------------------- */
 /* Measurement support.                                                    */
 /* ---------------------------------------------------------------------- */

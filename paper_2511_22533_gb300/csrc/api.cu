@@ -2,6 +2,7 @@
 // host-side schedule logic (Supp. Sec. D time shift; Sec. 4.2 PCSC;
 // Algorithm 1 phases and tau refresh), the cached step (Algorithm 1 steps
 // 2-3) and the sampler (Algorithm 1), plus kernel-level diagnostic calls.
+#include <algorithm>
 #include <cmath>
 #include <cstdio>
 #include <cstring>
@@ -278,6 +279,8 @@ struct f3dc_handle {
     int32_t *gemm_cnt = nullptr;       // split-K per-tile arrival counters (kept at 0)
     cudaStream_t last_stream = nullptr;
     int cond_B = 0;
+    int64_t *dyn_curve = nullptr;  // [T, max_batch] for f3dc_dynamic_voxel_curve
+    int32_t *zero_quota = nullptr; // [max_batch] zeros
     float *dec_scratch = nullptr;  // convolutional decoder (cfg.decoder == 1)
     uint32_t *dec_bits = nullptr;
     int cfg_B_now = 0;  // guided step in flight: samples >= cfg_B_now are the unguided copies
@@ -624,7 +627,7 @@ void free_handle(f3dc_handle *h)
     void *ptrs[] = {h->wblob, h->mod_w, h->mod_b, h->pos, h->x, h->v_active, h->freq, h->h1, h->temb, h->mod,
                     h->h, h->qkv, h->att, h->qc, h->u, h->ckv, h->ring, h->plan, h->tile_sample, h->active_idx,
                     h->row_of_token, h->n_active, h->mask, h->quota_dev, h->dyn, h->dev_err, h->gemm_ws,
-                    h->gemm_cnt, h->dec_scratch, h->dec_bits};
+                    h->gemm_cnt, h->dec_scratch, h->dec_bits, h->dyn_curve, h->zero_quota};
     for (void *p : ptrs)
         if (p) cudaFree(p);
     if (h->h_quota) cudaFreeHost(h->h_quota);
@@ -816,6 +819,9 @@ f3dc_status f3dc_create(const f3dc_config *cfg, const f3dc_weights *w, void *str
     CKC(dalloc(&h->mask, (size_t)B * N));
     CKC(dalloc(&h->quota_dev, (size_t)(h->T + 1) * B));
     CKC(dalloc(&h->dyn, (size_t)B));
+    CKC(dalloc(&h->dyn_curve, (size_t)h->T * B));
+    CKC(dalloc(&h->zero_quota, (size_t)B));
+    CKC(cudaMemsetAsync(h->zero_quota, 0, (size_t)B * sizeof(int32_t), s));
     if (cfg->decoder == 1) {
         CKC(dalloc(&h->dec_scratch, decode_scratch_floats(B, cfg->grid)));
         CKC(dalloc(&h->dec_bits, (size_t)B * 2 * N));
@@ -1126,6 +1132,100 @@ f3dc_status f3dc_sample(f3dc_handle *h, float *S_inout, const void *cond, int32_
     }
     CK(cudaEventRecord(h->quota_done[gen], s));
     if (quota_log) CK(cudaStreamSynchronize(s));
+    return F3DC_OK;
+}
+
+f3dc_status f3dc_dynamic_voxel_curve(f3dc_handle *h, float *S_inout, const void *cond, int32_t B,
+                                     int64_t *curve_out, void *stream)
+{
+    if (!h) return fail(nullptr, F3DC_ERR_INVALID_ARG, "null handle");
+    if (!S_inout || !cond || !curve_out) return fail(h, F3DC_ERR_INVALID_ARG, "null pointer");
+    if (B < 1 || B > h->cfg.max_batch) return fail(h, F3DC_ERR_INVALID_ARG, "B outside [1, max_batch]");
+    cudaStream_t s = (cudaStream_t)stream;
+    f3dc_status st = f3dc_set_cond(h, cond, B, stream);
+    if (st != F3DC_OK) return st;
+    CK(cudaMemsetAsync(h->ring, 0, (size_t)3 * B * h->N * kChannels * sizeof(uint16_t), s));
+    CK(cudaMemsetAsync(h->dyn_curve, 0, (size_t)h->T * B * sizeof(int64_t), s));
+    for (int k = 1; k <= h->T; ++k) {
+        st = f3dc_step(h, k, B, S_inout, h->ring, h->zero_quota, h->dyn_curve + (size_t)(k - 1) * B, stream);
+        if (st != F3DC_OK) return st;
+    }
+    CK(cudaMemcpyAsync(curve_out, h->dyn_curve, (size_t)h->T * B * sizeof(int64_t), cudaMemcpyDeviceToHost, s));
+    CK(cudaStreamSynchronize(s));
+    h->last_stream = s;
+    return F3DC_OK;
+}
+
+f3dc_status f3dc_fit_mu(const double *curves, int32_t n, int32_t T, int32_t k_lo, int32_t k_hi, double tol,
+                        double min_frac, double *mu_out, double *slopes_out, int32_t *kept_out)
+{
+    if (!curves || !mu_out || n < 0 || T < 1 || k_lo < 1 || k_hi < k_lo || !(tol >= 0.0) ||
+        !(min_frac >= 0.0 && min_frac <= 1.0))
+        return fail(nullptr, F3DC_ERR_INVALID_ARG, "fit_mu: bad arguments");
+    std::vector<double> kept_slopes;
+    for (int i = 0; i < n; ++i) {
+        // the window's points (k, ln dS_k), zero counts left out
+        std::vector<double> x, y;
+        for (int k = k_lo; k <= k_hi && k <= T; ++k) {
+            const double d = curves[(size_t)i * T + (k - 1)];
+            if (d > 0.0) {
+                x.push_back((double)k);
+                y.push_back(std::log(d));
+            }
+        }
+        const int m = (int)x.size();
+        double slope = std::nan("");
+        bool keep = false;
+        if (m >= 3) {
+            // exhaustive hypotheses: the line through every pair of points
+            int best_in = -1;
+            double best_sse = INFINITY, ba = 0.0, bb = 0.0;
+            for (int p = 0; p < m; ++p)
+                for (int q = p + 1; q < m; ++q) {
+                    const double b = (y[q] - y[p]) / (x[q] - x[p]);
+                    const double a = y[p] - b * x[p];
+                    int in = 0;
+                    double sse = 0.0;
+                    for (int j = 0; j < m; ++j) {
+                        const double r = y[j] - (a + b * x[j]);
+                        if (std::fabs(r) <= tol) {
+                            ++in;
+                            sse += r * r;
+                        }
+                    }
+                    if (in > best_in || (in == best_in && sse < best_sse)) {
+                        best_in = in;
+                        best_sse = sse;
+                        ba = a;
+                        bb = b;
+                    }
+                }
+            // least-squares slope over the winning line's inliers
+            double sx = 0.0, sy = 0.0, sxx = 0.0, sxy = 0.0;
+            int c = 0;
+            for (int j = 0; j < m; ++j)
+                if (std::fabs(y[j] - (ba + bb * x[j])) <= tol) {
+                    sx += x[j];
+                    sy += y[j];
+                    sxx += x[j] * x[j];
+                    sxy += x[j] * y[j];
+                    ++c;
+                }
+            const double den = c * sxx - sx * sx;
+            slope = den != 0.0 ? (c * sxy - sx * sy) / den : bb;
+            keep = (double)best_in >= min_frac * (double)m;
+        }
+        if (slopes_out) slopes_out[i] = slope;
+        if (kept_out) kept_out[i] = keep ? 1 : 0;
+        if (keep) kept_slopes.push_back(slope);
+    }
+    double mu = std::nan("");
+    if (!kept_slopes.empty()) {
+        std::sort(kept_slopes.begin(), kept_slopes.end());
+        const size_t c = kept_slopes.size();
+        mu = (c % 2) ? kept_slopes[c / 2] : 0.5 * (kept_slopes[c / 2 - 1] + kept_slopes[c / 2]);
+    }
+    *mu_out = mu;
     return F3DC_OK;
 }
 

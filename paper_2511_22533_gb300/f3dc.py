@@ -83,6 +83,9 @@ def lib():
                 "f3dc_set_cond": ([_vp, _vp, C.c_int32, _vp], C.c_int),
                 "f3dc_step": ([_vp, C.c_int32, C.c_int32, _vp, _vp, _vp, _vp, _vp], C.c_int),
                 "f3dc_sample": ([_vp, _vp, _vp, C.c_int32, _f64p, _i32p, _i32p, _f64p, _vp], C.c_int),
+                "f3dc_dynamic_voxel_curve": ([_vp, _vp, _vp, C.c_int32, C.POINTER(C.c_int64), _vp], C.c_int),
+                "f3dc_fit_mu": ([_f64p, C.c_int32, C.c_int32, C.c_int32, C.c_int32, C.c_double, C.c_double,
+                                 _f64p, _f64p, _i32p], C.c_int),
                 "f3dc_forward": ([_vp, C.c_float, C.c_int32, _vp, _vp, _vp, _vp, _vp], C.c_int),
                 "f3dc_profile": ([_vp, C.c_int32], C.c_int),
                 "f3dc_profile_read": ([_vp, C.POINTER(KernelStats), C.c_int32, _i32p], C.c_int),
@@ -226,6 +229,13 @@ class Handle:
                                    _np_ptr(ql, _i32p), _np_ptr(sg, _f64p), _stream(stream)))
         return ql, sg
 
+    def dynamic_voxel_curve(self, S, cond, B, stream=None) -> np.ndarray:
+        """Eq. 1's dS at every step of an uncached sampler run: int64 [T, B]."""
+        out = np.zeros((self.cfg.steps, B), np.int64)
+        self._ck(lib().f3dc_dynamic_voxel_curve(self.h, _ptr(S), _ptr(cond), B,
+                                                out.ctypes.data_as(C.POINTER(C.c_int64)), _stream(stream)))
+        return out
+
     def profile(self, enable: bool):
         self._ck(lib().f3dc_profile(self.h, 1 if enable else 0))
 
@@ -250,6 +260,18 @@ class Handle:
 
 
 # ---------------------------------------------------------------- kernels
+
+def fit_mu(curves, k_lo=8, k_hi=18, tol=0.1, min_frac=0.6):
+    """Data-driven PCSC slope from dS curves [n, T]: (mu, slopes [n], kept [n] bool)."""
+    c = np.ascontiguousarray(curves, np.float64)
+    n, T = c.shape
+    mu = C.c_double(0.0)
+    slopes = np.empty(n, np.float64)
+    kept = np.empty(n, np.int32)
+    _check(lib().f3dc_fit_mu(c.ctypes.data_as(_f64p), n, T, k_lo, k_hi, tol, min_frac, C.byref(mu),
+                             slopes.ctypes.data_as(_f64p), kept.ctypes.data_as(_i32p)))
+    return mu.value, slopes, kept.astype(bool)
+
 
 def gemm(A, Bw, bias, gate, out, M, N, K, epilogue, stream=None):
     _check(lib().f3dc_gemm(_ptr(A), _ptr(Bw), _ptr(bias), _ptr(gate), _ptr(out), M, N, K, epilogue,

@@ -76,3 +76,30 @@ def test_invalid_arguments_are_reported(L):
     st = L.f3dc_create(C.byref(bad), None, None, C.byref(h))
     assert st == 1 and not h
     assert b"channels" in L.f3dc_last_error(None)
+
+
+def test_fit_mu_matches_oracle(orc):
+    # the library's data-driven slope fit (host only) and the oracle's, on
+    # log-linear curves with noise, gross outliers, zero counts and hopeless
+    # instances
+    rng = np.random.default_rng(3)
+    T = 25
+    k = np.arange(1, T + 1, dtype=np.float64)
+    curves = []
+    for i in range(40):
+        slope = rng.uniform(-0.3, -0.01)
+        y = rng.uniform(6, 11) + slope * (k - 8) + rng.normal(0, rng.choice([0.005, 0.05, 1.0]), T)
+        d = np.exp(y)
+        for _ in range(rng.integers(0, 3)):
+            d[rng.integers(7, 18)] *= np.exp(rng.choice([-3.0, 2.5]))
+        if i % 7 == 0:
+            d[rng.integers(7, 18)] = 0.0
+        curves.append(np.round(d))
+    curves = np.stack(curves)
+    for tol, frac in ((0.1, 0.6), (0.05, 0.8), (0.3, 0.5)):
+        mu_l, sl_l, kept_l = f3dc.fit_mu(curves, tol=tol, min_frac=frac)
+        mu_o, sl_o, kept_o = orc.fit_mu(curves, tol=tol, min_frac=frac)
+        np.testing.assert_array_equal(kept_l, kept_o)
+        np.testing.assert_allclose(sl_l, sl_o, rtol=0, atol=1e-12)
+        assert abs(mu_l - mu_o) < 1e-12
+        assert 0 < kept_l.sum() < len(curves)

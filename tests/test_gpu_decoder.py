@@ -55,3 +55,23 @@ def test_sampler_sigma_with_conv_decoder(orc):
     assert np.all(np.abs(sigma - out["sigma"]) <= 0.02 * np.maximum(out["sigma"], 50)), (sigma, out["sigma"])
     assert_clean(h)
     h.close()
+
+
+@pytest.mark.parametrize("decoder", [0, 1])
+def test_dynamic_voxel_curve_against_oracle(orc, decoder):
+    # Eq. 1 at every step of an uncached run (the curve the PCSC slope is
+    # fitted to): both sides decode nearly the same latents at every step
+    shape = synth.SHAPES["tiny"]
+    B = 2
+    h, blob, _ = handle_for(shape, max_batch=B, decoder=decoder)
+    m = orc.Model(shape, blob)
+    cond = synth.cond_tokens(shape, B, 1)
+    S = synth.latents(shape, B, 1)
+    curve = h.dynamic_voxel_curve(dev_f32(S), dev_u16(cond), B)
+    T = shape.steps
+    out = m.sample(S, cond, T=T, quota_schedule=np.zeros((T, B), np.int32), tau=0, decoder=decoder, want_curve=True)
+    ref = out["dyn"]
+    assert curve.shape == (T, B) and np.all(curve >= 0)
+    assert np.all(np.abs(curve - ref) <= 0.02 * np.maximum(ref, 50)), (curve, ref)
+    assert_clean(h)
+    h.close()
