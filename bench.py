@@ -495,6 +495,16 @@ def run_gpu(args):
                     "ms_per_decode": per_decode, "gflops": dst["flops"] / (dst["total_ms"] / 1000.0) / 1e9,
                     "sigma_measured": float(sig_conv[0])}
 
+    # ---- data-driven PCSC slope (secondary): the dynamic-voxel curve of one
+    # uncached run with the linear stand-in decoder, fitted over steps 8..18
+    torch.cuda.synchronize()
+    t0 = time.perf_counter()
+    curve = h.dynamic_voxel_curve(S.copy_(noise_d), cond_d, 1)
+    curve_ms = (time.perf_counter() - t0) * 1000.0
+    mu_fit, _, kept_fit = f3dc.fit_mu(curve.T.astype(np.float64))
+    mu_line = {"curve_ms": curve_ms, "curve": [int(x) for x in curve[:, 0]], "steps_fitted": [8, 18],
+               "mu": None if not np.isfinite(mu_fit) else float(mu_fit), "kept": bool(kept_fit[0])}
+
     # ---- the HBM-bound kernels at batch 64 (secondary; not part of `value`)
     hbm64 = hbm_kernels_b64(f3dc, torch, blob_d, pk) if rank == 0 else None
     del blob_d
@@ -553,7 +563,7 @@ def run_gpu(args):
                      "tensor_tflops_per_gpu": mm_unc / (ms_unc / 1000.0) / 1e12},
         "active_tokens_per_step": [shape.tokens - int(c) for c in qlog[:, 0]],
         "sigma_measured_by_stand_in_decoder": float(sigma_meas[0]),
-        "roofline": roof, "kernels": kernels, "hbm_kernels_b64": hbm64, "cfg": cfg_line, "decoder_conv": dec_line,
+        "roofline": roof, "kernels": kernels, "hbm_kernels_b64": hbm64, "cfg": cfg_line, "decoder_conv": dec_line, "mu_fit": mu_line,
         "cpu_baseline": cpu,
         "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": int(noise.nbytes + cond_np.nbytes),
                 "d2h_bytes_per_step": int(noise.nbytes)},
