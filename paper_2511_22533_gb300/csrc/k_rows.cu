@@ -146,9 +146,10 @@ F3DC_DEV void row_stats(const float4 (&v)[NV], int W, float &mean, float &rstd)
 
 // One warp per row, lane l owning float4 columns q * 32 + l.  The per-column
 // modulation (adaLN scale / shift, or LN gain / bias) is staged in shared
-// memory once per CTA, and each warp loads its next row while it normalises
-// the current one, so the kernel streams rows at a persistent grid of two
-// CTAs per SM instead of paying two dependent memory round trips per row.
+// memory once per CTA while the first row is in flight, and each warp loads
+// its next row while it normalises the current one, so the kernel streams
+// rows at a persistent grid of two CTAs per SM instead of paying two
+// dependent memory round trips per row.
 template <int NV>
 __global__ void __launch_bounds__(kRowThreads, 2) k_layernorm(const float *x, int W, const Plan *plan, int mode,
                                                               const float *shift, const float *scale,
@@ -162,6 +163,13 @@ __global__ void __launch_bounds__(kRowThreads, 2) k_layernorm(const float *x, in
     const int stride = gridDim.x * wpb;
     int r = blockIdx.x * wpb + (threadIdx.x >> 5);
     if (blockIdx.x * wpb >= m_rows) return;  // the whole CTA is idle
+    // the first row's loads are issued before the modulation is staged, so
+    // the two memory round trips overlap
+    float4 v[NV];
+    if (r < m_rows) {
+#pragma unroll
+        for (int q = 0; q < NV; ++q) v[q] = ld_f4(x + (size_t)r * W + 4 * (q * 32 + lane));
+    }
     for (int c4 = threadIdx.x; c4 < NV * 32; c4 += blockDim.x) {
         const int n0 = 4 * c4;
         if (mode == 0) {
@@ -179,9 +187,6 @@ __global__ void __launch_bounds__(kRowThreads, 2) k_layernorm(const float *x, in
     }
     __syncthreads();
     if (r >= m_rows) return;
-    float4 v[NV];
-#pragma unroll
-    for (int q = 0; q < NV; ++q) v[q] = ld_f4(x + (size_t)r * W + 4 * (q * 32 + lane));
     for (;;) {
         const int rn = r + stride;
         float4 vn[NV];
