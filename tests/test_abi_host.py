@@ -103,3 +103,38 @@ def test_fit_mu_matches_oracle(orc):
         np.testing.assert_allclose(sl_l, sl_o, rtol=0, atol=1e-12)
         assert abs(mu_l - mu_o) < 1e-12
         assert 0 < kept_l.sum() < len(curves)
+
+
+@pytest.mark.parametrize("field,value,needle", [
+    ("cfg_strength", -1.0, b"cfg_strength"),
+    ("cfg_strength", float("inf"), b"cfg_strength"),
+    ("ssc_accel", 2, b"ssc_accel"),
+    ("decoder", 3, b"decoder"),
+    ("width", 384, b"width"),
+])
+def test_new_config_fields_are_validated(L, field, value, needle):
+    bad = f3dc.config_for(synth.SHAPES["tiny"], **{field: value})
+    assert f3dc.weights_elems(bad) == 0
+    h = C.c_void_p()
+    assert L.f3dc_create(C.byref(bad), None, None, C.byref(h)) == 1 and not h
+    assert needle in L.f3dc_last_error(None)
+
+
+def test_guidance_and_decoder_constraints(L):
+    # guidance runs 2B samples in one plan (B <= 32); the convolutional
+    # decoder yields 64 sub-voxels per token
+    ok = f3dc.config_for(synth.SHAPES["tiny"], 32, cfg_strength=2.0)
+    assert f3dc.weights_elems(ok) > 0
+    bad = f3dc.config_for(synth.SHAPES["tiny"], 33, cfg_strength=2.0)
+    assert f3dc.weights_elems(bad) == 0
+    bad = f3dc.config_for(synth.ModelShape(8, 8, 128, 2, 4, 4, 64, 128, 8, 8), decoder=1)
+    assert f3dc.weights_elems(bad) == 0
+    d = f3dc.default_config()
+    assert d.cfg_strength == 0.0 and d.cfg_t_lo == 0.5 and d.ssc_accel == 0 and d.decoder == 0
+
+
+def test_fit_mu_rejects_bad_arguments(L):
+    with pytest.raises(f3dc.F3dcError):
+        f3dc.fit_mu(np.ones((2, 25)), k_lo=10, k_hi=5)
+    with pytest.raises(f3dc.F3dcError):
+        f3dc.fit_mu(np.ones((2, 25)), min_frac=1.5)
