@@ -135,6 +135,14 @@ F3DC_DEV void tma_load_2d(void *smem_dst, const CUtensorMap *map, int x, int y, 
         : "memory");
 }
 
+// Pulls one box of a tiled tensor into L2 (no shared memory, no completion).
+F3DC_DEV void tma_prefetch_l2_2d(const CUtensorMap *map, int x, int y)
+{
+    asm volatile("cp.async.bulk.prefetch.tensor.2d.L2.global.tile [%0, {%1, %2}];" ::"l"((uint64_t)map), "r"(x),
+                 "r"(y)
+                 : "memory");
+}
+
 // Tiled TMA store of a shared-memory box to global memory (bulk-group
 // completion), and the same as an element-wise fp32 add into global memory.
 // Coordinates: x = innermost (column), y = row; the box is clipped at the

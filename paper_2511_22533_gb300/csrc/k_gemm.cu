@@ -600,6 +600,13 @@ __global__ void __launch_bounds__(kPairThreads, 1)
         tmem_alloc_pair(tmem_holder, kPairTmemCols);
         tmem_relinquish_pair();
     }
+    if (warp == 0 && lane == 0) {
+        // the weights are constant: pull this CTA's share of B into L2 while
+        // the previous kernel finishes, so the first stages' loads hit L2
+        const int kbx = p.K / 64, boxes = (p.N / (int)kGemmPairBBox) * kbx;
+        for (int i = blockIdx.x; i < boxes; i += gridDim.x)
+            tma_prefetch_l2_2d(&tmb, (i % kbx) * 64, (i / kbx) * (int)kGemmPairBBox);
+    }
     tc_fence_before();
     __syncthreads();
     cluster_sync();  // both CTAs' barriers are initialised before any remote signal
