@@ -472,6 +472,7 @@ cudaError_t run_attention(f3dc_handle *h, int mode, const CUtensorMap &tq, const
     p.nk_fixed = h->Nc;
     p.kv_null_from = mode == 1 ? h->cfg_B_now : 0;
     p.kv_null_sample = h->cfg.max_batch;
+    p.kv_prefetch_rows = mode == 1 ? h->cond_B * h->Nc : 0;  // the condition's K / V
     p.out = h->att;
     p.ldo = h->W;
     p.scale_log2 = (float)(1.4426950408889634 / std::sqrt((double)h->dh));

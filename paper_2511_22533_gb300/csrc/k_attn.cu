@@ -153,6 +153,15 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
         tmem_alloc(tmem_holder, Cfg::kTmemCols);
         tmem_relinquish();
     }
+    if (p.kv_prefetch_rows > 0 && warp == 0 && lane == 0) {
+        // keys / values written long before this launch (the condition's):
+        // pull this CTA's share into L2 while the previous kernel finishes
+        const int rb = (p.kv_prefetch_rows + 127) / 128, boxes = rb * p.heads * 2;
+        for (int i = blockIdx.x; i < boxes; i += gridDim.x) {
+            const int r = i % rb, hk = i / rb, h = hk >> 1;
+            tma_prefetch_l2_2d(hk & 1 ? &tmv : &tmk, (hk & 1 ? p.v_col0 : p.k_col0) + h * DH, r * 128);
+        }
+    }
     tc_fence_before();
     __syncthreads();
     tc_fence_after();

@@ -378,8 +378,11 @@ F3DC_DEV float silu(float v) { return v / (1.0f + expf(-v)); }
 constexpr int kGemvThreads = 512;
 constexpr int kGemvMaxK = 4096;
 
-__global__ void __launch_bounds__(kGemvThreads) k_gemv(const float *x, int K, const bf16 *w, const bf16 *bias,
-                                                       float *y, int rows, int silu_in, int silu_out)
+// One warp per pair of weight rows; each lane streams uint4 chunks of both
+// rows, four chunks per row issued before any is used (K = 1024: the whole
+// row pair in one round of loads), two CTAs of 16 warps per SM.
+__global__ void __launch_bounds__(kGemvThreads, 2) k_gemv(const float *x, int K, const bf16 *w, const bf16 *bias,
+                                                          float *y, int rows, int silu_in, int silu_out)
 {
     griddep_launch();
     griddep_wait();
@@ -392,17 +395,27 @@ __global__ void __launch_bounds__(kGemvThreads) k_gemv(const float *x, int K, co
     for (int r = (blockIdx.x * wpb + (threadIdx.x >> 5)) * 2; r < rows; r += gridDim.x * wpb * 2) {
         const bool two = r + 1 < rows;
         float acc0 = 0.f, acc1 = 0.f;
-        for (int q = lane; q < chunks; q += 32) {
-            const int k0 = q * 8;
-            const uint4 u0 = __ldg(W4 + ((size_t)r * K + k0) / 8);
-            const uint4 u1 = two ? __ldg(W4 + ((size_t)(r + 1) * K + k0) / 8) : make_uint4(0, 0, 0, 0);
-            float f0[8], f1[8];
-            bf16x8_to_f32(u0, f0);
-            bf16x8_to_f32(u1, f1);
+        for (int q0 = lane; q0 < chunks; q0 += 4 * 32) {
+            uint4 u0[4], u1[4];
 #pragma unroll
-            for (int j = 0; j < 8; ++j) {
-                acc0 = fmaf(f0[j], xs[k0 + j], acc0);
-                acc1 = fmaf(f1[j], xs[k0 + j], acc1);
+            for (int c = 0; c < 4; ++c) {
+                const int q = q0 + c * 32;
+                u0[c] = q < chunks ? __ldg(W4 + (size_t)r * (K / 8) + q) : make_uint4(0, 0, 0, 0);
+                u1[c] = two && q < chunks ? __ldg(W4 + (size_t)(r + 1) * (K / 8) + q) : make_uint4(0, 0, 0, 0);
+            }
+#pragma unroll
+            for (int c = 0; c < 4; ++c) {
+                const int q = q0 + c * 32;
+                if (q >= chunks) break;
+                const int k0 = q * 8;
+                float f0[8], f1[8];
+                bf16x8_to_f32(u0[c], f0);
+                bf16x8_to_f32(u1[c], f1);
+#pragma unroll
+                for (int j = 0; j < 8; ++j) {
+                    acc0 = fmaf(f0[j], xs[k0 + j], acc0);
+                    acc1 = fmaf(f1[j], xs[k0 + j], acc1);
+                }
             }
         }
         acc0 = warp_sum(acc0);
@@ -542,7 +555,7 @@ cudaError_t launch_gemv(const float *x, int K, const bf16 *w, const bf16 *b, flo
     if (K % 8 != 0 || K > kGemvMaxK) return cudaErrorInvalidValue;
     const int wpb = kGemvThreads / 32;
     int grid = (rows + 2 * wpb - 1) / (2 * wpb);
-    if (grid > num_sms * 4) grid = num_sms * 4;
+    if (grid > num_sms * 2) grid = num_sms * 2;
     launch_k(k_gemv, dim3(grid), dim3(kGemvThreads), 0, s, x, K, w, b, y, rows, silu_in, silu_out);
     return cudaGetLastError();
 }

@@ -231,6 +231,9 @@ struct AttnParams {
     // mode 1: samples b >= kv_null_from (0: none) attend to the keys of
     // sample slot kv_null_sample (the zero condition of a guided step)
     int kv_null_from, kv_null_sample;
+    // > 0: K / V rows [0, kv_prefetch_rows) are complete before the launch
+    // (not written by the previous kernel) and are prefetched into L2 first
+    int kv_prefetch_rows;
     uint32_t *err;
 };
 cudaError_t launch_attention(const CUtensorMap *tq, const CUtensorMap *tk, const CUtensorMap *tv,
