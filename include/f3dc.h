@@ -199,16 +199,19 @@ f3dc_status f3dc_set_cond(f3dc_handle *h, const void *cond, int32_t B, void *str
 
 /* One cached denoising step k (1-based) in place (Algorithm 1, steps 2-3):
  * SSC selection under quota_dev, the flow transformer at t_k on the active
- * tokens (condition from the last f3dc_set_cond), cache merge, Euler update
- * S <- S - (t_k - t_{k+1}) v_t.
+ * tokens (condition from the last f3dc_set_cond; with cfg_strength > 0 and
+ * t_k >= cfg_t_lo also for the zero condition, guided velocity), cache
+ * merge, Euler update S <- S - (t_k - t_{k+1}) v_t.
  *   S_inout: device fp32 [B, N, C]
  *   v_ring:  device bf16 [3, B, N, C] velocity history; slot k % 3 receives
- *            v_t, slots (k-1) % 3 and (k-2) % 3 hold v^(k-1), v^(k-2).  Zero
- *            it before step 1 (Algorithm 1 initialises v_cache to 0).
+ *            v_t, slots (k-1) % 3 and (k-2) % 3 hold v^(k-1), v^(k-2), and
+ *            slot k % 3 still holds v^(k-3) when the selection reads it
+ *            (ssc_accel = 1).  Zero it before step 1 (Algorithm 1
+ *            initialises v_cache to 0).
  *   quota_dev: device int32 [B] tokens to cache (apply tau beforehand).
  *   dyn_voxels_dev: nullable device int64 [B]; when given, the step also
- *            counts the dynamic voxels (Eq. 1) between the decoded grids
- *            before and after the update and ADDS them there.
+ *            counts the dynamic voxels (Eq. 1) between the grids decoded
+ *            (cfg.decoder) before and after the update and ADDS them there.
  * Asynchronous on `stream`. */
 f3dc_status f3dc_step(f3dc_handle *h, int32_t k, int32_t B, float *S_inout, void *v_ring,
                       const int32_t *quota_dev, int64_t *dyn_voxels_dev, void *stream);
