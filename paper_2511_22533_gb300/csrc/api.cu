@@ -264,6 +264,11 @@ struct f3dc_handle {
 
     bf16 *wblob = nullptr, *mod_w = nullptr, *mod_b = nullptr;
     int mod_rows = 0;
+    // every step's time embedding and modulation, computed at the start of
+    // f3dc_sample (one pass over the modulation weights per sample instead
+    // of one per step); mod_pre marks a sample in progress
+    float *t_all = nullptr, *freq_all = nullptr, *h1_all = nullptr, *temb_all = nullptr, *mod_all = nullptr;
+    bool mod_pre = false;
     float *pos = nullptr;
 
     float *x = nullptr, *v_active = nullptr, *freq = nullptr, *h1 = nullptr, *temb = nullptr, *mod = nullptr;
@@ -484,7 +489,9 @@ cudaError_t run_attention(f3dc_handle *h, int mode, const CUtensorMap &tq, const
 
 // The flow transformer on the packed active rows described by h->plan,
 // h->tile_sample and h->active_idx (Sec. 4.2; Supp. Sec. F).
-f3dc_status run_dit(f3dc_handle *h, float t, const float *S, cudaStream_t s)
+// mod_pre: nullable; this step's modulation vectors, computed beforehand
+// (f3dc_sample computes every step's at its start)
+f3dc_status run_dit(f3dc_handle *h, float t, const float *S, cudaStream_t s, const float *mod_pre = nullptr)
 {
     const int W = h->W, L = h->L, Wm = h->Wm;
     const double dW = W, dWm = Wm;
@@ -492,10 +499,14 @@ f3dc_status run_dit(f3dc_handle *h, float t, const float *S, cudaStream_t s)
     // timestep embedding and every block's modulation (adaLN): three GEMVs
     // streaming the embedding and the repacked [L*6W + 2W, W] weights
     const Work w_temb = wfix(2.0 * ((double)h->mod_rows * W + 256.0 * W + dW * W));
-    LAUNCH(KF_TEMB, Work(), launch_time_freq(t, h->freq, s));
-    LAUNCH(KF_TEMB, Work(), launch_gemv(h->freq, 256, h->wt(ly.t_w1), h->wt(ly.t_b1), h->h1, W, 0, 1, h->num_sms, s));
-    LAUNCH(KF_TEMB, Work(), launch_gemv(h->h1, W, h->wt(ly.t_w2), h->wt(ly.t_b2), h->temb, W, 0, 0, h->num_sms, s));
-    LAUNCH(KF_TEMB, w_temb, launch_gemv(h->temb, W, h->mod_w, h->mod_b, h->mod, h->mod_rows, 1, 0, h->num_sms, s));
+    const float *mod = mod_pre;
+    if (!mod) {
+        LAUNCH(KF_TEMB, Work(), launch_time_freq(t, h->freq, s));
+        LAUNCH(KF_TEMB, Work(), launch_gemv(h->freq, 256, h->wt(ly.t_w1), h->wt(ly.t_b1), h->h1, W, 0, 1, h->num_sms, s));
+        LAUNCH(KF_TEMB, Work(), launch_gemv(h->h1, W, h->wt(ly.t_w2), h->wt(ly.t_b2), h->temb, W, 0, 0, h->num_sms, s));
+        LAUNCH(KF_TEMB, w_temb, launch_gemv(h->temb, W, h->mod_w, h->mod_b, h->mod, h->mod_rows, 1, 0, h->num_sms, s));
+        mod = h->mod;
+    }
     // gather + embed the active tokens: 32 B latent + 4 B index in, 4W B out
     LAUNCH(KF_GATHER, wm(36.0 + 4.0 * dW),
            launch_gather_embed(S, h->N, W, h->active_idx, h->plan, h->tile_sample, h->wt(ly.in_w), h->wt(ly.in_b),
@@ -507,7 +518,7 @@ f3dc_status run_dit(f3dc_handle *h, float t, const float *S, cudaStream_t s)
     const Work w_cross = wm(4.0 * dW * h->Nc, true);
     for (int l = 0; l < L; ++l) {
         const BlockOffsets &b = ly.blk[l];
-        const float *m = h->mod + (size_t)l * 6 * W;
+        const float *m = mod + (size_t)l * 6 * W;
         // self-attention among the active tokens
         LAUNCH(KF_LN, w_ln, launch_layernorm(h->x, W, h->plan, 0, m, m + W, nullptr, nullptr, h->h, h->max_rows,
                                              h->num_sms, s));
@@ -538,7 +549,7 @@ f3dc_status run_dit(f3dc_handle *h, float t, const float *S, cudaStream_t s)
                run_gemm(h, h->tm_u, h->tm_fc2_w[l], W, Wm, h->bn_w, kEpiResid, h->x, W, h->wt(b.fc2_b), m + 5 * W,
                         nullptr, nullptr, s));
     }
-    const float *fm = h->mod + (size_t)L * 6 * W;
+    const float *fm = mod + (size_t)L * 6 * W;
     LAUNCH(KF_FINAL, wm(4.0 * dW + 32.0), launch_final_layer(h->x, W, h->plan, fm, fm + W, h->wt(ly.out_w),
                                                              h->wt(ly.out_b), h->v_active, h->max_rows, h->num_sms, s));
     return F3DC_OK;
@@ -628,7 +639,8 @@ void free_handle(f3dc_handle *h)
     void *ptrs[] = {h->wblob, h->mod_w, h->mod_b, h->pos, h->x, h->v_active, h->freq, h->h1, h->temb, h->mod,
                     h->h, h->qkv, h->att, h->qc, h->u, h->ckv, h->ring, h->plan, h->tile_sample, h->active_idx,
                     h->row_of_token, h->n_active, h->mask, h->quota_dev, h->dyn, h->dev_err, h->gemm_ws,
-                    h->gemm_cnt, h->dec_scratch, h->dec_bits, h->dyn_curve, h->zero_quota};
+                    h->gemm_cnt, h->dec_scratch, h->dec_bits, h->dyn_curve, h->zero_quota, h->t_all,
+                    h->freq_all, h->h1_all, h->temb_all, h->mod_all};
     for (void *p : ptrs)
         if (p) cudaFree(p);
     if (h->h_quota) cudaFreeHost(h->h_quota);
@@ -810,6 +822,16 @@ f3dc_status f3dc_create(const f3dc_config *cfg, const f3dc_weights *w, void *str
     CKC(dalloc(&h->h1, W));
     CKC(dalloc(&h->temb, W));
     CKC(dalloc(&h->mod, (size_t)h->mod_rows));
+    CKC(dalloc(&h->t_all, (size_t)h->T));
+    CKC(dalloc(&h->freq_all, (size_t)h->T * 256));
+    CKC(dalloc(&h->h1_all, (size_t)h->T * W));
+    CKC(dalloc(&h->temb_all, (size_t)h->T * W));
+    CKC(dalloc(&h->mod_all, (size_t)h->T * h->mod_rows));
+    {
+        std::vector<float> tt(h->T + 1);
+        time_schedule(*cfg, tt.data());
+        CKC(cudaMemcpy(h->t_all, tt.data(), (size_t)h->T * sizeof(float), cudaMemcpyHostToDevice));
+    }
     CKC(dalloc(&h->ring, (size_t)3 * B * N * kChannels));
     CKC(dalloc(&h->plan, 1));
     CKC(cudaMemsetAsync(h->plan, 0, sizeof(Plan), s));
@@ -1025,7 +1047,8 @@ f3dc_status f3dc_step(f3dc_handle *h, int32_t k, int32_t B, float *S_inout, void
 
     // FlowTransformer on the active tokens at t_k
     h->cfg_B_now = guided ? B : 0;
-    f3dc_status st = run_dit(h, t[k - 1], S_inout, s);
+    f3dc_status st = run_dit(h, t[k - 1], S_inout, s,
+                             h->mod_pre ? h->mod_all + (size_t)(k - 1) * h->mod_rows : nullptr);
     h->cfg_B_now = 0;
     if (st != F3DC_OK) return st;
 
@@ -1056,8 +1079,35 @@ f3dc_status f3dc_step(f3dc_handle *h, int32_t k, int32_t B, float *S_inout, void
     return F3DC_OK;
 }
 
+static f3dc_status sample_run(f3dc_handle *h, float *S_inout, const void *cond, int32_t B, const double *sigma_override,
+                       const int32_t *quota_schedule, int32_t *quota_log, double *sigma_out, void *stream);
+
 f3dc_status f3dc_sample(f3dc_handle *h, float *S_inout, const void *cond, int32_t B, const double *sigma_override,
                         const int32_t *quota_schedule, int32_t *quota_log, double *sigma_out, void *stream)
+{
+    if (!h) return fail(nullptr, F3DC_ERR_INVALID_ARG, "null handle");
+    // the time embedding and the modulation of all T steps depend only on
+    // t_k and the weights: computed once here, in four passes per 8 steps
+    // over the modulation weights, and read by each step
+    const int W = h->W;
+    const Layout &ly = h->lay;
+    cudaStream_t s = (cudaStream_t)stream;
+    const Work w_pre = wfix(2.0 * ((double)h->mod_rows * W + 256.0 * W + (double)W * W) * ((h->T + 7) / 8));
+    LAUNCH(KF_TEMB, Work(), launch_time_freq_many(h->t_all, h->T, h->freq_all, s));
+    LAUNCH(KF_TEMB, Work(), launch_gemv_many(h->freq_all, h->T, 256, h->wt(ly.t_w1), h->wt(ly.t_b1), h->h1_all, W, 0, 1,
+                                             h->num_sms, s));
+    LAUNCH(KF_TEMB, Work(), launch_gemv_many(h->h1_all, h->T, W, h->wt(ly.t_w2), h->wt(ly.t_b2), h->temb_all, W, 0, 0,
+                                             h->num_sms, s));
+    LAUNCH(KF_TEMB, w_pre, launch_gemv_many(h->temb_all, h->T, W, h->mod_w, h->mod_b, h->mod_all, h->mod_rows, 1, 0,
+                                            h->num_sms, s));
+    h->mod_pre = true;
+    const f3dc_status st = sample_run(h, S_inout, cond, B, sigma_override, quota_schedule, quota_log, sigma_out, stream);
+    h->mod_pre = false;
+    return st;
+}
+
+static f3dc_status sample_run(f3dc_handle *h, float *S_inout, const void *cond, int32_t B, const double *sigma_override,
+                       const int32_t *quota_schedule, int32_t *quota_log, double *sigma_out, void *stream)
 {
     if (!h) return fail(nullptr, F3DC_ERR_INVALID_ARG, "null handle");
     if (!S_inout || !cond) return fail(h, F3DC_ERR_INVALID_ARG, "null pointer");

@@ -362,10 +362,8 @@ __global__ void k_scatter_rows(const float *v_active, const Plan *plan, int N, f
 }
 
 // ------------------------------------------------------------------ K9
-__global__ void k_time_freq(float t, float *freq)
+F3DC_DEV void time_freq(float t, float *freq)
 {
-    griddep_launch();
-    griddep_wait();
     const int f = threadIdx.x;  // 128 threads
     const float w = expf(-9.210340371976184f * (float)f / 128.0f);  // ln(10000)
     const float arg = 1000.0f * t * w;
@@ -373,28 +371,49 @@ __global__ void k_time_freq(float t, float *freq)
     freq[128 + f] = sinf(arg);
 }
 
+__global__ void k_time_freq(float t, float *freq)
+{
+    griddep_launch();
+    griddep_wait();
+    time_freq(t, freq);
+}
+
+// one block per time: freq[v] = sinusoid of t[v]
+__global__ void k_time_freq_many(const float *t, float *freq)
+{
+    griddep_launch();
+    griddep_wait();
+    time_freq(t[blockIdx.x], freq + (size_t)blockIdx.x * 256);
+}
+
 F3DC_DEV float silu(float v) { return v / (1.0f + expf(-v)); }
 
 constexpr int kGemvThreads = 512;
 constexpr int kGemvMaxK = 4096;
+constexpr int kGemvXs = 8192;  // staged input floats: NV * K <= 8192
 
 // One warp per pair of weight rows; each lane streams uint4 chunks of both
 // rows, four chunks per row issued before any is used (K = 1024: the whole
-// row pair in one round of loads), two CTAs of 16 warps per SM.
+// row pair in one round of loads), two CTAs of 16 warps per SM.  NV vectors
+// (x [NV, K] -> y [NV, rows], row strides K and rows) share each weight
+// load; every output is summed in the same order for any NV.
+template <int NV>
 __global__ void __launch_bounds__(kGemvThreads, 2) k_gemv(const float *x, int K, const bf16 *w, const bf16 *bias,
                                                           float *y, int rows, int silu_in, int silu_out)
 {
     griddep_launch();
     griddep_wait();
-    __shared__ float xs[kGemvMaxK];
-    for (int k = threadIdx.x; k < K; k += blockDim.x) xs[k] = silu_in ? silu(x[k]) : x[k];
+    __shared__ float xs[kGemvXs];  // NV * K floats
+    for (int k = threadIdx.x; k < NV * K; k += blockDim.x) xs[k] = silu_in ? silu(x[k]) : x[k];
     __syncthreads();
     const int lane = threadIdx.x & 31, wpb = blockDim.x >> 5;
     const int chunks = K / 8;  // 8 bf16 (one uint4) per lane per step
     const uint4 *W4 = reinterpret_cast<const uint4 *>(w);
     for (int r = (blockIdx.x * wpb + (threadIdx.x >> 5)) * 2; r < rows; r += gridDim.x * wpb * 2) {
         const bool two = r + 1 < rows;
-        float acc0 = 0.f, acc1 = 0.f;
+        float acc0[NV], acc1[NV];
+#pragma unroll
+        for (int v = 0; v < NV; ++v) acc0[v] = acc1[v] = 0.f;
         for (int q0 = lane; q0 < chunks; q0 += 4 * 32) {
             uint4 u0[4], u1[4];
 #pragma unroll
@@ -412,20 +431,24 @@ __global__ void __launch_bounds__(kGemvThreads, 2) k_gemv(const float *x, int K,
                 bf16x8_to_f32(u0[c], f0);
                 bf16x8_to_f32(u1[c], f1);
 #pragma unroll
-                for (int j = 0; j < 8; ++j) {
-                    acc0 = fmaf(f0[j], xs[k0 + j], acc0);
-                    acc1 = fmaf(f1[j], xs[k0 + j], acc1);
-                }
+                for (int v = 0; v < NV; ++v)
+#pragma unroll
+                    for (int j = 0; j < 8; ++j) {
+                        acc0[v] = fmaf(f0[j], xs[v * K + k0 + j], acc0[v]);
+                        acc1[v] = fmaf(f1[j], xs[v * K + k0 + j], acc1[v]);
+                    }
             }
         }
-        acc0 = warp_sum(acc0);
-        acc1 = warp_sum(acc1);
-        if (lane == 0) {
-            float v0 = acc0 + (bias ? bf16_at(bias, r) : 0.f);
-            y[r] = silu_out ? silu(v0) : v0;
-            if (two) {
-                float v1 = acc1 + (bias ? bf16_at(bias, r + 1) : 0.f);
-                y[r + 1] = silu_out ? silu(v1) : v1;
+#pragma unroll
+        for (int v = 0; v < NV; ++v) {
+            const float s0 = warp_sum(acc0[v]), s1 = warp_sum(acc1[v]);
+            if (lane == 0) {
+                float v0 = s0 + (bias ? bf16_at(bias, r) : 0.f);
+                y[(size_t)v * rows + r] = silu_out ? silu(v0) : v0;
+                if (two) {
+                    float v1 = s1 + (bias ? bf16_at(bias, r + 1) : 0.f);
+                    y[(size_t)v * rows + r + 1] = silu_out ? silu(v1) : v1;
+                }
             }
         }
     }
@@ -549,14 +572,40 @@ cudaError_t launch_time_freq(float t, float *freq, cudaStream_t s)
     return cudaGetLastError();
 }
 
+cudaError_t launch_time_freq_many(const float *t, int n, float *freq, cudaStream_t s)
+{
+    if (n < 1) return cudaErrorInvalidValue;
+    launch_k(k_time_freq_many, dim3(n), dim3(128), 0, s, t, freq);
+    return cudaGetLastError();
+}
+
 cudaError_t launch_gemv(const float *x, int K, const bf16 *w, const bf16 *b, float *y, int rows, int silu_in,
                         int silu_out, int num_sms, cudaStream_t s)
 {
-    if (K % 8 != 0 || K > kGemvMaxK) return cudaErrorInvalidValue;
+    return launch_gemv_many(x, 1, K, w, b, y, rows, silu_in, silu_out, num_sms, s);
+}
+
+cudaError_t launch_gemv_many(const float *x, int nv, int K, const bf16 *w, const bf16 *b, float *y, int rows,
+                             int silu_in, int silu_out, int num_sms, cudaStream_t s)
+{
+    if (K % 8 != 0 || K > kGemvMaxK || nv < 1) return cudaErrorInvalidValue;
     const int wpb = kGemvThreads / 32;
     int grid = (rows + 2 * wpb - 1) / (2 * wpb);
     if (grid > num_sms * 2) grid = num_sms * 2;
-    launch_k(k_gemv, dim3(grid), dim3(kGemvThreads), 0, s, x, K, w, b, y, rows, silu_in, silu_out);
+    // vectors in groups whose inputs fit the shared staging (8, 4, 2 or 1)
+    for (int v0 = 0; v0 < nv;) {
+        const int left = nv - v0;
+        const int g = left >= 8 && 8 * K <= kGemvXs ? 8 : (left >= 4 && 4 * K <= kGemvXs ? 4 : (left >= 2 && 2 * K <= kGemvXs ? 2 : 1));
+        const float *xg = x + (size_t)v0 * K;
+        float *yg = y + (size_t)v0 * rows;
+        switch (g) {
+        case 8: launch_k(k_gemv<8>, dim3(grid), dim3(kGemvThreads), 0, s, xg, K, w, b, yg, rows, silu_in, silu_out); break;
+        case 4: launch_k(k_gemv<4>, dim3(grid), dim3(kGemvThreads), 0, s, xg, K, w, b, yg, rows, silu_in, silu_out); break;
+        case 2: launch_k(k_gemv<2>, dim3(grid), dim3(kGemvThreads), 0, s, xg, K, w, b, yg, rows, silu_in, silu_out); break;
+        default: launch_k(k_gemv<1>, dim3(grid), dim3(kGemvThreads), 0, s, xg, K, w, b, yg, rows, silu_in, silu_out); break;
+        }
+        v0 += g;
+    }
     return cudaGetLastError();
 }
 

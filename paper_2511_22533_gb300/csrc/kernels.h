@@ -120,9 +120,15 @@ cudaError_t launch_scatter_rows(const float *v_active, const Plan *plan, int B, 
 
 // ------------------------------------------------------------ t-embedding
 cudaError_t launch_time_freq(float t, float *freq, cudaStream_t s);
+// freq [n, 256] for the n times t[0..n) (device)
+cudaError_t launch_time_freq_many(const float *t, int n, float *freq, cudaStream_t s);
 // y[n] = act_out(sum_k act_in(x[k]) w[n, k] + b[n]); act = SiLU when flag set
 cudaError_t launch_gemv(const float *x, int K, const bf16 *w, const bf16 *b, float *y, int rows, int silu_in,
                         int silu_out, int num_sms, cudaStream_t s);
+// the same for nv vectors x [nv, K] -> y [nv, rows]; each output equals the
+// single-vector launch's bit for bit
+cudaError_t launch_gemv_many(const float *x, int nv, int K, const bf16 *w, const bf16 *b, float *y, int rows,
+                             int silu_in, int silu_out, int num_sms, cudaStream_t s);
 
 // ------------------------------------------------------------ GEMM
 enum GemmEpi { kEpiBias = 0, kEpiGelu = 1, kEpiResid = 2, kEpiQKNorm = 3 };
