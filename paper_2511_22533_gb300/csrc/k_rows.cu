@@ -392,51 +392,58 @@ constexpr int kGemvThreads = 512;
 constexpr int kGemvMaxK = 4096;
 constexpr int kGemvXs = 8192;  // staged input floats: NV * K <= 8192
 
-// One warp per pair of weight rows; each lane streams uint4 chunks of both
-// rows, four chunks per row issued before any is used (K = 1024: the whole
-// row pair in one round of loads), two CTAs of 16 warps per SM.  NV vectors
-// (x [NV, K] -> y [NV, rows], row strides K and rows) share each weight
-// load; every output is summed in the same order for any NV.
+// One warp per pair of weight rows.  Lane l owns the 4-wide column groups
+// g = l, l + 32, ... (k = 4g .. 4g + 3): it loads them as 8-byte pieces of
+// both rows -- eight pieces per row in flight for one or two vectors, fewer
+// for more -- and reads the matching inputs as one float4 each, so a
+// warp's shared-memory reads are consecutive (conflict-free).  NV vectors (x [NV, K] -> y [NV, rows], row
+// strides K and rows) share each weight load; every output is summed in the
+// same order for any NV.  Two CTAs of 16 warps per SM.
 template <int NV>
 __global__ void __launch_bounds__(kGemvThreads, 2) k_gemv(const float *x, int K, const bf16 *w, const bf16 *bias,
                                                           float *y, int rows, int silu_in, int silu_out)
 {
     griddep_launch();
     griddep_wait();
-    __shared__ float xs[kGemvXs];  // NV * K floats
+    __shared__ float4 xs4[kGemvXs / 4];  // NV * K floats
+    float *xs = reinterpret_cast<float *>(xs4);
     for (int k = threadIdx.x; k < NV * K; k += blockDim.x) xs[k] = silu_in ? silu(x[k]) : x[k];
     __syncthreads();
     const int lane = threadIdx.x & 31, wpb = blockDim.x >> 5;
-    const int chunks = K / 8;  // 8 bf16 (one uint4) per lane per step
-    const uint4 *W4 = reinterpret_cast<const uint4 *>(w);
+    const int groups = K / 4;  // 4 bf16 (one uint2) per lane per step
+    const uint2 *W2 = reinterpret_cast<const uint2 *>(w);
     for (int r = (blockIdx.x * wpb + (threadIdx.x >> 5)) * 2; r < rows; r += gridDim.x * wpb * 2) {
         const bool two = r + 1 < rows;
         float acc0[NV], acc1[NV];
 #pragma unroll
         for (int v = 0; v < NV; ++v) acc0[v] = acc1[v] = 0.f;
-        for (int q0 = lane; q0 < chunks; q0 += 4 * 32) {
-            uint4 u0[4], u1[4];
+        constexpr int kDepth = NV >= 8 ? 2 : (NV >= 4 ? 4 : 8);  // pieces per row in flight
+        for (int g0 = lane; g0 < groups; g0 += kDepth * 32) {
+            uint2 u0[kDepth], u1[kDepth];
 #pragma unroll
-            for (int c = 0; c < 4; ++c) {
-                const int q = q0 + c * 32;
-                u0[c] = q < chunks ? __ldg(W4 + (size_t)r * (K / 8) + q) : make_uint4(0, 0, 0, 0);
-                u1[c] = two && q < chunks ? __ldg(W4 + (size_t)(r + 1) * (K / 8) + q) : make_uint4(0, 0, 0, 0);
+            for (int c = 0; c < kDepth; ++c) {
+                const int g = g0 + c * 32;
+                u0[c] = g < groups ? __ldg(W2 + (size_t)r * (K / 4) + g) : make_uint2(0, 0);
+                u1[c] = two && g < groups ? __ldg(W2 + (size_t)(r + 1) * (K / 4) + g) : make_uint2(0, 0);
             }
 #pragma unroll
-            for (int c = 0; c < 4; ++c) {
-                const int q = q0 + c * 32;
-                if (q >= chunks) break;
-                const int k0 = q * 8;
-                float f0[8], f1[8];
-                bf16x8_to_f32(u0[c], f0);
-                bf16x8_to_f32(u1[c], f1);
+            for (int c = 0; c < kDepth; ++c) {
+                const int g = g0 + c * 32;
+                if (g >= groups) break;
+                const float f0[4] = {bf16_bits_to_f32(u0[c].x & 0xFFFFu), bf16_bits_to_f32(u0[c].x >> 16),
+                                     bf16_bits_to_f32(u0[c].y & 0xFFFFu), bf16_bits_to_f32(u0[c].y >> 16)};
+                const float f1[4] = {bf16_bits_to_f32(u1[c].x & 0xFFFFu), bf16_bits_to_f32(u1[c].x >> 16),
+                                     bf16_bits_to_f32(u1[c].y & 0xFFFFu), bf16_bits_to_f32(u1[c].y >> 16)};
 #pragma unroll
-                for (int v = 0; v < NV; ++v)
+                for (int v = 0; v < NV; ++v) {
+                    const float4 xv = xs4[(v * K) / 4 + g];
+                    const float xa[4] = {xv.x, xv.y, xv.z, xv.w};
 #pragma unroll
-                    for (int j = 0; j < 8; ++j) {
-                        acc0[v] = fmaf(f0[j], xs[v * K + k0 + j], acc0[v]);
-                        acc1[v] = fmaf(f1[j], xs[v * K + k0 + j], acc1[v]);
+                    for (int j = 0; j < 4; ++j) {
+                        acc0[v] = fmaf(f0[j], xa[j], acc0[v]);
+                        acc1[v] = fmaf(f1[j], xa[j], acc1[v]);
                     }
+                }
             }
         }
 #pragma unroll
