@@ -219,12 +219,15 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
             const uint64_t k_desc0 = make_sdesc(smem_u32(sK), 16, Cfg::kAtom, Cfg::kSwz);
             const uint64_t v_desc0 = make_sdesc(smem_u32(sV), Cfg::kAtom, Cfg::kAtom, Cfg::kSwz);
             constexpr uint64_t kStageStep = Cfg::kTileBytes >> 4, kVRowStep = (16 * Cfg::kRowBytes) >> 4;
-            auto s_mmas = [&](uint32_t gt) {  // S_gt = Q K_gt^T into S buffer gt % 2
+            // S_gt = Q K_gt^T into S buffer gt % 2.  Only an item's first two
+            // tiles commit to s_full; a later tile's S is issued just before
+            // P V of the tile two back and reported by that P V's commit
+            auto s_mmas = [&](uint32_t gt, bool commit) {
                 const uint64_t kd = k_desc0 + (gt % kKVStages) * kStageStep;
 #pragma unroll
                 for (int kk = 0; kk < DH / 16; ++kk)
                     mma_bf16(tmem + (gt & 1) * 128, q_desc + 2 * kk, kd + 2 * kk, idesc_s, kk > 0);
-                mma_commit(&s_full[gt & 1]);
+                if (commit) mma_commit(&s_full[gt & 1]);
             };
             // O_e (+)= P_e V for tile gt of parity e = gt % 2, P_e read from
             // TMEM (8 columns per 16 keys); `fresh` overwrites O_e (the item's
@@ -258,11 +261,11 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
                 q_desc = q_desc0 + qb * (Cfg::kTileBytes >> 4);
                 if (!kv_wait(g)) break;
                 tc_fence_after();
-                s_mmas(g);
+                s_mmas(g, true);
                 if (nkt > 1) {
                     if (!kv_wait(g + 1)) break;
                     tc_fence_after();
-                    s_mmas(g + 1);
+                    s_mmas(g + 1, true);
                 }
                 // O_0 / O_1 are overwritten by this item's first P V: the
                 // softmax must have read the previous item's result
@@ -277,8 +280,8 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
                         break;
                     }
                     tc_fence_after();
-                    s_mmas(gt + 2);
-                    pv_mmas(gt, j < 2);
+                    s_mmas(gt + 2, false);
+                    pv_mmas(gt, j < 2);  // its commit also reports S_(gt+2)
                 }
                 if (!ok) break;
                 mma_commit(&q_empty[qb]);  // every S of the item issued: its Q buffer may be refilled
@@ -304,12 +307,15 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
         const uint32_t o_addr = tmem + tl + Cfg::kColO + par * DH;
         const uint32_t p_addr = tmem + tl + Cfg::kColP + par * 64;
         uint32_t g = 0, item_it = 0;  // global key-tile counter at the start of the item
-        // s_full[par] completes once per tile of this parity, in tile order
-        // (tile t with parity (t / 2) % 2); P V of tile t is awaited on
-        // kv_empty[t % 4] with parity (t / 4) % 2.  A warp waits for P V of
-        // its previous tile (t - 2) before it writes P again, and P V of its
-        // next tile cannot start before that, so no barrier it reads is ever
-        // more than one phase ahead of it.
+        uint32_t s_use = 0;           // s_full[par] completions consumed
+        // S of an item's first tile of this parity completes s_full[par]
+        // (once per item in which the parity has a tile; s_use counts them);
+        // S of every later tile t is reported with P V of tile t - 2 on
+        // kv_empty[(t - 2) % 4] (parity ((t - 2) / 4) % 2), which also frees
+        // P and O for tile t.  A warp waits for P V of its previous tile
+        // before it writes P again, and P V of its next tile cannot start
+        // before that, so no barrier it reads is ever more than one phase
+        // ahead of it.
         for (int w = blockIdx.x; w < total; w += gridDim.x, ++item_it) {
             const Item it = decode_item(p, w);
             const int nkt = (it.nk + 127) / 128;
@@ -317,8 +323,11 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
             bool ok = true, any = false;
             uint32_t g_last = 0;
             for (int j = (int)((par - g) & 1); j < nkt; j += 2) {
-                const uint32_t gt = g + (uint32_t)j, ph = (gt >> 1) & 1;
-                if (!mbar_wait(&s_full[par], ph, abort_flag, p.err)) {
+                const uint32_t gt = g + (uint32_t)j;
+                const bool first = j < 2;  // S reported on s_full, else with P V of tile gt - 2
+                if (first ? !mbar_wait(&s_full[par], (s_use++) & 1, abort_flag, p.err)
+                          : !mbar_wait(&kv_empty[(gt - 2) % kKVStages], ((gt - 2) / kKVStages) & 1, abort_flag,
+                                       p.err)) {
                     ok = false;
                     break;
                 }
@@ -364,7 +373,8 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
                 }
                 const float m_use = m_ref == -INFINITY ? 0.f : m_ref;
                 // P_par and O_par: P V of this parity's previous tile must be done
-                if (gt >= 2 && !mbar_wait(&kv_empty[(gt - 2) % kKVStages], ((gt - 2) / kKVStages) & 1, abort_flag, p.err)) {
+                if (first && gt >= 2 &&
+                    !mbar_wait(&kv_empty[(gt - 2) % kKVStages], ((gt - 2) / kKVStages) & 1, abort_flag, p.err)) {
                     ok = false;
                     break;
                 }
