@@ -201,12 +201,44 @@ F3DC_DEV void put_bf16x32(OutStage &o, const float *v)
     }
 }
 
+// Per-column operands of one 32-column chunk (BIAS, GELU, RESID epilogues),
+// loaded ahead of the chunk's accumulator so their L2 latency is hidden.
+struct ColOps {
+    uint4 b[4];   // 32 bf16 biases (zeros without a bias)
+    float4 g[8];  // 32 fp32 gates (RESID; ones without a gate)
+};
+
+template <int EPI>
+F3DC_DEV void load_colops(const GemmParams &p, int col, ColOps &c)
+{
+    if (p.bias) {
+        const uint4 *pb = reinterpret_cast<const uint4 *>(p.bias + col);
+#pragma unroll
+        for (int q = 0; q < 4; ++q) c.b[q] = __ldg(pb + q);
+    } else {
+#pragma unroll
+        for (int q = 0; q < 4; ++q) c.b[q] = make_uint4(0u, 0u, 0u, 0u);
+    }
+    if constexpr (EPI == kEpiResid) {
+        if (p.gate) {
+            const float4 *pg = reinterpret_cast<const float4 *>(p.gate + col);
+#pragma unroll
+            for (int q = 0; q < 8; ++q) c.g[q] = __ldg(pg + q);
+        } else {
+#pragma unroll
+            for (int q = 0; q < 8; ++q) c.g[q] = make_float4(1.f, 1.f, 1.f, 1.f);
+        }
+    }
+}
+
 // Applies the epilogue to the column chunks k0, k0 + kstep, ... of a tile
 // bn columns wide (chunks of 64 columns for QKNORM, whose RMSNorm groups
-// span 64, else 32).
+// span 64, else 32).  Outside QKNORM the next chunk's biases and gates are
+// loaded while the current chunk is processed; `first`, when given, holds the
+// first chunk's (loaded by the caller before it waited for the accumulator).
 template <int EPI, typename Src>
 F3DC_DEV void epilogue_tile(const GemmParams &p, const Src &src, OutStage &o, int m0, int n0, int bn, int k0 = 0,
-                            int kstep = 1)
+                            int kstep = 1, const ColOps *first = nullptr)
 {
     if constexpr (EPI == kEpiQKNorm) {
 #pragma unroll 1
@@ -240,15 +272,27 @@ F3DC_DEV void epilogue_tile(const GemmParams &p, const Src &src, OutStage &o, in
             o.template emit<false>(col + 32, m0);
         }
     } else {
+        ColOps nxt;
+        if (first)
+            nxt = *first;
+        else if (32 * k0 < bn)
+            load_colops<EPI>(p, n0 + 32 * k0, nxt);
 #pragma unroll 1
         for (int c0 = 32 * k0; c0 < bn; c0 += 32 * kstep) {
+            const int col = n0 + c0;
+            const ColOps cur = nxt;
+            if (c0 + 32 * kstep < bn) load_colops<EPI>(p, col + 32 * kstep, nxt);
             float v[32];
             src(c0, v);
-            const int col = n0 + c0;
-            float b[32];
-            load_bias32(p.bias, col, b);
 #pragma unroll
-            for (int j = 0; j < 32; ++j) v[j] += b[j];
+            for (int q = 0; q < 4; ++q) {
+                const uint32_t w[4] = {cur.b[q].x, cur.b[q].y, cur.b[q].z, cur.b[q].w};
+#pragma unroll
+                for (int j = 0; j < 4; ++j) {
+                    v[q * 8 + 2 * j] += bf16_bits_to_f32(w[j] & 0xFFFFu);
+                    v[q * 8 + 2 * j + 1] += bf16_bits_to_f32(w[j] >> 16);
+                }
+            }
             if constexpr (EPI == kEpiGelu) {
 #pragma unroll
                 for (int j = 0; j < 32; ++j) v[j] = gelu_tanh(v[j]);
@@ -259,8 +303,7 @@ F3DC_DEV void epilogue_tile(const GemmParams &p, const Src &src, OutStage &o, in
                 for (int h = 0; h < 2; ++h) {
 #pragma unroll
                     for (int q = 0; q < 4; ++q) {
-                        const float4 g = p.gate ? __ldg(reinterpret_cast<const float4 *>(p.gate + col + 16 * h) + q)
-                                                : make_float4(1.f, 1.f, 1.f, 1.f);
+                        const float4 g = cur.g[4 * h + q];
                         const float *w = v + 16 * h + 4 * q;
                         o.put16(q, make_uint4(__float_as_uint(g.x * w[0]), __float_as_uint(g.y * w[1]),
                                               __float_as_uint(g.z * w[2]), __float_as_uint(g.w * w[3])));
@@ -703,6 +746,9 @@ __global__ void __launch_bounds__(kPairThreads, 1)
         for (int t = cl; t < tiles; t += ncl, ++it) {
             const int buf = it & 1;
             const uint32_t aph = (it >> 1) & 1;
+            const int n0 = (t / pm_tiles) * bn;
+            ColOps first;
+            if constexpr (EPI != kEpiQKNorm) load_colops<EPI>(p, n0 + 32 * grp, first);
             const uint32_t got = mbar_wait(&accf[buf], aph, abort_flag, p.err) ? 1u : 0u;
             uint32_t all;
             asm volatile("{\n .reg .pred p, q;\n setp.ne.u32 p, %1, 0;\n bar.red.and.pred q, %2, 128, p;\n"
@@ -713,12 +759,11 @@ __global__ void __launch_bounds__(kPairThreads, 1)
             if (!all) break;
             tc_fence_after();
             const int m0 = (t % pm_tiles) * 256 + (int)rank * 128;
-            const int n0 = (t / pm_tiles) * bn;
             // the odd CTA's rows of the last pair lie beyond the plan when
             // the tile count is odd: computed, not stored
             if (m0 < m_tiles * 128) {
                 const TmemSrc tsrc{tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(buf * 256)};
-                epilogue_tile<EPI>(p, tsrc, o, m0, n0, bn, grp, 2);
+                epilogue_tile<EPI>(p, tsrc, o, m0, n0, bn, grp, 2, &first);
             }
             tc_fence_before();
             __syncwarp();
