@@ -35,6 +35,8 @@
 // V is the MN-major B operand of the P V MMA straight from its row-major
 // TMA tile.  Keys beyond a sample's count are masked to -inf before the
 // exponent; padding rows are finite by construction, so 0 * pad = 0.
+#include <atomic>
+
 #include "common.cuh"
 #include "kernels.h"
 
@@ -520,12 +522,17 @@ template <int DH>
 cudaError_t launch_dh(const CUtensorMap *tq, const CUtensorMap *tk, const CUtensorMap *tv, const AttnParams &p,
                       int grid, cudaStream_t s)
 {
-    static bool attr_set = false;
+    // the shared-memory attribute is per device: set it on each device's first launch
+    static std::atomic<uint64_t> attr_devices{0};
     const size_t smem = AttnCfg<DH>::kSmem;
-    if (!attr_set) {
-        cudaError_t e = cudaFuncSetAttribute(k_attn<DH>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    const uint64_t bit = 1ull << (dev & 63);
+    if (!(attr_devices.load(std::memory_order_acquire) & bit)) {
+        e = cudaFuncSetAttribute(k_attn<DH>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
         if (e != cudaSuccess) return e;
-        attr_set = true;
+        attr_devices.fetch_or(bit, std::memory_order_acq_rel);
     }
     launch_k(k_attn<DH>, dim3(grid), dim3(kAttnThreads), smem, s, *tq, *tk, *tv, p);
     return cudaGetLastError();

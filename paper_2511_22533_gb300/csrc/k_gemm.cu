@@ -23,6 +23,8 @@
 // same launch serves any number of active tokens.
 #include <stdio.h>
 
+#include <atomic>
+
 #include <cudaTypedefs.h>
 
 #include "common.cuh"
@@ -793,10 +795,15 @@ template <int EPI>
 cudaError_t launch_pair_one(const CUtensorMap *ta, const CUtensorMap *tb, const CUtensorMap *to, const GemmParams &p,
                             int max_pair_tiles, cudaStream_t s)
 {
-    static int max_clusters = 0;
+    // per device: the shared-memory attribute and the resident-cluster count
+    // are taken on each device's first launch (0 = not yet known)
+    static std::atomic<int> max_clusters_of[64];
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    int max_clusters = max_clusters_of[dev & 63].load(std::memory_order_acquire);
     if (!max_clusters) {
-        cudaError_t e =
-            cudaFuncSetAttribute(k_gemm_pair<EPI>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kPairSmem);
+        e = cudaFuncSetAttribute(k_gemm_pair<EPI>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kPairSmem);
         if (e != cudaSuccess) return e;
         cudaLaunchConfig_t cfg = {};
         cfg.gridDim = dim3(2);
@@ -814,6 +821,7 @@ cudaError_t launch_pair_one(const CUtensorMap *ta, const CUtensorMap *tb, const 
         if (e != cudaSuccess) return e;
         if (n < 1) return cudaErrorInvalidConfiguration;
         max_clusters = n;
+        max_clusters_of[dev & 63].store(n, std::memory_order_release);
     }
     const int clusters = max_pair_tiles < max_clusters ? (max_pair_tiles > 0 ? max_pair_tiles : 1) : max_clusters;
     cudaLaunchConfig_t cfg = {};
@@ -830,7 +838,7 @@ cudaError_t launch_pair_one(const CUtensorMap *ta, const CUtensorMap *tb, const 
     at[1].val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = at;
     cfg.numAttrs = 2;
-    cudaError_t e = cudaLaunchKernelEx(&cfg, k_gemm_pair<EPI>, *ta, *tb, *to, p);
+    e = cudaLaunchKernelEx(&cfg, k_gemm_pair<EPI>, *ta, *tb, *to, p);
     if (e != cudaSuccess) return e;
     return cudaGetLastError();
 }
@@ -839,12 +847,17 @@ template <int BN, int EPI>
 cudaError_t launch_one(const CUtensorMap *ta, const CUtensorMap *tb, const CUtensorMap *to, const CUtensorMap *tw,
                        const GemmParams &p, int grid, cudaStream_t s)
 {
-    static bool attr_set = false;
+    // the shared-memory attribute is per device: set it on each device's first launch
+    static std::atomic<uint64_t> attr_devices{0};
     const size_t smem = GemmCfg<BN>::kSmem;
-    if (!attr_set) {
-        cudaError_t e = cudaFuncSetAttribute(k_gemm<BN, EPI>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    const uint64_t bit = 1ull << (dev & 63);
+    if (!(attr_devices.load(std::memory_order_acquire) & bit)) {
+        e = cudaFuncSetAttribute(k_gemm<BN, EPI>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
         if (e != cudaSuccess) return e;
-        attr_set = true;
+        attr_devices.fetch_or(bit, std::memory_order_acq_rel);
     }
     launch_k(k_gemm<BN, EPI>, dim3(grid), dim3(kGemmThreads), smem, s, *ta, *tb, *to, *tw, p);
     return cudaGetLastError();
