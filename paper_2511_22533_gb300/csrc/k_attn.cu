@@ -27,11 +27,10 @@
 //              only raised (and O_e, l rescaled in place) when a tile's max
 //              exceeds it by more than 2^8, so most tiles need no O traffic.
 //              The two parities of a row are combined once per work item.
-//              The exponent unit (16 results per clock per SM) bounds the
-//              softmax; because the two warps of an SM sub-partition work on
+//              Because the two warps of an SM sub-partition work on
 //              different tiles, one warp's TMEM load, maximum and barrier
 //              phases overlap the other's exponents instead of leaving the
-//              unit idle.
+//              exponent unit idle.
 // V is the MN-major B operand of the P V MMA straight from its row-major
 // TMA tile.  Keys beyond a sample's count are masked to -inf before the
 // exponent; padding rows are finite by construction, so 0 * pad = 0.
