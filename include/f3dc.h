@@ -135,7 +135,7 @@ typedef struct f3dc_handle f3dc_handle;
  * (Supp. Sec. D) and gamma_up 64.  Host only. */
 f3dc_status f3dc_config_default(f3dc_config *cfg);
 
-/* Number of bf16 elements of a layout-v1 weight blob for cfg.  Host only;
+/* Number of bf16 elements of a layout-v2 weight blob for cfg.  Host only;
  * returns 0 for an invalid cfg. */
 size_t f3dc_weights_elems(const f3dc_config *cfg);
 

@@ -260,7 +260,7 @@ def f32_to_bf16(x: float) -> int:
 # ------------------------------------------------------------------ model
 
 class Model:
-    """Oracle flow transformer built from a layout-v1 weight blob."""
+    """Oracle flow transformer built from a layout-v2 weight blob."""
 
     def __init__(self, shape, blob_bits: np.ndarray):
         self.shape = shape

@@ -176,7 +176,7 @@ def pcsc_quota(cfg: Config, sigma: float, k: int, consec=None):
 # ---------------------------------------------------------------- handle
 
 class Handle:
-    """Owns an f3dc_handle.  `blob` is a CUDA tensor of the layout-v1 bf16
+    """Owns an f3dc_handle.  `blob` is a CUDA tensor of the layout-v2 bf16
     weights (any 16-bit dtype); it may be freed after construction."""
 
     def __init__(self, cfg: Config, blob, stream=None):

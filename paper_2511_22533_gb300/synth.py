@@ -29,7 +29,7 @@ import math
 
 import numpy as np
 
-LAYOUT_VERSION = 1
+LAYOUT_VERSION = 2
 ALIGN_ELEMS = 64
 
 
