@@ -5,7 +5,10 @@
 // out[m, n] = epilogue( sum_k A[m, k] B[n, k] ),  A = activations [M, K]
 // bf16, B = weights [N, K] bf16 (nn.Linear layout), fp32 accumulation.
 //
-// Persistent warp-specialised kernel, one CTA per SM (192 threads):
+// Two kernels.  The transformer's step GEMMs (N a multiple of 256) run on
+// k_gemm_pair, a CTA-pair (cta_group::2) version described with it below.
+// k_gemm, the single-CTA kernel, serves the other widths and split K: a
+// persistent warp-specialised kernel, one CTA per SM (192 threads):
 //   warp 0     TMA producer: 128x64 A and BNx64 B tiles, 128B-swizzled, into
 //              a STAGES-deep shared-memory ring (mbarrier full / empty)
 //   warp 1     TMEM allocator + single-thread tcgen05.mma issuer
