@@ -6,7 +6,7 @@ import numpy as np
 import pytest
 import torch
 
-from gpu_helpers import (VEL_MAX_ABS, VEL_REL_L2, assert_clean, dev_f32, dev_i32, dev_u16, handle_for, host_u16,
+from gpu_helpers import (VEL_REL_L2, assert_clean, dev_f32, dev_i32, dev_u16, handle_for, host_u16,
                          rel_l2, stored_vel_excess)
 from paper_2511_22533_gb300 import synth
 

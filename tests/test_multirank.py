@@ -3,7 +3,6 @@ max-over-ranks timing, whole-job throughput) on CPU with gloo ranks."""
 import os
 import socket
 
-import numpy as np
 import pytest
 import torch.distributed as dist
 import torch.multiprocessing as mp

@@ -3,7 +3,6 @@
 upsampling, 16 -> 8 at (2D)^3, 2x, 8 -> 1 at (4D)^3; occupied iff logit > 0),
 checked against closed forms on hand-set weights."""
 import numpy as np
-import pytest
 
 from paper_2511_22533_gb300 import synth
 

@@ -1,6 +1,5 @@
 """Oracle pins: time schedule (Supp. Sec. D), phases and PCSC (Sec. 4.2,
 Algorithm 1 step 1) and the tau refresh rule (Sec. 4.3, Algorithm 1 SSC)."""
-import math
 
 import numpy as np
 import pytest
