@@ -90,6 +90,47 @@ def test_zeroed_branches_make_block_identity(orc):
     assert np.abs(v3 - v2).max() > 1e-3
 
 
+def test_identity_blocks_leave_embedding_and_final_layer(orc):
+    # with every block an identity (zero modulation: gates 0; zero
+    # cross-attention output), the forward is the final layer applied to the
+    # input embedding: v_i = W_out (LN(x_i) (1 + scale) + shift) + b_out,
+    # x_i = W_in S_i + b_in + pos(i), (shift, scale) = Linear(SiLU(temb)).
+    # At t = 0 the timestep sinusoid is [1]*128 + [0]*128, so the expected
+    # value is plain NumPy on the blob's weights (plus the position table,
+    # pinned by its closed form); this fixes the embedding and final-layer
+    # wiring: operand orientation, the shift / scale order and the 1 + scale.
+    s = synth.ModelShape(4, 8, 64, 2, 2, 4, 5, 64, 4, 8)
+    blob = synth.weights_blob(s, 7)
+    for l in range(s.blocks):
+        for name in ("mod_w", "mod_b", "co_w", "co_b"):
+            synth.set_weight(blob, s, name, l, 0.0)
+    offs, _ = synth.weight_offsets(s)
+
+    def w(name):
+        off, dims = offs[(name, -1)]
+        return synth.bf16_bits_to_f32(blob[off:off + int(np.prod(dims))]).astype(np.float64).reshape(dims)
+
+    def silu(z):
+        return z / (1.0 + np.exp(-z))
+
+    m = orc.Model(s, blob)
+    rng = np.random.default_rng(5)
+    S = rng.standard_normal((s.tokens, 8)).astype(np.float32)
+    idx = np.sort(rng.choice(s.tokens, 40, replace=False)).astype(np.int32)
+    cond = synth.cond_tokens(s, 1, 4)[0]
+    got = m.forward(S, idx, 0.0, m.cond_kv(cond)).astype(np.float64)
+
+    freq = np.concatenate([np.ones(128), np.zeros(128)])
+    temb = w("t_w2") @ silu(w("t_w1") @ freq + w("t_b1")) + w("t_b2")
+    mod = w("fmod_w") @ silu(temb) + w("fmod_b")
+    shift, scale = mod[:s.width], mod[s.width:]
+    pos = np.stack([orc.pos_embed(s.grid, s.width, int(i)) for i in idx]).astype(np.float64)
+    x = S[idx].astype(np.float64) @ w("in_w").T + w("in_b") + pos
+    xh = (x - x.mean(axis=1, keepdims=True)) / np.sqrt(x.var(axis=1, keepdims=True) + 1e-6)
+    ref = (xh * (1.0 + scale) + shift) @ w("out_w").T + w("out_b")
+    np.testing.assert_allclose(got, ref, rtol=2e-4, atol=2e-5)
+
+
 def test_sample_quota_zero_is_plain_euler(tiny, orc):
     # quota 0 at every step must reproduce the uncached sampler exactly
     m, S, cond = tiny["model"], tiny["S"][:1], tiny["cond"][:1]
