@@ -131,6 +131,91 @@ def test_identity_blocks_leave_embedding_and_final_layer(orc):
     np.testing.assert_allclose(got, ref, rtol=2e-4, atol=2e-5)
 
 
+def _numpy_head_tail(s, blob):
+    """NumPy input embedding and t = 0 final layer on the blob's weights."""
+    offs, _ = synth.weight_offsets(s)
+
+    def w(name, blk=-1):
+        off, dims = offs[(name, blk)]
+        return synth.bf16_bits_to_f32(blob[off:off + int(np.prod(dims))]).astype(np.float64).reshape(dims)
+
+    def silu(z):
+        return z / (1.0 + np.exp(-z))
+
+    def ln(x):
+        return (x - x.mean(axis=1, keepdims=True)) / np.sqrt(x.var(axis=1, keepdims=True) + 1e-6)
+
+    freq = np.concatenate([np.ones(128), np.zeros(128)])
+    temb = w("t_w2") @ silu(w("t_w1") @ freq + w("t_b1")) + w("t_b2")
+    fmod = w("fmod_w") @ silu(temb) + w("fmod_b")
+
+    def tail(x):
+        return (ln(x) * (1.0 + fmod[s.width:]) + fmod[:s.width]) @ w("out_w").T + w("out_b")
+
+    return w, ln, tail
+
+
+def _one_branch_model(orc, gate_slot, seed):
+    # blocks are identities except block 0's branch `gate_slot` (2: the
+    # self-attention gate, 5: the MLP gate), whose modulation is the constant
+    # bias shift = 0.25, scale = 0.125, gate = 0.5 (exact in bf16)
+    s = synth.ModelShape(4, 8, 64, 2, 2, 4, 5, 64, 4, 8)
+    blob = synth.weights_blob(s, seed)
+    for l in range(s.blocks):
+        for name in ("mod_w", "mod_b", "co_w", "co_b"):
+            synth.set_weight(blob, s, name, l, 0.0)
+    mb = np.zeros(6 * s.width, np.float32)
+    base = (gate_slot - 2) * s.width  # shift of the same branch
+    mb[base:base + s.width] = 0.25
+    mb[base + s.width:base + 2 * s.width] = 0.125
+    mb[base + 2 * s.width:base + 3 * s.width] = 0.5
+    synth.set_weight(blob, s, "mod_b", 0, mb)
+    return s, blob
+
+
+def test_single_token_self_attention_branch(orc):
+    # one active token attends to itself only (softmax over one key is 1),
+    # so block 0's self-attention branch reduces to its value and output
+    # projections: x += gate1 (W_o (W_v h + b_v) + b_o), h = LN(x)(1 +
+    # scale1) + shift1 -- pins the value rows of the QKV projection, the
+    # output projection and the (shift, scale, gate) order of the modulation
+    s, blob = _one_branch_model(orc, 2, 11)
+    w, ln, tail = _numpy_head_tail(s, blob)
+    m = orc.Model(s, blob)
+    S = np.random.default_rng(6).standard_normal((s.tokens, 8)).astype(np.float32)
+    cond = synth.cond_tokens(s, 1, 4)[0]
+    i = 37
+    got = m.forward(S, np.array([i], np.int32), 0.0, m.cond_kv(cond)).astype(np.float64)
+    W = s.width
+    x = S[[i]].astype(np.float64) @ w("in_w").T + w("in_b") + orc.pos_embed(s.grid, W, i).astype(np.float64)
+    h = ln(x) * 1.125 + 0.25
+    qkv = h @ w("qkv_w", 0).T + w("qkv_b", 0)
+    y = qkv[:, 2 * W:] @ w("o_w", 0).T + w("o_b", 0)
+    ref = tail(x + 0.5 * y)
+    np.testing.assert_allclose(got, ref, rtol=2e-4, atol=2e-5)
+
+
+def test_mlp_branch(orc):
+    # block 0's MLP branch alone: x += gate2 fc2(GELU_tanh(fc1(LN(x)(1 +
+    # scale2) + shift2))) on every active token independently
+    s, blob = _one_branch_model(orc, 5, 12)
+    w, ln, tail = _numpy_head_tail(s, blob)
+    m = orc.Model(s, blob)
+    S = np.random.default_rng(7).standard_normal((s.tokens, 8)).astype(np.float32)
+    cond = synth.cond_tokens(s, 1, 4)[0]
+    idx = np.array([3, 17, 40, 63], np.int32)
+    got = m.forward(S, idx, 0.0, m.cond_kv(cond)).astype(np.float64)
+    W = s.width
+    pos = np.stack([orc.pos_embed(s.grid, W, int(i)) for i in idx]).astype(np.float64)
+    x = S[idx].astype(np.float64) @ w("in_w").T + w("in_b") + pos
+    h = ln(x) * 1.125 + 0.25
+    u = h @ w("fc1_w", 0).T + w("fc1_b", 0)
+    g = 0.5 * u * (1.0 + np.tanh(np.sqrt(2.0 / np.pi) * (u + 0.044715 * u ** 3)))
+    y = g @ w("fc2_w", 0).T + w("fc2_b", 0)
+    ref = tail(x + 0.5 * y)
+    np.testing.assert_allclose(got, ref, rtol=2e-4, atol=2e-5)
+
+
 def test_sample_quota_zero_is_plain_euler(tiny, orc):
     # quota 0 at every step must reproduce the uncached sampler exactly
     m, S, cond = tiny["model"], tiny["S"][:1], tiny["cond"][:1]
