@@ -216,6 +216,34 @@ def test_mlp_branch(orc):
     np.testing.assert_allclose(got, ref, rtol=2e-4, atol=2e-5)
 
 
+def test_single_condition_token_cross_attention_branch(orc):
+    # with one condition token every query's cross-attention weight is 1, so
+    # block 0's cross-attention branch (no gate) adds W_co V_c + b_co with
+    # V_c the value half of the condition projection: pins the K/V split of
+    # that projection, the output projection and the ungated residual
+    s = synth.ModelShape(4, 8, 64, 2, 2, 4, 1, 64, 4, 8)
+    blob = synth.weights_blob(s, 13)
+    for l in range(s.blocks):
+        for name in ("mod_w", "mod_b"):
+            synth.set_weight(blob, s, name, l, 0.0)
+    for name in ("co_w", "co_b"):
+        synth.set_weight(blob, s, name, 1, 0.0)
+    w, ln, tail = _numpy_head_tail(s, blob)
+    m = orc.Model(s, blob)
+    S = np.random.default_rng(8).standard_normal((s.tokens, 8)).astype(np.float32)
+    cond = synth.cond_tokens(s, 1, 9)[0]
+    idx = np.array([0, 21, 50], np.int32)
+    got = m.forward(S, idx, 0.0, m.cond_kv(cond)).astype(np.float64)
+    W = s.width
+    pos = np.stack([orc.pos_embed(s.grid, W, int(i)) for i in idx]).astype(np.float64)
+    x = S[idx].astype(np.float64) @ w("in_w").T + w("in_b") + pos
+    c = synth.bf16_bits_to_f32(np.asarray(cond).reshape(-1)).astype(np.float64)
+    kv = w("ckv_w", 0) @ c + w("ckv_b", 0)
+    y = w("co_w", 0) @ kv[W:] + w("co_b", 0)
+    ref = tail(x + y)
+    np.testing.assert_allclose(got, ref, rtol=2e-4, atol=2e-5)
+
+
 def test_sample_quota_zero_is_plain_euler(tiny, orc):
     # quota 0 at every step must reproduce the uncached sampler exactly
     m, S, cond = tiny["model"], tiny["S"][:1], tiny["cond"][:1]
