@@ -244,6 +244,38 @@ def test_single_condition_token_cross_attention_branch(orc):
     np.testing.assert_allclose(got, ref, rtol=2e-4, atol=2e-5)
 
 
+def test_qk_rmsnorm_invariance(orc):
+    # per-head RMSNorm of Q and K (Supp. Sec. F self-attention): scaling the
+    # query or key projection (rows and bias, by powers of two, exact in
+    # bf16) leaves the block unchanged, while scaling the norm's gain does
+    # not -- pins that both are normalised before the scores, gain after
+    s, blob = _one_branch_model(orc, 2, 14)
+    W = s.width
+    offs, _ = synth.weight_offsets(s)
+    S = np.random.default_rng(9).standard_normal((s.tokens, 8)).astype(np.float32)
+    cond = synth.cond_tokens(s, 1, 4)[0]
+    idx = np.arange(0, s.tokens, 5, dtype=np.int32)
+
+    def run(b):
+        m = orc.Model(s, b)
+        return m.forward(S, idx, 0.0, m.cond_kv(cond)).astype(np.float64)
+
+    def scaled(b, name, lo, hi, f):
+        out = b.copy()
+        off, dims = offs[(name, 0)]
+        cols = dims[1] if len(dims) > 1 else 1
+        seg = synth.bf16_bits_to_f32(out[off + lo * cols:off + hi * cols]) * np.float32(f)
+        out[off + lo * cols:off + hi * cols] = synth.f32_to_bf16_bits(seg)
+        return out
+
+    base = run(blob)
+    for lo, hi, f in ((0, W, 2.0), (W, 2 * W, 4.0)):  # Q rows, K rows
+        b = scaled(scaled(blob, "qkv_w", lo, hi, f), "qkv_b", lo, hi, f)
+        np.testing.assert_allclose(run(b), base, rtol=1e-5, atol=1e-5)
+    assert np.abs(run(scaled(blob, "qn_g", 0, W, 2.0)) - base).max() > 1e-3
+    assert np.abs(run(scaled(blob, "kn_g", 0, W, 2.0)) - base).max() > 1e-3
+
+
 def test_sample_quota_zero_is_plain_euler(tiny, orc):
     # quota 0 at every step must reproduce the uncached sampler exactly
     m, S, cond = tiny["model"], tiny["S"][:1], tiny["cond"][:1]
