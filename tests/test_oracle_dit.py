@@ -362,3 +362,69 @@ def test_modulation_is_linear_of_silu(orc):
         w = synth.weight_view(blob, shape, name + "_w", blk).astype(np.float64)
         b = synth.weight_view(blob, shape, name + "_b", blk).astype(np.float64)
         np.testing.assert_allclose(m.modulation(temb, blk), w @ s + b, rtol=1e-5, atol=1e-6)
+
+
+def test_cross_attention_query_path_multi_token(orc):
+    # block 0's cross-attention branch alone (every modulation zero, so the
+    # gated self-attention and MLP branches add exactly 0; block 1's output
+    # projection zero) with five condition tokens, so the softmax weights
+    # depend on the query: y = W_co softmax_h(q_h K_h^T / sqrt(dh)) V_h + b_co
+    # with q = W_cq (LN(x) g2 + b2) + b_cq and [K | V] = W_ckv c + b_ckv, added
+    # ungated.  LN2's gain and bias are drawn wide so that dropping either,
+    # applying the bias before the gain, projecting x instead of LN2(x) or
+    # swapping the key and value halves moves the output far beyond the
+    # tolerance (checked below against NumPy variants with each mistake).
+    s = synth.ModelShape(4, 8, 64, 2, 2, 4, 5, 64, 4, 8)
+    blob = synth.weights_blob(s, 15)
+    for l in range(s.blocks):
+        for name in ("mod_w", "mod_b"):
+            synth.set_weight(blob, s, name, l, 0.0)
+    for name in ("co_w", "co_b"):
+        synth.set_weight(blob, s, name, 1, 0.0)
+    rng = np.random.default_rng(21)
+    W = s.width
+    synth.set_weight(blob, s, "ln2_g", 0, (1.0 + 0.5 * rng.standard_normal(W)).astype(np.float32))
+    synth.set_weight(blob, s, "ln2_b", 0, (0.5 * rng.standard_normal(W)).astype(np.float32))
+    # a sharper query projection makes the attention weights far from uniform
+    cq = synth.weight_view(blob, s, "cq_w", 0) * np.float32(4.0)
+    synth.set_weight(blob, s, "cq_w", 0, cq)
+    w, ln, tail = _numpy_head_tail(s, blob)
+    m = orc.Model(s, blob)
+    S = rng.standard_normal((s.tokens, 8)).astype(np.float32)
+    cond = synth.cond_tokens(s, 1, 17)[0]
+    idx = np.array([2, 9, 26, 41, 58, 63], np.int32)
+    got = m.forward(S, idx, 0.0, m.cond_kv(cond)).astype(np.float64)
+
+    pos = np.stack([orc.pos_embed(s.grid, W, int(i)) for i in idx]).astype(np.float64)
+    x = S[idx].astype(np.float64) @ w("in_w").T + w("in_b") + pos
+    c = synth.bf16_bits_to_f32(np.asarray(cond).reshape(s.cond_tokens, s.cond_dim)).astype(np.float64)
+    kv = c @ w("ckv_w", 0).T + w("ckv_b", 0)
+    dh = W // s.heads
+
+    def branch(h_in, k_half=0):
+        q = h_in @ w("cq_w", 0).T + w("cq_b", 0)
+        K, V = kv[:, k_half * W:(k_half + 1) * W], kv[:, (1 - k_half) * W:(2 - k_half) * W]
+        o = np.empty_like(q)
+        for hd in range(s.heads):
+            sl = slice(hd * dh, (hd + 1) * dh)
+            sc = q[:, sl] @ K[:, sl].T / np.sqrt(dh)
+            p = np.exp(sc - sc.max(axis=1, keepdims=True))
+            p /= p.sum(axis=1, keepdims=True)
+            o[:, sl] = p @ V[:, sl]
+        return o @ w("co_w", 0).T + w("co_b", 0)
+
+    g2, b2 = w("ln2_g", 0), w("ln2_b", 0)
+    ref = tail(x + branch(ln(x) * g2 + b2))
+    np.testing.assert_allclose(got, ref, rtol=2e-4, atol=2e-5)
+
+    # the pin separates each plausible slip from the right reading
+    scale = np.abs(ref).max()
+    wrong = {
+        "no LN2 bias": ln(x) * g2,
+        "no LN2 gain": ln(x) + b2,
+        "bias before gain": (ln(x) + b2) * g2,
+        "query from x": x,
+    }
+    for what, h_in in wrong.items():
+        assert np.abs(tail(x + branch(h_in)) - ref).max() > 100 * (2e-5 + 2e-4 * scale), what
+    assert np.abs(tail(x + branch(ln(x) * g2 + b2, k_half=1)) - ref).max() > 100 * (2e-5 + 2e-4 * scale)

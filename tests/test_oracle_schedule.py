@@ -99,3 +99,24 @@ def test_tau_literal_reading(orc):
 def test_tau_counter_resets_on_natural_full_step(orc):
     g = orc.TauGate(3, 0)
     assert [g(q) for q in (100, 0, 100, 100, 100)] == [100, 0, 100, 100, 0]
+
+
+def test_phase_table_file_matches_its_generator():
+    # the stored table is exactly what its committed generator writes (50-digit
+    # decimal arithmetic, independent of the oracle), and every Phase-2 value
+    # lies far from an integer compared with fp64 rounding (the closest,
+    # step 8, by 0.038), so the floor is not decided by rounding
+    import importlib.util
+    import io
+    import os
+    here = os.path.join(os.path.dirname(os.path.abspath(__file__)), "golden")
+    spec = importlib.util.spec_from_file_location("make_phase_table_T25",
+                                                  os.path.join(here, "make_phase_table_T25.py"))
+    gen = importlib.util.module_from_spec(spec)
+    spec.loader.exec_module(gen)
+    buf = io.StringIO()
+    gen.main(buf)
+    with open(os.path.join(here, "phase_table_T25.txt")) as f:
+        assert f.read() == buf.getvalue()
+    margins = [m for *_, m in gen.table() if m is not None]
+    assert len(margins) == 13 and min(margins) > 0.03
