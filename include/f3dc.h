@@ -323,7 +323,9 @@ f3dc_status f3dc_forward(f3dc_handle *h, float t, int32_t B, const float *S,
  * partials go to a split-K workspace that this call allocates once per device
  * and keeps for the life of the process; results do not depend on the split
  * (partials are summed in a fixed order), and calls on one device must not
- * overlap.
+ * overlap.  A bounded wait inside the kernel that runs out (F3DC_DEV_TIMEOUT;
+ * the output is then incomplete) is recorded in the device status word that
+ * f3dc_gemm_status reads.
  *   A: device bf16 [M, K] row-major; B: device bf16 [N, K] row-major;
  *   bias: device bf16 [N], nullable; gate: device fp32 [N], nullable;
  *   out: device bf16 [M, N] (BIAS, GELU) or fp32 [M, N] (RESID).
@@ -338,11 +340,13 @@ f3dc_status f3dc_gemm(const void *A, const void *B, const void *bias, const floa
  * device memory through their own pool and forbid side allocations, and
  * latency-critical loops must not enter the driver's allocator; f3dc_gemm,
  * which allocates its split-K workspace on first use per device, serves none
- * of them.  This call computes the same result as f3dc_gemm (same tiling,
- * same split rule, same summation order), with the same arguments and
- * errors, but takes the split-K workspace from a fixed 20 MiB array (plus
- * 4 KiB of counters) compiled into libf3dc; every GPU that loads the library
- * holds that array until the process exits.  It calls no allocation routine.
+ * of them.  This call makes f3dc_gemm's launch decisions (the CTA-pair kernel
+ * for 256-wide tiles without a split, otherwise the single-CTA kernel with
+ * the same split rule and summation order), so its output equals f3dc_gemm's
+ * bit for bit, with the same arguments and errors; but it takes the split-K
+ * workspace from a fixed 20 MiB array (plus 4 KiB of counters) compiled into
+ * libf3dc; every GPU that loads the library holds that array until the
+ * process exits.  It calls no allocation routine.
  *   - The first call on a device resolves the array's device address (with
  *     that device current); make that first call before any stream capture.
  *   - A problem whose split-K partials would exceed 20 MiB is rejected with
@@ -350,12 +354,47 @@ f3dc_status f3dc_gemm(const void *A, const void *B, const void *bias, const floa
  *     SMs) every shape fits, since a split never uses more partial tiles than
  *     the device has SMs.
  *   - All calls share the array and it keeps the previous call's contents:
- *     the call clears the arrival counters on `stream` before its launch, and
- *     calls whose executions overlap on the GPU (different streams, or
- *     different host threads without ordering) race on it.
+ *     a call that splits K clears the arrival counters on `stream` before its
+ *     launch, and calls whose executions overlap on the GPU (different
+ *     streams, or different host threads without ordering) race on it.
+ *   - A bounded wait that runs out is recorded like f3dc_gemm's (read it with
+ *     f3dc_gemm_status).
  * Failures are described by f3dc_last_error(NULL).  Asynchronous on `stream`. */
 f3dc_status f3dc_gemm_noalloc(const void *A, const void *B, const void *bias, const float *gate, void *out,
                               int32_t M, int32_t N, int32_t K, int32_t epilogue, void *stream);
+
+/* Reads and clears the current device's status word of the standalone GEMM
+ * calls (f3dc_gemm, f3dc_gemm_noalloc): F3DC_DEV_* bits recorded by their
+ * kernels since the last read, e.g. F3DC_DEV_TIMEOUT when a split-K arrival
+ * wait ran out and a tile was left unwritten.  Synchronizes the device first.
+ * The word is a static device variable of the library: this call allocates
+ * nothing.  Failures are described by f3dc_last_error(NULL). */
+f3dc_status f3dc_gemm_status(uint32_t *status_out);
+
+/* ---------------------------------------------------------------------- */
+/* Fault injection (tests of the failure paths).                           */
+/* ---------------------------------------------------------------------- */
+
+/* Process-wide, host-side fault injection for tests; off by default.  Nothing
+ * here faults, traps or hangs a GPU.  Not thread-safe: set it while no other
+ * thread calls the library.
+ *   fail_alloc_at: f3dc_create's device allocation number fail_alloc_at
+ *     (counted from 0 in each call) is reported as failed without being
+ *     attempted, so f3dc_create frees what it holds and returns F3DC_ERR_OOM;
+ *     -1 turns it off.
+ *   gemm_missing_arrivals, gemm_wait_ns: the split-K arrival wait of f3dc_gemm
+ *     expects this many arrivals beyond the splits that exist (arrivals no CTA
+ *     makes) and gives up after gemm_wait_ns nanoseconds (0: the default 1 s);
+ *     the kernel then records F3DC_DEV_TIMEOUT (read with f3dc_gemm_status),
+ *     leaves the waiting tiles unwritten and returns.  0 turns it off. */
+typedef struct f3dc_fault_injection {
+    int32_t fail_alloc_at;
+    int32_t gemm_missing_arrivals;
+    int64_t gemm_wait_ns;
+} f3dc_fault_injection;
+
+/* Sets the fault injection (NULL: all off).  Host only. */
+f3dc_status f3dc_set_fault_injection(const f3dc_fault_injection *fi);
 
 /* Single-sequence multi-head attention softmax(q k^T / sqrt(dh)) v with the
  * tensor-core flash kernel.

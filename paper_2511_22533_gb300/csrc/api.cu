@@ -254,6 +254,12 @@ struct Profiler {
 
 void f3dc::set_host_error(const std::string &msg) { g_last_error = msg; }
 
+f3dc::FaultInjection &f3dc::fault_injection()
+{
+    static FaultInjection fi;
+    return fi;
+}
+
 struct f3dc_handle {
     f3dc_config cfg;
     int N = 0, W = 0, Wm = 0, H = 0, dh = 0, L = 0, Nc = 0, Dc = 0, G = 0, T = 0;
@@ -403,9 +409,14 @@ f3dc_status prof_drain(f3dc_handle *h, cudaStream_t s)
     return F3DC_OK;
 }
 
+// f3dc_create's device allocations, numbered from 0 per call (fault injection)
+int g_alloc_no = 0;
+
 template <typename T>
 cudaError_t dalloc(T **p, size_t count)
 {
+    const FaultInjection &fi = fault_injection();
+    if (fi.fail_alloc_at >= 0 && g_alloc_no++ == fi.fail_alloc_at) return cudaErrorMemoryAllocation;
     return cudaMalloc(reinterpret_cast<void **>(p), count * sizeof(T) + 256);
 }
 
@@ -783,6 +794,7 @@ f3dc_status f3dc_create(const f3dc_config *cfg, const f3dc_weights *w, void *str
     }
 
     const size_t R = h->max_rows, W = h->W, N = h->N;
+    g_alloc_no = 0;
     CKC(dalloc(&h->wblob, lay.total));
     CKC(cudaMemcpyAsync(h->wblob, w->blob, lay.total * sizeof(bf16), cudaMemcpyDeviceToDevice, s));
     // modulation weights of every block and of the final layer, repacked into
@@ -1378,6 +1390,9 @@ f3dc_status f3dc_gemm(const void *A, const void *B, const void *bias, const floa
     p.ldo = N;
     p.bias = reinterpret_cast<const bf16 *>(bias);
     p.gate = gate;
+    // a bounded wait that runs out is recorded here (read by f3dc_gemm_status)
+    p.err = gemm_status_word();
+    if (!p.err) return fail(nullptr, F3DC_ERR_CUDA, "cannot resolve the GEMM status word");
     const int tiles = p.m_tiles * (N / bn);
     const int epi = epilogue == F3DC_EPI_BIAS ? kEpiBias : (epilogue == F3DC_EPI_GELU ? kEpiGelu : kEpiResid);
     cudaStream_t s = (cudaStream_t)stream;
@@ -1387,7 +1402,7 @@ f3dc_status f3dc_gemm(const void *A, const void *B, const void *bias, const floa
         return F3DC_OK;
     }
     // split-K workspace: allocated once per device on first use and kept for
-    // the life of the process (its counters return to 0 after every launch)
+    // the life of the process
     static std::mutex ws_lock;
     static std::vector<std::pair<int, void *>> ws_per_device;
     void *ws = nullptr;
@@ -1405,7 +1420,28 @@ f3dc_status f3dc_gemm(const void *A, const void *B, const void *bias, const floa
     p.ws = reinterpret_cast<float *>(ws);
     p.counters = reinterpret_cast<int32_t *>(reinterpret_cast<char *>(ws) + gemm_ws_bytes(256, sms));
     p.ws_units = sms;
+    p.split_extra = fault_injection().gemm_missing_arrivals;
+    p.split_wait_ns = fault_injection().gemm_wait_ns;
+    // a launch whose split wait ran out leaves its tile counters raised: they
+    // start at zero for every launch
+    CK(cudaMemsetAsync(p.counters, 0, kGemmMaxCounterTiles * sizeof(int32_t), s));
     CK(launch_gemm(&ta, &tb, p, epi, bn, gemm_grid(tiles, sms), s));
+    return F3DC_OK;
+}
+
+f3dc_status f3dc_set_fault_injection(const f3dc_fault_injection *fi)
+{
+    FaultInjection &f = fault_injection();
+    if (!fi) {
+        f = FaultInjection();
+        return F3DC_OK;
+    }
+    if (fi->fail_alloc_at < -1 || fi->gemm_missing_arrivals < 0 || fi->gemm_missing_arrivals > 1024 ||
+        fi->gemm_wait_ns < 0)
+        return fail(nullptr, F3DC_ERR_INVALID_ARG, "fault injection: values out of range");
+    f.fail_alloc_at = fi->fail_alloc_at;
+    f.gemm_missing_arrivals = fi->gemm_missing_arrivals;
+    f.gemm_wait_ns = (uint64_t)fi->gemm_wait_ns;
     return F3DC_OK;
 }
 

@@ -539,8 +539,9 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
                 atomicAdd(p.counters + tile, 1);
                 int ok = 1;
                 const uint64_t t0 = globaltimer();
-                while (*reinterpret_cast<volatile int32_t *>(p.counters + tile) < U.splits) {
-                    if (*abort_flag || globaltimer() - t0 > kWaitLimitNs) {
+                const uint64_t limit = p.split_wait_ns ? p.split_wait_ns : kWaitLimitNs;
+                while (*reinterpret_cast<volatile int32_t *>(p.counters + tile) < U.splits + p.split_extra) {
+                    if (*abort_flag || globaltimer() - t0 > limit) {
                         *abort_flag = 1;
                         raise_error(p.err, kDevTimeout);
                         ok = 0;

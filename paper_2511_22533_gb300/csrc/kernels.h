@@ -155,6 +155,11 @@ struct GemmParams {
     // bn = 256 without a workspace: when the device-side tile count of
     // 256-wide tiles is below this, the kernel runs 128-wide tiles (0: never)
     int narrow_below;
+    // fault injection (tests of the failure path; 0 in normal use): the
+    // split-K arrival wait expects split_extra arrivals beyond the splits
+    // that exist, and gives up after split_wait_ns (0: kWaitLimitNs)
+    int split_extra;
+    uint64_t split_wait_ns;
     uint32_t *err;
 };
 // bn in {64, 128, 256}.  ta: A [M, K] in boxes of 128 rows x 64 columns; tb:
@@ -249,6 +254,23 @@ size_t attn_smem_bytes(int dh);
 // ------------------------------------------------------------ host helpers
 // Records the message f3dc_last_error(NULL) returns on this thread.
 void set_host_error(const std::string &msg);
+
+// Host-side fault injection for the tests of the failure paths (process
+// wide; f3dc_set_fault_injection).  Nothing here faults a GPU: an allocation
+// is reported as failed without being attempted, and the GEMM's split-K wait
+// is given an arrival no CTA makes, so its bounded wait runs out.
+struct FaultInjection {
+    int fail_alloc_at = -1;        // f3dc_create's n-th device allocation fails (-1: off)
+    int gemm_missing_arrivals = 0; // split-K arrivals the standalone GEMM's wait also expects
+    uint64_t gemm_wait_ns = 0;     // that wait's limit (0: the default)
+};
+FaultInjection &fault_injection();
+
+// Device address of the current device's status word of the standalone GEMM
+// calls (f3dc_gemm, f3dc_gemm_noalloc; read by f3dc_gemm_status), or null if
+// it cannot be resolved.  The word is a static device variable, not an
+// allocation.
+uint32_t *gemm_status_word();
 
 // 2-D bf16 tensor map over a row-major [rows, cols] matrix with leading
 // dimension ld (elements), box [box_rows, box_cols], 128B (box_cols = 64) or

@@ -50,6 +50,10 @@ class Weights(C.Structure):
     _fields_ = [("layout_version", C.c_int32), ("blob", C.c_void_p), ("blob_elems", C.c_size_t)]
 
 
+class FaultInjection(C.Structure):
+    _fields_ = [("fail_alloc_at", C.c_int32), ("gemm_missing_arrivals", C.c_int32), ("gemm_wait_ns", C.c_int64)]
+
+
 _lock = threading.Lock()
 _lib = None
 _vp, _i32p, _f32p, _f64p, _u32p = C.c_void_p, C.POINTER(C.c_int32), C.POINTER(C.c_float), C.POINTER(
@@ -94,6 +98,8 @@ def lib():
                 "f3dc_gemm": ([_vp, _vp, _vp, _vp, _vp, C.c_int32, C.c_int32, C.c_int32, C.c_int32, _vp], C.c_int),
                 "f3dc_gemm_noalloc": ([_vp, _vp, _vp, _vp, _vp, C.c_int32, C.c_int32, C.c_int32, C.c_int32, _vp],
                                       C.c_int),
+                "f3dc_gemm_status": ([_u32p], C.c_int),
+                "f3dc_set_fault_injection": ([C.POINTER(FaultInjection)], C.c_int),
                 "f3dc_attention": ([_vp, C.c_int32, _vp, _vp, C.c_int32, _vp, C.c_int32, C.c_int32, C.c_int32,
                                     C.c_int32, _vp], C.c_int),
             }
@@ -282,6 +288,21 @@ def gemm_noalloc(A, Bw, bias, gate, out, M, N, K, epilogue, stream=None):
     """f3dc_gemm without any allocation (split-K scratch in a static array)."""
     _check(lib().f3dc_gemm_noalloc(_ptr(A), _ptr(Bw), _ptr(bias), _ptr(gate), _ptr(out), M, N, K, epilogue,
                                    _stream(stream)))
+
+
+def set_fault_injection(fail_alloc_at=-1, gemm_missing_arrivals=0, gemm_wait_ns=0):
+    """Test-only, host-side fault injection (see f3dc_set_fault_injection);
+    called with no arguments it turns everything off."""
+    fi = FaultInjection(fail_alloc_at, gemm_missing_arrivals, gemm_wait_ns)
+    _check(lib().f3dc_set_fault_injection(C.byref(fi)))
+
+
+def gemm_status() -> int:
+    """Reads and clears the current device's status word of the standalone
+    GEMM calls (synchronizes the device)."""
+    v = C.c_uint32(0)
+    _check(lib().f3dc_gemm_status(C.byref(v)))
+    return v.value
 
 
 def attention(q, ldq, k, v, ldkv, out, nq, nk, heads, dh, stream=None):

@@ -138,3 +138,15 @@ def test_fit_mu_rejects_bad_arguments(L):
         f3dc.fit_mu(np.ones((2, 25)), k_lo=10, k_hi=5)
     with pytest.raises(f3dc.F3dcError):
         f3dc.fit_mu(np.ones((2, 25)), min_frac=1.5)
+
+
+def test_fault_injection_argument_checks():
+    # host only: out-of-range settings are refused, valid ones and "off" accepted
+    for bad in [dict(fail_alloc_at=-2), dict(gemm_missing_arrivals=-1), dict(gemm_missing_arrivals=5000),
+                dict(gemm_wait_ns=-1)]:
+        with pytest.raises(f3dc.F3dcError) as e:
+            f3dc.set_fault_injection(**bad)
+        assert e.value.status == 1
+    f3dc.set_fault_injection(fail_alloc_at=3, gemm_missing_arrivals=1, gemm_wait_ns=1000)
+    f3dc.set_fault_injection()
+    assert f3dc.lib().f3dc_set_fault_injection(None) == 0
