@@ -45,3 +45,68 @@ def test_attention_rows_beyond_nq_untouched():
     torch.cuda.synchronize()
     assert torch.all(out[nq:] == 3.0)
     assert torch.isfinite(out[:nq].float()).all()
+
+
+def _rescale_case(nq, nk, H, dh, seed):
+    """Queries and keys along one direction u per head (entries +-1) so that
+    each row's scores are set per key tile.  The first two tiles (one per
+    parity) hold keys of strength 1; tile j >= 2 holds keys one strength step
+    above the previous tile of its parity -- all its keys, except in the last
+    tile of each parity, which holds a single such key.  A step is worth
+    8.4-9.3 log2 units of scaled score for query strengths in [0.9, 1], just
+    past the kernel's 2^8 margin, so each parity raises its reference max
+    (and rescales O and l in place) at every later tile, while the full tiles
+    before a parity's last one keep a visible share of the softmax weight;
+    the last tile is ragged."""
+    g = np.random.default_rng(seed)
+    W = H * dh
+    u = np.where(g.random((H, dh)) < 0.5, -1.0, 1.0)
+    c = g.uniform(0.9, 1.0, nq)                        # per-row query strength
+    q = np.einsum("r,hd->rhd", c, u).reshape(nq, W) + 0.02 * g.standard_normal((nq, W))
+    step = 8.85 / (0.95 * np.sqrt(dh) * np.log2(np.e))
+    a = np.full(nk, 1.0)                               # per-key strength
+    nkt = (nk + 127) // 128
+    for j in range(2, nkt):
+        lo, hi = 128 * j, min(nk, 128 * j + 128)
+        if j >= nkt - 2:
+            a[lo + (j * 37) % (hi - lo)] = 1.0 + step * (j // 2)
+        else:
+            a[lo:hi] = 1.0 + step * (j // 2)
+    k = np.einsum("j,hd->jhd", a, u).reshape(nk, W) + 0.02 * g.standard_normal((nk, W))
+    v = g.standard_normal((nk, W))
+    return [synth.f32_to_bf16_bits(x.astype(np.float32)) for x in (q, k, v)]
+
+
+@pytest.mark.parametrize("nq,nk,H,dh", [(256, 700, 2, 64), (200, 900, 2, 32), (130, 641, 1, 64)])
+def test_attention_reference_max_raised_in_late_tiles(orc, nq, nk, H, dh):
+    # the kernel keeps a per-row reference max and raises it (rescaling O and
+    # l in TMEM) only when a key tile's max exceeds it by more than 2^8; keys
+    # drawn N(0, 1) never get there, so these cases place the strongest keys
+    # in late tiles of both parities and check the outcome against the
+    # oracle's fp64 softmax attention
+    W = H * dh
+    q, k, v = _rescale_case(nq, nk, H, dh, nq + nk)
+    qf, kf, vf = (synth.bf16_bits_to_f32(x).astype(np.float64) for x in (q, k, v))
+    # the branch is taken: per row and head, every later tile of a parity
+    # beats the previous tile of that parity by more than 8 (log2 units of
+    # scaled score), with a margin for fp32 scores; and the raised-over tiles
+    # still carry a visible share of the softmax weight
+    sc = np.einsum("rhd,jhd->rhj", qf.reshape(nq, H, dh), kf.reshape(nk, H, dh)) * np.log2(np.e) / np.sqrt(dh)
+    nkt = (nk + 127) // 128
+    tmax = np.stack([sc[:, :, 128 * j:min(nk, 128 * j + 128)].max(axis=2) for j in range(nkt)], axis=2)
+    assert nkt >= 4 and np.all(tmax[:, :, 2:] - tmax[:, :, :-2] > 8.2)
+    p = np.exp2(sc - sc.max(axis=2, keepdims=True))
+    p /= p.sum(axis=2, keepdims=True)
+    top = np.argmax(sc, axis=2) // 128  # the tile that holds each row's strongest key
+    rest = 1.0 - np.take_along_axis(np.stack([p[:, :, 128 * j:128 * j + 128].sum(axis=2) for j in range(nkt)], 2),
+                                    top[:, :, None], axis=2)[:, :, 0]
+    assert rest.min() > 0.05
+    out = torch.zeros((nq, W), dtype=torch.bfloat16, device="cuda")
+    kd, vd = dev_bf16(k), dev_bf16(v)
+    f3dc.attention(dev_bf16(q), W, kd, vd, W, out, nq, nk, H, dh)
+    torch.cuda.synchronize()
+    ref = orc.attention(qf.astype(np.float32), kf.astype(np.float32), vf.astype(np.float32), H).astype(np.float64)
+    got = out.float().cpu().numpy()
+    assert np.isfinite(got).all()
+    assert rel_l2(got, ref) < 1e-2
+    assert np.max(np.abs(got - ref)) < 2e-2

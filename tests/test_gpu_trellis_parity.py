@@ -1,0 +1,154 @@
+"""Oracle parity at the configuration the benchmark is quoted on -- the
+TRELLIS-L-shaped transformer at full depth and width (24 blocks, width 1024,
+16 heads, 1374 x 1024 condition; Sec. 4.2 compacted forward, Supp. Sec. F
+block) -- plus the exact dynamic-voxel count of the default decoder (Sec. 4.1
+Eq. 1) and free-running occupancy agreement at TRELLIS width."""
+import numpy as np
+import pytest
+import torch
+
+from gpu_helpers import (VEL_MAX_ABS, VEL_REL_L2, assert_clean, dev_f32, dev_i32, dev_u16, handle_for, host_u16,
+                         max_abs, rel_l2, stored_vel_excess)
+from paper_2511_22533_gb300 import synth
+
+pytestmark = pytest.mark.gpu
+
+SHAPE = synth.SHAPES["trellis_l"]
+
+
+def _forward(h, t, S, idx):
+    N = S.shape[0]
+    a = len(idx)
+    lst = np.zeros((1, N), np.int32)
+    lst[0, :a] = idx
+    v = torch.zeros((1, N, 8), dtype=torch.float32, device="cuda")
+    h.forward(t, 1, dev_f32(S[None]), dev_i32(lst), dev_i32([a]), v)
+    torch.cuda.synchronize()
+    return v.cpu().numpy()[0, :a]
+
+
+@pytest.fixture(scope="module")
+def full(orc):
+    h, blob, cfg = handle_for(SHAPE, max_batch=1, seed=0)
+    m = orc.Model(SHAPE, blob)
+    cond = synth.cond_tokens(SHAPE, 1, 0)
+    kv = m.cond_kv(cond[0])
+    h.set_cond(dev_u16(cond), 1)
+    S = synth.latents(SHAPE, 1, 0)[0]
+    yield dict(h=h, m=m, kv=kv, S=S, blob=blob)
+    h.close()
+
+
+@pytest.mark.parametrize("k,quota", [(6, 3141), (19, 2867)])
+def test_teacher_forced_step_full_depth(orc, full, k, quota):
+    # one cached step of the benchmark at its Phase-2 entry (3141 cached, 955
+    # active) and on a Phase-3 cached step (2867 cached, 1229 active): exact
+    # selection and cached tokens; the fused step's stored velocities and the
+    # forward's fp32 velocities against the oracle's 24-block forward
+    h, m, kv, S = full["h"], full["m"], full["kv"], full["S"]
+    N = SHAPE.tokens
+    hist = synth.velocity_history(16, 8, 1, seed=20 + k)
+    ring = np.zeros((3, 1, N, 8), np.uint16)
+    ring[(k - 1) % 3] = hist[2]
+    ring[(k - 2) % 3] = hist[1]
+    ring_d, S_d = dev_u16(ring), dev_f32(S[None])
+    h.step(k, 1, S_d, ring_d, dev_i32([quota]))
+    torch.cuda.synchronize()
+    assert_clean(h)
+    vt = host_u16(ring_d)[k % 3][0]
+    cached, idx = orc.select(orc.ssc_score(hist[2, 0], hist[1, 0], 0.7), quota)
+    cm = cached.astype(bool)
+    assert len(idx) == N - quota
+    np.testing.assert_array_equal(vt[cm], hist[2, 0][cm])
+    fresh = np.any(vt != hist[2, 0], axis=1)
+    assert not fresh[cm].any()
+    t = orc.time_schedule(SHAPE.steps, 3.0)
+    ref = m.forward(S, idx, float(t[k - 1]), kv).astype(np.float64)
+    got = _forward(h, float(t[k - 1]), S, idx)
+    assert np.isfinite(got).all()
+    assert max_abs(got, ref) < VEL_MAX_ABS, max_abs(got, ref)
+    assert rel_l2(got, ref) < VEL_REL_L2, rel_l2(got, ref)
+    vs = synth.bf16_bits_to_f32(vt[idx])
+    assert stored_vel_excess(vs, synth.bf16_bits_to_f32(synth.f32_to_bf16_bits(ref.astype(np.float32)))) < 0
+    assert rel_l2(vs, ref) < VEL_REL_L2
+    # the Euler update of the step is the oracle's given the stored velocities
+    S_o, vt_o = orc.merge_euler(S, idx, vs, hist[2, 0], float(t[k - 1] - t[k]))
+    np.testing.assert_array_equal(S_d.cpu().numpy()[0], S_o)
+    np.testing.assert_array_equal(vt, vt_o)
+
+
+def test_full_step_all_tokens_full_depth(orc, full):
+    # an uncached (Phase-1) step: all 4096 tokens through all 24 blocks, self-
+    # attention over 4096 keys; every 8th row compared with the oracle
+    h, m, kv, S = full["h"], full["m"], full["kv"], full["S"]
+    idx = np.arange(SHAPE.tokens, dtype=np.int32)
+    t = orc.time_schedule(SHAPE.steps, 3.0)
+    got = _forward(h, float(t[0]), S, idx)
+    ref = m.forward(S, idx, float(t[0]), kv).astype(np.float64)
+    rows = np.arange(0, SHAPE.tokens, 8)
+    assert np.isfinite(got).all()
+    assert max_abs(got[rows], ref[rows]) < VEL_MAX_ABS, max_abs(got[rows], ref[rows])
+    assert rel_l2(got, ref) < VEL_REL_L2, rel_l2(got, ref)
+    assert_clean(h)
+
+
+def test_dynamic_voxels_exact_linear_decoder(orc):
+    # Eq. 1 at the anchor step with the default (linear) stand-in decoder:
+    # the count fused into the merge kernel equals the oracle's XOR count of
+    # the two grids it decodes -- the latents before the step and the GPU's
+    # latents after it -- exactly, for a ragged batch on the 16^3 grid
+    shape = synth.ModelShape(16, 8, 128, 2, 4, 4, 64, 128, 25, 64)
+    B, N = 3, shape.tokens
+    h, blob, _ = handle_for(shape, max_batch=B, seed=3)
+    cond = synth.cond_tokens(shape, B, 3)
+    h.set_cond(dev_u16(cond), B)
+    S = synth.latents(shape, B, 3)
+    offs, _ = synth.weight_offsets(shape)
+    off, dims = offs[("dec_w", -1)]
+    dec = blob[off:off + dims[0] * dims[1]]
+    hist = synth.velocity_history(16, 8, B, seed=4)
+    for k, quotas in ((5, [0, 0, 0]), (9, [3141, 0, 4000])):
+        ring = np.zeros((3, B, N, 8), np.uint16)
+        ring[(k - 1) % 3] = hist[2]
+        ring[(k - 2) % 3] = hist[1]
+        S_d = dev_f32(S)
+        dyn = torch.zeros(B, dtype=torch.int64, device="cuda")
+        h.step(k, B, S_d, dev_u16(ring), dev_i32(quotas), dyn)
+        torch.cuda.synchronize()
+        assert_clean(h)
+        S_new = S_d.cpu().numpy()
+        got = dyn.cpu().numpy()
+        for b in range(B):
+            ref = orc.dynamic_voxels(orc.occupancy(S[b], dec), orc.occupancy(S_new[b], dec))
+            assert got[b] == ref, (k, b, got[b], ref)
+            assert ref > 0
+    h.close()
+
+
+def test_free_running_occupancy_trellis_width(orc):
+    # three independently seeded samples at TRELLIS width (W 1024, 16 heads,
+    # 1374 x 1024 condition, 2 blocks) on the 16^3 grid, six Euler steps: two
+    # full, then 70 % cached (2867 tokens) with the tau rule off; final
+    # occupancy of the linear decoder agrees on >= 99.5 % of the voxels
+    shape = synth.ModelShape(16, 8, 1024, 2, 16, 4, 1374, 1024, 6, 64)
+    B, T = 3, 6
+    h, blob, _ = handle_for(shape, max_batch=B, seed=7, tau=0)
+    m = orc.Model(shape, blob)
+    cond = synth.cond_tokens(shape, B, 7)
+    S = synth.latents(shape, B, 7)
+    qs = np.zeros((T, B), np.int32)
+    qs[2:] = 2867
+    S_d = dev_f32(S)
+    qlog, _ = h.sample(S_d, dev_u16(cond), B, quota_schedule=qs)
+    S_gpu = S_d.cpu().numpy()
+    out = m.sample(S, cond, T=T, quota_schedule=qs, tau=0)
+    np.testing.assert_array_equal(qlog, out["quota"])
+    offs, _ = synth.weight_offsets(shape)
+    off, dims = offs[("dec_w", -1)]
+    dec = blob[off:off + dims[0] * dims[1]]
+    for b in range(B):
+        agree = float(np.mean(orc.occupancy(S_gpu[b], dec) == orc.occupancy(out["S"][b], dec)))
+        assert agree >= 0.995, (b, agree)
+        assert rel_l2(S_gpu[b], out["S"][b]) < 5e-2
+    assert_clean(h)
+    h.close()
