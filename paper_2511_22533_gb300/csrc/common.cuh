@@ -480,4 +480,40 @@ F3DC_DEV float warp_sum(float v)
     return v;
 }
 
+// LayerNorm of one row held by a warp (Supp. Sec. F; eps 1e-6): lane l holds
+// the float4 groups q * 32 + l (q < NV) of the row's W = 128 NV values.  The
+// mean first, then the mean of squared deviations, each summed per lane in
+// q order and then across the warp; every kernel that normalises rows (the
+// LayerNorm kernel, the final layer, the fused LayerNorm of the residual
+// GEMM) uses these two helpers, so their outputs agree bit for bit.
+template <int NV>
+F3DC_DEV void ln_row_stats(const float4 (&v)[NV], int W, float &mean, float &rstd)
+{
+    float s = 0.f;
+#pragma unroll
+    for (int q = 0; q < NV; ++q) s += (v[q].x + v[q].y) + (v[q].z + v[q].w);
+    mean = warp_sum(s) / (float)W;
+    float ss = 0.f;
+#pragma unroll
+    for (int q = 0; q < NV; ++q) {
+        const float a = v[q].x - mean, b = v[q].y - mean, c = v[q].z - mean, d = v[q].w - mean;
+        ss += (a * a + b * b) + (c * c + d * d);
+    }
+    const float var = warp_sum(ss) / (float)W;
+    rstd = rsqrtf(var + 1e-6f);
+}
+
+// (x - mean) rstd mul + add for four columns, packed to bf16 pairs.
+F3DC_DEV uint2 ln_out4(float4 v, float mean, float rstd, float4 mu, float4 ad)
+{
+    const float y0 = (v.x - mean) * rstd * mu.x + ad.x;
+    const float y1 = (v.y - mean) * rstd * mu.y + ad.y;
+    const float y2 = (v.z - mean) * rstd * mu.z + ad.z;
+    const float y3 = (v.w - mean) * rstd * mu.w + ad.w;
+    uint2 pk;
+    pk.x = pack_bf16x2(y0, y1);
+    pk.y = pack_bf16x2(y2, y3);
+    return pk;
+}
+
 }  // namespace f3dc

@@ -127,23 +127,6 @@ __global__ void __launch_bounds__(GatherCfg<NV>::kThreads, GatherCfg<NV>::kThrea
 }
 
 // ------------------------------------------------------------------ K7
-template <int NV>
-F3DC_DEV void row_stats(const float4 (&v)[NV], int W, float &mean, float &rstd)
-{
-    float s = 0.f;
-#pragma unroll
-    for (int q = 0; q < NV; ++q) s += (v[q].x + v[q].y) + (v[q].z + v[q].w);
-    mean = warp_sum(s) / (float)W;
-    float ss = 0.f;
-#pragma unroll
-    for (int q = 0; q < NV; ++q) {
-        const float a = v[q].x - mean, b = v[q].y - mean, c = v[q].z - mean, d = v[q].w - mean;
-        ss += (a * a + b * b) + (c * c + d * d);
-    }
-    const float var = warp_sum(ss) / (float)W;
-    rstd = rsqrtf(var + 1e-6f);
-}
-
 // One warp per row, lane l owning float4 columns q * 32 + l.  The per-column
 // modulation (adaLN scale / shift, or LN gain / bias) is staged in shared
 // memory once per CTA while the first row is in flight, and each warp loads
@@ -195,20 +178,12 @@ __global__ void __launch_bounds__(kRowThreads, 2) k_layernorm(const float *x, in
             for (int q = 0; q < NV; ++q) vn[q] = ld_f4(x + (size_t)rn * W + 4 * (q * 32 + lane));
         }
         float mean, rstd;
-        row_stats<NV>(v, W, mean, rstd);
+        ln_row_stats<NV>(v, W, mean, rstd);
         uint16_t *orow = reinterpret_cast<uint16_t *>(out) + (size_t)r * W;
 #pragma unroll
         for (int q = 0; q < NV; ++q) {
             const int n0 = 4 * (q * 32 + lane);
-            const float4 mu = s_mul[q * 32 + lane], ad = s_add[q * 32 + lane];
-            const float y0 = (v[q].x - mean) * rstd * mu.x + ad.x;
-            const float y1 = (v[q].y - mean) * rstd * mu.y + ad.y;
-            const float y2 = (v[q].z - mean) * rstd * mu.z + ad.z;
-            const float y3 = (v[q].w - mean) * rstd * mu.w + ad.w;
-            uint2 pk;
-            pk.x = pack_bf16x2(y0, y1);
-            pk.y = pack_bf16x2(y2, y3);
-            *reinterpret_cast<uint2 *>(orow + n0) = pk;
+            *reinterpret_cast<uint2 *>(orow + n0) = ln_out4(v[q], mean, rstd, s_mul[q * 32 + lane], s_add[q * 32 + lane]);
         }
         if (rn >= m_rows) break;
         r = rn;
@@ -232,7 +207,7 @@ __global__ void __launch_bounds__(kRowThreads) k_final_layer(const float *x, int
 #pragma unroll
         for (int q = 0; q < NV; ++q) v[q] = ld_f4(xr + 4 * (q * 32 + lane));
         float mean, rstd;
-        row_stats<NV>(v, W, mean, rstd);
+        ln_row_stats<NV>(v, W, mean, rstd);
         float acc[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
 #pragma unroll
         for (int q = 0; q < NV; ++q) {
@@ -263,7 +238,13 @@ __global__ void __launch_bounds__(kRowThreads) k_final_layer(const float *x, int
 }
 
 // ------------------------------------------------------------------ K3
+// Two tokens per thread (256 apart, so a warp's 32 consecutive tokens stay
+// in one sample): the latent, the token's packed row and its cached
+// velocity are loaded for both tokens at once, and only an active token's
+// fresh velocity waits for its row index -- one dependent round trip
+// instead of two.
 constexpr int kMergeThreads = 256;
+constexpr int kMergeTok = 2;
 constexpr int kMaxG = 512;
 
 __global__ void __launch_bounds__(kMergeThreads) k_merge_euler(const MergeArgs a)
@@ -278,72 +259,110 @@ __global__ void __launch_bounds__(kMergeThreads) k_merge_euler(const MergeArgs a
         __syncthreads();
     }
     const size_t total = (size_t)a.B * a.N;
-    const size_t tok = (size_t)blockIdx.x * blockDim.x + threadIdx.x;
-    const bool valid = tok < total;
-    int flips = 0;
-    int b = 0;
-    if (valid) {
-        b = (int)(tok / a.N);
-        float *Sp = a.S + tok * 8;
-        const float4 s0 = ld_f4(Sp), s1 = ld_f4(Sp + 4);
-        const float so[8] = {s0.x, s0.y, s0.z, s0.w, s1.x, s1.y, s1.z, s1.w};
-        const int row = a.row_of_token[tok];
-        uint32_t vb[8];
-        if (row >= 0) {
-            const size_t ru = a.cfg_s != 0.0f ? (size_t)row + (size_t)(a.plan->m_rows / 2) : 0;
-            if (row >= a.max_rows || ru >= (size_t)a.max_rows) {
-                raise_error(a.err, kDevBadIndex);
-                for (int c = 0; c < 8; ++c) vb[c] = 0;
-            } else {
-                const float4 v0 = ld_f4(a.v_active + (size_t)row * 8), v1 = ld_f4(a.v_active + (size_t)row * 8 + 4);
-                float va[8] = {v0.x, v0.y, v0.z, v0.w, v1.x, v1.y, v1.z, v1.w};
-                if (a.cfg_s != 0.0f) {
-                    // guided step: v_u + s (v_c - v_u), the unguided copy's row
-                    // half the plan further (subtract, multiply, add)
-                    const float4 u0 = ld_f4(a.v_active + ru * 8), u1 = ld_f4(a.v_active + ru * 8 + 4);
-                    const float vu[8] = {u0.x, u0.y, u0.z, u0.w, u1.x, u1.y, u1.z, u1.w};
+    const size_t tok0 = (size_t)blockIdx.x * (kMergeThreads * kMergeTok) + threadIdx.x;
+    float so[kMergeTok][8];
+    int row[kMergeTok];
+    uint4 pv[kMergeTok];
 #pragma unroll
-                    for (int c = 0; c < 8; ++c) va[c] = __fadd_rn(vu[c], __fmul_rn(a.cfg_s, __fsub_rn(va[c], vu[c])));
-                }
-#pragma unroll
-                for (int c = 0; c < 8; ++c) vb[c] = f32_to_bf16_bits(va[c]);
-            }
-        } else {  // cached token: reuse the stored velocity bit for bit
-            const uint4 p = *reinterpret_cast<const uint4 *>(a.v_prev1 + tok * 8);
-            const uint32_t pw[4] = {p.x, p.y, p.z, p.w};
-#pragma unroll
-            for (int c = 0; c < 8; ++c) vb[c] = (pw[c >> 1] >> ((c & 1) * 16)) & 0xFFFFu;
+    for (int u = 0; u < kMergeTok; ++u) {
+        const size_t tok = tok0 + (size_t)u * kMergeThreads;
+        row[u] = -1;
+        if (tok < total) {
+            const float4 s0 = ld_f4(a.S + tok * 8), s1 = ld_f4(a.S + tok * 8 + 4);
+            so[u][0] = s0.x; so[u][1] = s0.y; so[u][2] = s0.z; so[u][3] = s0.w;
+            so[u][4] = s1.x; so[u][5] = s1.y; so[u][6] = s1.z; so[u][7] = s1.w;
+            row[u] = a.row_of_token[tok];
+            pv[u] = *reinterpret_cast<const uint4 *>(a.v_prev1 + tok * 8);
         }
-        float sn[8];
+    }
+    const size_t half = a.cfg_s != 0.0f ? (size_t)(a.plan->m_rows / 2) : 0;
+    float va[kMergeTok][8], vu[kMergeTok][8];
+    bool bad[kMergeTok];
 #pragma unroll
-        for (int c = 0; c < 8; ++c) sn[c] = __fsub_rn(so[c], __fmul_rn(a.dt, bf16_bits_to_f32(vb[c])));
-        st_f4(Sp, make_float4(sn[0], sn[1], sn[2], sn[3]));
-        st_f4(Sp + 4, make_float4(sn[4], sn[5], sn[6], sn[7]));
-        uint4 vo;
-        vo.x = vb[0] | (vb[1] << 16);
-        vo.y = vb[2] | (vb[3] << 16);
-        vo.z = vb[4] | (vb[5] << 16);
-        vo.w = vb[6] | (vb[7] << 16);
-        *reinterpret_cast<uint4 *>(a.v_out + tok * 8) = vo;
-        if (count) {
-            for (int j = 0; j < a.G; ++j) {
-                float lo = 0.0f, ln = 0.0f;
-#pragma unroll
-                for (int c = 0; c < 8; ++c) {
-                    lo = __fadd_rn(lo, __fmul_rn(so[c], dec[c * a.G + j]));
-                    ln = __fadd_rn(ln, __fmul_rn(sn[c], dec[c * a.G + j]));
+    for (int u = 0; u < kMergeTok; ++u) {
+        const size_t tok = tok0 + (size_t)u * kMergeThreads;
+        bad[u] = false;
+        if (tok < total && row[u] >= 0) {
+            const size_t ru = a.cfg_s != 0.0f ? (size_t)row[u] + half : 0;
+            if (row[u] >= a.max_rows || ru >= (size_t)a.max_rows) {
+                bad[u] = true;
+            } else {
+                const float4 v0 = ld_f4(a.v_active + (size_t)row[u] * 8), v1 = ld_f4(a.v_active + (size_t)row[u] * 8 + 4);
+                va[u][0] = v0.x; va[u][1] = v0.y; va[u][2] = v0.z; va[u][3] = v0.w;
+                va[u][4] = v1.x; va[u][5] = v1.y; va[u][6] = v1.z; va[u][7] = v1.w;
+                if (a.cfg_s != 0.0f) {
+                    const float4 u0 = ld_f4(a.v_active + ru * 8), u1 = ld_f4(a.v_active + ru * 8 + 4);
+                    vu[u][0] = u0.x; vu[u][1] = u0.y; vu[u][2] = u0.z; vu[u][3] = u0.w;
+                    vu[u][4] = u1.x; vu[u][5] = u1.y; vu[u][6] = u1.z; vu[u][7] = u1.w;
                 }
-                flips += (lo > 0.0f) != (ln > 0.0f);
             }
         }
     }
-    if (count) {
-        // N % 32 == 0 is enforced at create, so a warp never spans two samples
-        int f = flips;
 #pragma unroll
-        for (int o = 16; o > 0; o >>= 1) f += __shfl_xor_sync(0xffffffffu, f, o);
-        if ((threadIdx.x & 31) == 0 && valid && f)
-            atomicAdd(reinterpret_cast<unsigned long long *>(a.dyn + b), (unsigned long long)f);
+    for (int u = 0; u < kMergeTok; ++u) {
+        const size_t tok = tok0 + (size_t)u * kMergeThreads;
+        const bool valid = tok < total;
+        int flips = 0;
+        int b = 0;
+        if (valid) {
+            b = (int)(tok / a.N);
+            uint32_t vb[8];
+            if (row[u] >= 0) {
+                if (bad[u]) {
+                    raise_error(a.err, kDevBadIndex);
+#pragma unroll
+                    for (int c = 0; c < 8; ++c) vb[c] = 0;
+                } else {
+                    float v[8];
+#pragma unroll
+                    for (int c = 0; c < 8; ++c) v[c] = va[u][c];
+                    if (a.cfg_s != 0.0f) {
+                        // guided step: v_u + s (v_c - v_u), the unguided copy's row
+                        // half the plan further (subtract, multiply, add)
+#pragma unroll
+                        for (int c = 0; c < 8; ++c)
+                            v[c] = __fadd_rn(vu[u][c], __fmul_rn(a.cfg_s, __fsub_rn(v[c], vu[u][c])));
+                    }
+#pragma unroll
+                    for (int c = 0; c < 8; ++c) vb[c] = f32_to_bf16_bits(v[c]);
+                }
+            } else {  // cached token: reuse the stored velocity bit for bit
+                const uint32_t pw[4] = {pv[u].x, pv[u].y, pv[u].z, pv[u].w};
+#pragma unroll
+                for (int c = 0; c < 8; ++c) vb[c] = (pw[c >> 1] >> ((c & 1) * 16)) & 0xFFFFu;
+            }
+            float sn[8];
+#pragma unroll
+            for (int c = 0; c < 8; ++c) sn[c] = __fsub_rn(so[u][c], __fmul_rn(a.dt, bf16_bits_to_f32(vb[c])));
+            st_f4(a.S + tok * 8, make_float4(sn[0], sn[1], sn[2], sn[3]));
+            st_f4(a.S + tok * 8 + 4, make_float4(sn[4], sn[5], sn[6], sn[7]));
+            uint4 vo;
+            vo.x = vb[0] | (vb[1] << 16);
+            vo.y = vb[2] | (vb[3] << 16);
+            vo.z = vb[4] | (vb[5] << 16);
+            vo.w = vb[6] | (vb[7] << 16);
+            *reinterpret_cast<uint4 *>(a.v_out + tok * 8) = vo;
+            if (count) {
+                for (int j = 0; j < a.G; ++j) {
+                    float lo = 0.0f, ln = 0.0f;
+#pragma unroll
+                    for (int c = 0; c < 8; ++c) {
+                        lo = __fadd_rn(lo, __fmul_rn(so[u][c], dec[c * a.G + j]));
+                        ln = __fadd_rn(ln, __fmul_rn(sn[c], dec[c * a.G + j]));
+                    }
+                    flips += (lo > 0.0f) != (ln > 0.0f);
+                }
+            }
+        }
+        if (count) {
+            // N % 32 == 0 is enforced at create, so a warp's 32 consecutive
+            // tokens never span two samples
+            int f = flips;
+#pragma unroll
+            for (int o = 16; o > 0; o >>= 1) f += __shfl_xor_sync(0xffffffffu, f, o);
+            if ((threadIdx.x & 31) == 0 && valid && f)
+                atomicAdd(reinterpret_cast<unsigned long long *>(a.dyn + b), (unsigned long long)f);
+        }
     }
 }
 
@@ -560,7 +579,7 @@ cudaError_t launch_merge_euler(const MergeArgs &a, cudaStream_t s)
 {
     if (a.dyn && (a.G > kMaxG || a.N % 32 != 0)) return cudaErrorInvalidValue;
     const size_t total = (size_t)a.B * a.N;
-    const int grid = (int)((total + kMergeThreads - 1) / kMergeThreads);
+    const int grid = (int)((total + kMergeThreads * kMergeTok - 1) / (kMergeThreads * kMergeTok));
     launch_k(k_merge_euler, dim3(grid), dim3(kMergeThreads), 0, s, a);
     return cudaGetLastError();
 }
