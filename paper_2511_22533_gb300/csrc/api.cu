@@ -1112,6 +1112,8 @@ f3dc_status f3dc_sample(f3dc_handle *h, float *S_inout, const void *cond, int32_
                                              h->num_sms, s));
     LAUNCH(KF_TEMB, w_pre, launch_gemv_many(h->temb_all, h->T, W, h->mod_w, h->mod_b, h->mod_all, h->mod_rows, 1, 0,
                                             h->num_sms, s));
+    // each of the three calls above launches one kernel per group of vectors
+    h->launches += (gemv_many_kernels(h->T, 256) - 1) + 2 * (gemv_many_kernels(h->T, W) - 1);
     h->mod_pre = true;
     const f3dc_status st = sample_run(h, S_inout, cond, B, sigma_override, quota_schedule, quota_log, sigma_out, stream);
     h->mod_pre = false;

@@ -611,6 +611,19 @@ cudaError_t launch_gemv(const float *x, int K, const bf16 *w, const bf16 *b, flo
     return launch_gemv_many(x, 1, K, w, b, y, rows, silu_in, silu_out, num_sms, s);
 }
 
+// vectors per launch: 8, 4, 2 or 1, as many as the shared staging holds
+static int gemv_group(int left, int K)
+{
+    return left >= 8 && 8 * K <= kGemvXs ? 8 : (left >= 4 && 4 * K <= kGemvXs ? 4 : (left >= 2 && 2 * K <= kGemvXs ? 2 : 1));
+}
+
+int gemv_many_kernels(int nv, int K)
+{
+    int n = 0;
+    for (int v0 = 0; v0 < nv; v0 += gemv_group(nv - v0, K)) ++n;
+    return n;
+}
+
 cudaError_t launch_gemv_many(const float *x, int nv, int K, const bf16 *w, const bf16 *b, float *y, int rows,
                              int silu_in, int silu_out, int num_sms, cudaStream_t s)
 {
@@ -620,8 +633,7 @@ cudaError_t launch_gemv_many(const float *x, int nv, int K, const bf16 *w, const
     if (grid > num_sms * 2) grid = num_sms * 2;
     // vectors in groups whose inputs fit the shared staging (8, 4, 2 or 1)
     for (int v0 = 0; v0 < nv;) {
-        const int left = nv - v0;
-        const int g = left >= 8 && 8 * K <= kGemvXs ? 8 : (left >= 4 && 4 * K <= kGemvXs ? 4 : (left >= 2 && 2 * K <= kGemvXs ? 2 : 1));
+        const int g = gemv_group(nv - v0, K);
         const float *xg = x + (size_t)v0 * K;
         float *yg = y + (size_t)v0 * rows;
         switch (g) {

@@ -129,6 +129,8 @@ cudaError_t launch_gemv(const float *x, int K, const bf16 *w, const bf16 *b, flo
 // single-vector launch's bit for bit
 cudaError_t launch_gemv_many(const float *x, int nv, int K, const bf16 *w, const bf16 *b, float *y, int rows,
                              int silu_in, int silu_out, int num_sms, cudaStream_t s);
+// kernels one launch_gemv_many call launches (vectors in groups of 8, 4, 2, 1)
+int gemv_many_kernels(int nv, int K);
 
 // ------------------------------------------------------------ GEMM
 enum GemmEpi { kEpiBias = 0, kEpiGelu = 1, kEpiResid = 2, kEpiQKNorm = 3 };
