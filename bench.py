@@ -44,6 +44,14 @@ WORKLOAD = "trellis_l"
 CFG_STRENGTH = 5.0  # guidance strength of the secondary CFG measurement (the work does not depend on it)
 SIGMA = 65536.0
 FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
+# DRAM traffic of the GEMM family, from one ncu capture of the six projections
+# of a 1229-row cached-step block (profiles/k_gemm_pair_cached_step_1229rows.md):
+# 68.9 MB over 6 launches against 67.1 MB of operand bytes.  Valid only for the
+# kernel source it was taken on (sha256 of csrc/k_gemm.cu); null otherwise.
+GEMM_TRAFFIC = {"dram_bytes_per_launch": 68.9e6 / 6, "algorithmic_bytes_per_launch": 67.1e6 / 6,
+                "shape": "QKV, attention out, cross Q, cross out, fc1, fc2 at 1229 active rows, width 1024",
+                "profile": "profiles/k_gemm_pair_cached_step_1229rows.md",
+                "k_gemm_cu_sha256": "1c2cbc85b684b77c0b482c531383b424fd7530a096cd28cbff42e463c0121b2d"}
 
 
 def parse():
@@ -53,6 +61,19 @@ def parse():
     p.add_argument("--warmup", type=int, default=3)
     p.add_argument("--impl", default="f3dc", choices=["f3dc", "reference"])
     return p.parse_args()
+
+
+def gemm_traffic():
+    """The captured GEMM traffic per launch, or None once k_gemm.cu has changed
+    since the counters were taken."""
+    import hashlib
+    path = os.path.join(ROOT, "paper_2511_22533_gb300", "csrc", "k_gemm.cu")
+    try:
+        with open(path, "rb") as f:
+            sha = hashlib.sha256(f.read()).hexdigest()
+    except OSError:
+        return None
+    return GEMM_TRAFFIC if sha == GEMM_TRAFFIC["k_gemm_cu_sha256"] else None
 
 
 def peaks():
@@ -667,6 +688,12 @@ def run_gpu(args):
         achieved = dom["flops"] / (dom["total_ms"] / 1000.0) / 1e12
         roof = {"kernel": dom["name"], "bound": "tensor", "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
                 "frac": achieved / peak, "traffic": None, "peak_source": f"bf16_tflops_sustained ({pk_src})"}
+        gt = gemm_traffic() if dom["name"] == "gemm" else None
+        if gt:
+            roof["traffic"] = gt["dram_bytes_per_launch"]
+            roof["traffic_note"] = (f"ncu dram__bytes_read + write per launch of {gt['shape']} "
+                                    f"({gt['profile']}); algorithmic operand bytes "
+                                    f"{gt['algorithmic_bytes_per_launch']:.4g} per launch")
     else:
         peak = pk["hbm_gbs"]
         achieved = dom["bytes"] / (dom["total_ms"] / 1000.0) / 1e9
