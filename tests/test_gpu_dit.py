@@ -347,3 +347,37 @@ def test_sample_graph_replay_matches_eager(orc):
     np.testing.assert_array_equal(res[0][1], res[1][1])
     assert_clean(c.h)
     c.h.close()
+
+
+def test_step_batch64_32cubed_merge(orc):
+    # the largest step workload of the merge / Euler kernel: 64 samples of the
+    # 32^3 grid (32768 tokens each, half cached), a one-block width-128 model;
+    # selection, cached velocities and the Euler update of every token are
+    # bit-exact with the oracle given the velocities the step stored
+    shape = synth.ModelShape(32, 8, 128, 1, 4, 4, 64, 128, 50, 64)
+    B, N, k = 64, shape.tokens, 8
+    h, blob, _ = handle_for(shape, max_batch=B, seed=9)
+    cond = synth.cond_tokens(shape, 1, 9)
+    h.set_cond(dev_u16(np.ascontiguousarray(np.broadcast_to(cond, (B,) + cond.shape[1:]))), B)
+    hist = synth.velocity_history(32, 8, B, seed=33)
+    ring = np.zeros((3, B, N, 8), np.uint16)
+    ring[(k - 1) % 3], ring[(k - 2) % 3] = hist[2], hist[1]
+    S = synth.latents(shape, B, 9)
+    quotas = np.full(B, N // 2, np.int32)
+    ring_d, S_d = dev_u16(ring), dev_f32(S)
+    h.step(k, B, S_d, ring_d, dev_i32(quotas))
+    torch.cuda.synchronize()
+    assert_clean(h)
+    vt = host_u16(ring_d)[k % 3]
+    S_gpu = S_d.cpu().numpy()
+    t = orc.time_schedule(shape.steps, 3.0)
+    for b in (0, 17, 63):
+        cached, idx = orc.select(orc.ssc_score(hist[2, b], hist[1, b], 0.7), N // 2)
+        cm = cached.astype(bool)
+        np.testing.assert_array_equal(vt[b][cm], hist[2, b][cm])
+        S_o, vt_o = orc.merge_euler(S[b], idx, synth.bf16_bits_to_f32(vt[b][idx]), hist[2, b],
+                                    float(t[k - 1] - t[k]))
+        np.testing.assert_array_equal(vt[b], vt_o)
+        np.testing.assert_array_equal(S_gpu[b], S_o)
+        assert np.isfinite(synth.bf16_bits_to_f32(vt[b])).all()
+    h.close()

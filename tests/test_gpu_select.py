@@ -104,3 +104,15 @@ def test_selection_other_grids(orc, grid, B):
     idx, na, mask = _run(h, hist, qs)
     _check(orc, hist, qs, idx, na, mask)
     h.close()
+
+
+def test_selection_batch64_32cubed(orc):
+    # the largest selection workload: 64 samples of 32768 tokens (the 32^3
+    # grid), quotas 10-90 %, bit-exact on every sample
+    h, _, _ = handle_for(_shape(32), max_batch=64)
+    hist = synth.velocity_history(32, 8, 64, seed=32)
+    N = 32768
+    qs = np.array([int(np.floor(q * N)) for q in np.tile([0.1, 0.3, 0.5, 0.7, 0.9], 13)[:64]], np.int32)
+    idx, na, mask = _run(h, hist, qs)
+    _check(orc, hist, qs, idx, na, mask)
+    h.close()

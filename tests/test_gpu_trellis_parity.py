@@ -152,3 +152,24 @@ def test_free_running_occupancy_trellis_width(orc):
         assert rel_l2(S_gpu[b], out["S"][b]) < 5e-2
     assert_clean(h)
     h.close()
+
+
+def test_scaled_grid_width1024_over_16k_active(orc):
+    # the 32^3 grid (32768 tokens) at TRELLIS width (1024, 16 heads of 64,
+    # 1374 x 1024 condition), 2 blocks, 16384 active tokens: self-attention
+    # over 16384 keys (128 key tiles per work item) against the oracle
+    shape = synth.ModelShape(32, 8, 1024, 2, 16, 4, 1374, 1024, 50, 64)
+    h, blob, _ = handle_for(shape, max_batch=1, seed=10)
+    m = orc.Model(shape, blob)
+    cond = synth.cond_tokens(shape, 1, 10)
+    h.set_cond(dev_u16(cond), 1)
+    S = synth.latents(shape, 1, 10)[0]
+    idx = np.sort(np.random.default_rng(10).choice(shape.tokens, 16384, replace=False)).astype(np.int32)
+    got = _forward(h, 0.6, S, idx)
+    ref = m.forward(S, idx, 0.6, m.cond_kv(cond[0])).astype(np.float64)
+    rows = np.arange(0, len(idx), 16)
+    assert np.isfinite(got).all()
+    assert max_abs(got[rows], ref[rows]) < VEL_MAX_ABS, max_abs(got[rows], ref[rows])
+    assert rel_l2(got, ref) < VEL_REL_L2, rel_l2(got, ref)
+    assert_clean(h)
+    h.close()
