@@ -363,10 +363,11 @@ f3dc_status f3dc_gemm(const void *A, const void *B, const void *bias, const floa
 f3dc_status f3dc_gemm_noalloc(const void *A, const void *B, const void *bias, const float *gate, void *out,
                               int32_t M, int32_t N, int32_t K, int32_t epilogue, void *stream);
 
-/* Reads and clears the current device's status word of the standalone GEMM
- * calls (f3dc_gemm, f3dc_gemm_noalloc): F3DC_DEV_* bits recorded by their
- * kernels since the last read, e.g. F3DC_DEV_TIMEOUT when a split-K arrival
- * wait ran out and a tile was left unwritten.  Synchronizes the device first.
+/* Reads and clears the current device's status word of the standalone
+ * kernel calls (f3dc_gemm, f3dc_gemm_noalloc, f3dc_attention): F3DC_DEV_*
+ * bits recorded by their kernels since the last read, e.g. F3DC_DEV_TIMEOUT
+ * when a bounded wait ran out and part of the output was left unwritten.
+ * Synchronizes the device first.
  * The word is a static device variable of the library: this call allocates
  * nothing.  Failures are described by f3dc_last_error(NULL). */
 f3dc_status f3dc_gemm_status(uint32_t *status_out);
@@ -386,11 +387,17 @@ f3dc_status f3dc_gemm_status(uint32_t *status_out);
  *     expects this many arrivals beyond the splits that exist (arrivals no CTA
  *     makes) and gives up after gemm_wait_ns nanoseconds (0: the default 1 s);
  *     the kernel then records F3DC_DEV_TIMEOUT (read with f3dc_gemm_status),
- *     leaves the waiting tiles unwritten and returns.  0 turns it off. */
+ *     leaves the waiting tiles unwritten and returns.  0 turns it off.
+ *   attn_missing_kv: 1 makes f3dc_attention's first CTA skip the load of the
+ *     last key tile of its first item, so the waits on that tile run out
+ *     (after 1 s); the kernel records F3DC_DEV_TIMEOUT (read with
+ *     f3dc_gemm_status), leaves that CTA's items unwritten and returns.  0
+ *     turns it off. */
 typedef struct f3dc_fault_injection {
     int32_t fail_alloc_at;
     int32_t gemm_missing_arrivals;
     int64_t gemm_wait_ns;
+    int32_t attn_missing_kv;
 } f3dc_fault_injection;
 
 /* Sets the fault injection (NULL: all off).  Host only. */

@@ -1439,11 +1439,12 @@ f3dc_status f3dc_set_fault_injection(const f3dc_fault_injection *fi)
         return F3DC_OK;
     }
     if (fi->fail_alloc_at < -1 || fi->gemm_missing_arrivals < 0 || fi->gemm_missing_arrivals > 1024 ||
-        fi->gemm_wait_ns < 0)
+        fi->gemm_wait_ns < 0 || (fi->attn_missing_kv != 0 && fi->attn_missing_kv != 1))
         return fail(nullptr, F3DC_ERR_INVALID_ARG, "fault injection: values out of range");
     f.fail_alloc_at = fi->fail_alloc_at;
     f.gemm_missing_arrivals = fi->gemm_missing_arrivals;
     f.gemm_wait_ns = (uint64_t)fi->gemm_wait_ns;
+    f.attn_missing_kv = fi->attn_missing_kv;
     return F3DC_OK;
 }
 
@@ -1470,6 +1471,10 @@ f3dc_status f3dc_attention(const void *q, int32_t ldq, const void *k, const void
     p.out = reinterpret_cast<bf16 *>(out);
     p.ldo = heads * dh;
     p.scale_log2 = (float)(1.4426950408889634 / std::sqrt((double)dh));
+    // a bounded wait that runs out is recorded here (read by f3dc_gemm_status)
+    p.err = gemm_status_word();
+    if (!p.err) return fail(nullptr, F3DC_ERR_CUDA, "cannot resolve the status word");
+    p.fault_skip_kv = fault_injection().attn_missing_kv;
     int dev = 0, sms = 0;
     CK(cudaGetDevice(&dev));
     CK(cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev));

@@ -90,6 +90,10 @@ F3DC_DEV Item decode_item(const AttnParams &p, int w)
     return it;
 }
 
+// every lane's outcome, so a warp takes the same branch around its
+// warp-collective TMEM accesses even when a bounded wait gives up in one lane
+F3DC_DEV bool warp_all(bool v) { return __all_sync(0xffffffffu, v); }
+
 F3DC_DEV bool wait_bounded(uint64_t *bar, uint32_t parity, uint64_t ns)
 {
     const uint64_t t0 = globaltimer();
@@ -195,6 +199,11 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
                         ok = false;
                         break;
                     }
+                    // fault injection (tests of the failure path): the last
+                    // key tile of CTA 0's first item is never loaded, so the
+                    // waits on it (and on what follows it) run out while the
+                    // earlier tiles went through, and the kernel aborts
+                    if (p.fault_skip_kv && blockIdx.x == 0 && item_it == 0 && j == nkt - 1) continue;
                     mbar_arrive_expect_tx(&kv_full[s], 2 * Cfg::kTileBytes);
                     tma_load_2d(sK + s * Cfg::kTileBytes, &tmk, p.k_col0 + it.h * DH, it.kv_row0 + j * 128,
                                 &kv_full[s]);
@@ -309,6 +318,7 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
         const uint32_t p_addr = tmem + tl + Cfg::kColP + par * 64;
         uint32_t g = 0, item_it = 0;  // global key-tile counter at the start of the item
         uint32_t s_use = 0;           // s_full[par] completions consumed
+        volatile int *stop_flag = abort_flag + 1;
         // S of an item's first tile of this parity completes s_full[par]
         // (once per item in which the parity has a tile; s_use counts them);
         // S of every later tile t is reported with P V of tile t - 2 on
@@ -326,9 +336,9 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
             for (int j = (int)((par - g) & 1); j < nkt; j += 2) {
                 const uint32_t gt = g + (uint32_t)j;
                 const bool first = j < 2;  // S reported on s_full, else with P V of tile gt - 2
-                if (first ? !mbar_wait(&s_full[par], (s_use++) & 1, abort_flag, p.err)
-                          : !mbar_wait(&kv_empty[(gt - 2) % kKVStages], ((gt - 2) / kKVStages) & 1, abort_flag,
-                                       p.err)) {
+                if (!warp_all(first ? mbar_wait(&s_full[par], (s_use++) & 1, abort_flag, p.err)
+                                    : mbar_wait(&kv_empty[(gt - 2) % kKVStages], ((gt - 2) / kKVStages) & 1,
+                                                abort_flag, p.err))) {
                     ok = false;
                     break;
                 }
@@ -375,7 +385,8 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
                 const float m_use = m_ref == -INFINITY ? 0.f : m_ref;
                 // P_par and O_par: P V of this parity's previous tile must be done
                 if (first && gt >= 2 &&
-                    !mbar_wait(&kv_empty[(gt - 2) % kKVStages], ((gt - 2) / kKVStages) & 1, abort_flag, p.err)) {
+                    !warp_all(mbar_wait(&kv_empty[(gt - 2) % kKVStages], ((gt - 2) / kKVStages) & 1, abort_flag,
+                                        p.err))) {
                     ok = false;
                     break;
                 }
@@ -440,14 +451,19 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
                 g_last = gt;
             }
             g += (uint32_t)nkt;
-            if (!ok) break;
             // every P V of this parity done: read O_par, release it (a parity
-            // without tiles in this item contributes m = -inf, l = 0, O = 0)
+            // without tiles in this item contributes m = -inf, l = 0, O = 0).
+            // After a wait gave up (the kernel is aborting) the warps still go
+            // through the combine's barriers below, with zeros, and leave the
+            // item loop together after it: no warp waits at a named barrier
+            // for one that has left.
             float acc[DH];
 #pragma unroll
             for (int d = 0; d < DH; ++d) acc[d] = 0.f;
-            if (any) {
-                if (!mbar_wait(&kv_empty[g_last % kKVStages], (g_last / kKVStages) & 1, abort_flag, p.err)) break;
+            if (ok && any &&
+                !warp_all(mbar_wait(&kv_empty[g_last % kKVStages], (g_last / kKVStages) & 1, abort_flag, p.err)))
+                ok = false;
+            if (ok && any) {
                 tc_fence_after();
 #pragma unroll
                 for (int d0 = 0; d0 < DH; d0 += 32) {
@@ -499,7 +515,11 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
                     }
                 }
             }
+            // one snapshot of the abort flag, read by every softmax thread
+            // after the barrier, decides for all whether to go on
+            if (threadIdx.x == 64) *stop_flag = *abort_flag;
             asm volatile("bar.sync 1, %0;" ::"n"(kSoftmaxThreads) : "memory");
+            if (*stop_flag) break;
         }
     }
     __syncthreads();

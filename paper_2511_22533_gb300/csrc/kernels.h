@@ -247,6 +247,10 @@ struct AttnParams {
     // > 0: K / V rows [0, kv_prefetch_rows) are complete before the launch
     // (not written by the previous kernel) and are prefetched into L2 first
     int kv_prefetch_rows;
+    // fault injection (tests; 0 in normal use): CTA 0 never loads the last
+    // key tile of its first item, so the waits on it run out and the kernel
+    // aborts cleanly
+    int fault_skip_kv;
     uint32_t *err;
 };
 cudaError_t launch_attention(const CUtensorMap *tq, const CUtensorMap *tk, const CUtensorMap *tv,
@@ -265,11 +269,12 @@ struct FaultInjection {
     int fail_alloc_at = -1;        // f3dc_create's n-th device allocation fails (-1: off)
     int gemm_missing_arrivals = 0; // split-K arrivals the standalone GEMM's wait also expects
     uint64_t gemm_wait_ns = 0;     // that wait's limit (0: the default)
+    int attn_missing_kv = 0;       // f3dc_attention: CTA 0 never loads its first item's last key tile
 };
 FaultInjection &fault_injection();
 
-// Device address of the current device's status word of the standalone GEMM
-// calls (f3dc_gemm, f3dc_gemm_noalloc; read by f3dc_gemm_status), or null if
+// Device address of the current device's status word of the standalone calls
+// (f3dc_gemm, f3dc_gemm_noalloc, f3dc_attention; read by f3dc_gemm_status), or null if
 // it cannot be resolved.  The word is a static device variable, not an
 // allocation.
 uint32_t *gemm_status_word();

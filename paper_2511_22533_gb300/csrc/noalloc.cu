@@ -1,6 +1,7 @@
 // noalloc.cu -- f3dc_gemm_noalloc: the transformer's tcgen05 GEMM for
 // callers that must not allocate device memory, and the device status word
-// of the standalone GEMM calls (f3dc_gemm, f3dc_gemm_noalloc, f3dc_gemm_status).
+// of the standalone kernel calls (f3dc_gemm, f3dc_gemm_noalloc,
+// f3dc_attention; read by f3dc_gemm_status).
 //
 // Some callers cannot call cudaMalloc: code that runs while a CUDA graph is
 // being captured in global mode (allocation calls are illegal there), code
@@ -36,8 +37,9 @@ constexpr size_t kCounterBytes = kGemmMaxCounterTiles * sizeof(int32_t);
 // Every GPU that loads libf3dc holds this array until the process exits.
 static __device__ __align__(256) unsigned char g_gemm_scratch[kPartialBytes + kCounterBytes];
 
-// Status word (F3DC_DEV_* bits) that the standalone GEMM kernels record into
-// (a bounded wait that ran out), sticky until f3dc_gemm_status reads it.
+// Status word (F3DC_DEV_* bits) that the standalone GEMM and attention
+// kernels record into (a bounded wait that ran out), sticky until
+// f3dc_gemm_status reads it.
 // __device__ variables start at zero.
 static __device__ __align__(256) uint32_t g_gemm_status;
 

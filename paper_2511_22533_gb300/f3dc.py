@@ -51,7 +51,8 @@ class Weights(C.Structure):
 
 
 class FaultInjection(C.Structure):
-    _fields_ = [("fail_alloc_at", C.c_int32), ("gemm_missing_arrivals", C.c_int32), ("gemm_wait_ns", C.c_int64)]
+    _fields_ = [("fail_alloc_at", C.c_int32), ("gemm_missing_arrivals", C.c_int32), ("gemm_wait_ns", C.c_int64),
+                ("attn_missing_kv", C.c_int32)]
 
 
 _lock = threading.Lock()
@@ -290,16 +291,16 @@ def gemm_noalloc(A, Bw, bias, gate, out, M, N, K, epilogue, stream=None):
                                    _stream(stream)))
 
 
-def set_fault_injection(fail_alloc_at=-1, gemm_missing_arrivals=0, gemm_wait_ns=0):
+def set_fault_injection(fail_alloc_at=-1, gemm_missing_arrivals=0, gemm_wait_ns=0, attn_missing_kv=0):
     """Test-only, host-side fault injection (see f3dc_set_fault_injection);
     called with no arguments it turns everything off."""
-    fi = FaultInjection(fail_alloc_at, gemm_missing_arrivals, gemm_wait_ns)
+    fi = FaultInjection(fail_alloc_at, gemm_missing_arrivals, gemm_wait_ns, attn_missing_kv)
     _check(lib().f3dc_set_fault_injection(C.byref(fi)))
 
 
 def gemm_status() -> int:
     """Reads and clears the current device's status word of the standalone
-    GEMM calls (synchronizes the device)."""
+    kernel calls: GEMMs and attention (synchronizes the device)."""
     v = C.c_uint32(0)
     _check(lib().f3dc_gemm_status(C.byref(v)))
     return v.value

@@ -143,10 +143,10 @@ def test_fit_mu_rejects_bad_arguments(L):
 def test_fault_injection_argument_checks():
     # host only: out-of-range settings are refused, valid ones and "off" accepted
     for bad in [dict(fail_alloc_at=-2), dict(gemm_missing_arrivals=-1), dict(gemm_missing_arrivals=5000),
-                dict(gemm_wait_ns=-1)]:
+                dict(gemm_wait_ns=-1), dict(attn_missing_kv=2)]:
         with pytest.raises(f3dc.F3dcError) as e:
             f3dc.set_fault_injection(**bad)
         assert e.value.status == 1
-    f3dc.set_fault_injection(fail_alloc_at=3, gemm_missing_arrivals=1, gemm_wait_ns=1000)
+    f3dc.set_fault_injection(fail_alloc_at=3, gemm_missing_arrivals=1, gemm_wait_ns=1000, attn_missing_kv=1)
     f3dc.set_fault_injection()
     assert f3dc.lib().f3dc_set_fault_injection(None) == 0

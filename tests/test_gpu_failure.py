@@ -86,3 +86,36 @@ def test_create_reports_oom_and_frees(n):
     # what the failed calls allocated was freed (driver granularity aside)
     assert free0 - torch.cuda.mem_get_info()[0] < 8 << 20
     _tiny_step_clean()
+
+
+def test_attention_wait_runs_out_and_is_reported(orc):
+    # the attention kernel's first CTA is told to skip the load of its first
+    # item's last key tile (the earlier tiles go through): the MMA issuer's and the softmax warps' bounded waits on it run
+    # out (1 s), every warp leaves the work loop together, the kernel returns
+    # and the timeout is reported; the next call computes the right result
+    nq, nk, H, dh = 256, 512, 2, 64
+    W = H * dh
+    g = np.random.default_rng(3)
+    q = synth.f32_to_bf16_bits(g.standard_normal((nq, W)).astype(np.float32))
+    kv = synth.f32_to_bf16_bits(g.standard_normal((nk, 2 * W)).astype(np.float32))
+    qd, kvd = dev_bf16(q), dev_bf16(kv)
+    out = torch.zeros((nq, W), dtype=torch.bfloat16, device="cuda")
+    assert f3dc.gemm_status() == 0
+    f3dc.set_fault_injection(attn_missing_kv=1)
+    try:
+        t0 = time.perf_counter()
+        f3dc.attention(qd, W, kvd, kvd[:, W:], 2 * W, out, nq, nk, H, dh)
+        st = f3dc.gemm_status()
+        elapsed = time.perf_counter() - t0
+    finally:
+        f3dc.set_fault_injection()
+    assert st & TIMEOUT, st
+    assert elapsed < 10.0
+    out.zero_()
+    f3dc.attention(qd, W, kvd, kvd[:, W:], 2 * W, out, nq, nk, H, dh)
+    assert f3dc.gemm_status() == 0
+    kf = synth.bf16_bits_to_f32(kv)
+    ref = orc.attention(synth.bf16_bits_to_f32(q), kf[:, :W], kf[:, W:], H).astype(np.float64)
+    got = out.float().cpu().numpy()
+    assert np.max(np.abs(got - ref)) < 2e-2
+    _tiny_step_clean()
