@@ -11,7 +11,7 @@
 //   warp 0     TMA producer: Q tile once per item, K / V tiles of 128 keys
 //              into a 4-deep ring
 //   warp 1     TMEM allocator + tcgen05.mma issuer (the whole warp runs the
-//              loop and votes on every barrier outcome; lane 0 issues):
+//              loop and votes on every barrier outcome; elect.sync issues):
 //                S_j = Q K_j^T     (M=128, N=128, K=dh)  -> TMEM S[j%2]
 //                O_e += P_j V_j    (M=128, N=dh, K=128)  -> TMEM O_e, e = j%2,
 //                                   with P_j read from TMEM P_e
@@ -27,7 +27,11 @@
 //              O_e stays in TMEM for the whole item; the reference max m is
 //              only raised (and O_e, l rescaled in place) when a tile's max
 //              exceeds it by more than 2^8, so most tiles need no O traffic.
-//              The two parities of a row are combined once per work item.
+//              The two parities of a row are combined once per work item:
+//              the parity that finished first leaves its (m, l, O) in shared
+//              memory (mbarrier hand-over per lane quarter) and moves on to
+//              the next item's first tile, while the other combines and
+//              stores, so no item boundary stalls both.
 //              Because the two warps of an SM sub-partition work on
 //              different tiles, one warp's TMEM load, maximum and barrier
 //              phases overlap the other's exponents instead of leaving the
@@ -103,12 +107,18 @@ F3DC_DEV bool wait_bounded(uint64_t *bar, uint32_t parity, uint64_t ns)
     return true;
 }
 
-// tcgen05 issue from a converged warp (every lane runs the issuer's loop, so
-// its descriptors stay warp-uniform); lane 0 issues
+// tcgen05 issue from a converged warp: every lane runs the issuer's loop and
+// elect.sync picks the issuing lane inside each instruction's asm (the same
+// lane every time: the warp is converged and the member mask full, so the
+// commits track the MMAs of the thread that issued them).  Measured in
+// isolation, this form issues the tile's 12 MMAs in ~525 cycles against
+// ~580 for a loop run by lane 0 alone, and keeps ~945 cycles (lane 0 alone:
+// ~2600) when two warps busy with FMAs share the issuer's SM sub-partition,
+// as the softmax warps do here.
 F3DC_DEV void mma_ss_w(uint32_t d, uint64_t a, uint64_t b, uint32_t id, uint32_t acc)
 {
     asm volatile(
-        "{\n .reg .pred p, e;\n .reg .u32 l;\n mov.u32 l, %%laneid;\n setp.eq.u32 e, l, 0;\n"
+        "{\n .reg .pred p, e;\n elect.sync _|e, 0xffffffff;\n"
         " setp.ne.b32 p, %4, 0;\n @e tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n}\n" ::"r"(d),
         "l"(a), "l"(b), "r"(id), "r"(acc)
         : "memory");
@@ -116,7 +126,7 @@ F3DC_DEV void mma_ss_w(uint32_t d, uint64_t a, uint64_t b, uint32_t id, uint32_t
 F3DC_DEV void mma_ts_w(uint32_t d, uint32_t a, uint64_t b, uint32_t id, uint32_t acc)
 {
     asm volatile(
-        "{\n .reg .pred p, e;\n .reg .u32 l;\n mov.u32 l, %%laneid;\n setp.eq.u32 e, l, 0;\n"
+        "{\n .reg .pred p, e;\n elect.sync _|e, 0xffffffff;\n"
         " setp.ne.b32 p, %4, 0;\n @e tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], %2, %3, p;\n}\n" ::"r"(d),
         "r"(a), "l"(b), "r"(id), "r"(acc)
         : "memory");
@@ -124,9 +134,37 @@ F3DC_DEV void mma_ts_w(uint32_t d, uint32_t a, uint64_t b, uint32_t id, uint32_t
 F3DC_DEV void commit_w(uint64_t *bar)
 {
     asm volatile(
-        "{\n .reg .pred e;\n .reg .u32 l;\n mov.u32 l, %%laneid;\n setp.eq.u32 e, l, 0;\n"
+        "{\n .reg .pred e;\n elect.sync _|e, 0xffffffff;\n"
         " @e tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];\n}\n" ::"r"(smem_u32(bar))
         : "memory");
+}
+
+// One output row of the end-of-item combine, in parity order whichever
+// parity combines: O = (O_0 a_0 + O_1 a_1) / l with a_e = 2^(m_e - m); `acc`
+// is the combining thread's own O (parity 1's when SWAP), the other parity's
+// row is read from its hand-over slot (float4 d4 at d4 ^ (row % (DH / 4))).
+template <int DH, bool SWAP>
+F3DC_DEV void combine_row(const float (&acc)[DH], const float4 *slot, int row, float a0, float a1, float inv,
+                          uint4 *dst)
+{
+    constexpr int kV4 = DH / 4;
+#pragma unroll
+    for (int d = 0; d < DH; d += 8) {
+        const float4 b0 = slot[(d / 4) ^ (row & (kV4 - 1))], b1 = slot[(d / 4 + 1) ^ (row & (kV4 - 1))];
+        const float ob[8] = {b0.x, b0.y, b0.z, b0.w, b1.x, b1.y, b1.z, b1.w};
+        float o[8];
+#pragma unroll
+        for (int e = 0; e < 8; ++e) {
+            const float o0 = SWAP ? ob[e] : acc[d + e], o1 = SWAP ? acc[d + e] : ob[e];
+            o[e] = __fmul_rn(__fmaf_rn(o0, a0, __fmul_rn(o1, a1)), inv);
+        }
+        uint4 u;
+        u.x = pack_bf16x2(o[0], o[1]);
+        u.y = pack_bf16x2(o[2], o[3]);
+        u.z = pack_bf16x2(o[4], o[5]);
+        u.w = pack_bf16x2(o[6], o[7]);
+        dst[d / 8] = u;
+    }
 }
 
 template <int DH>
@@ -142,7 +180,8 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
     uint8_t *sQ = smem;
     uint8_t *sK = sQ + 2 * Cfg::kTileBytes;
     uint8_t *sV = sK + kKVStages * Cfg::kTileBytes;
-    // the end-of-item combine hands parity 1's O and (m, l) to parity 0
+    // the end-of-item hand-over: the parity that finishes an item first
+    // leaves its O and (m, l) here for the other one, which combines
     float *sComb = reinterpret_cast<float *>(sV + kKVStages * Cfg::kTileBytes);
     uint64_t *bars = reinterpret_cast<uint64_t *>(reinterpret_cast<uint8_t *>(sComb) + Cfg::kCombineBytes);
     float2 *sML = reinterpret_cast<float2 *>(reinterpret_cast<uint8_t *>(bars) + 512);
@@ -157,7 +196,10 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
     uint64_t *s_full = kv_empty + kKVStages, *p_full = s_full + 2;
     uint64_t *o_free = p_full + 2;
     uint64_t *drain = o_free + 1;
-    uint32_t *tmem_holder = reinterpret_cast<uint32_t *>(drain + 1);
+    // end-of-item hand-over of one parity's (m, l, O) to the other, per TMEM
+    // lane quarter (the softmax section explains the protocol)
+    uint64_t *comb_full = drain + 1, *comb_free = comb_full + 4;
+    uint32_t *tmem_holder = reinterpret_cast<uint32_t *>(comb_free + 4);
     volatile int *abort_flag = reinterpret_cast<volatile int *>(tmem_holder + 1);
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -178,6 +220,10 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
         }
         mbar_init(o_free, kSoftmaxWarps);
         mbar_init(drain, 1);
+        for (int q = 0; q < 4; ++q) {  // one arrival per thread of the quarter's warp
+            mbar_init(&comb_full[q], 32);
+            mbar_init(&comb_free[q], 32);
+        }
         *abort_flag = 0;
         fence_mbar_init();
     }
@@ -245,9 +291,8 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
         // each tile tests its two barriers back to back (one exposed
         // latency) and takes the bounded wait only if a test fails; the
         // steady-state loop carries no other branches.  Every lane runs the
-        // loop (a converged warp keeps the descriptors warp-uniform, which
-        // measured 1-3 % faster than a lane-0-only loop) and takes each
-        // barrier outcome as a warp vote.
+        // loop (a converged warp keeps the descriptors warp-uniform) and
+        // takes each barrier outcome as a warp vote.
         {
             constexpr uint32_t idesc_s = make_idesc_bf16(128, 128, 0, 0);
             constexpr uint32_t idesc_o = make_idesc_bf16(128, DH, 0, 1);
@@ -348,7 +393,7 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
         const uint32_t p_addr = tmem + tl + Cfg::kColP + par * 64;
         uint32_t g = 0, item_it = 0;  // global key-tile counter at the start of the item
         uint32_t s_use = 0;           // s_full[par] completions consumed
-        volatile int *stop_flag = abort_flag + 1;
+        uint32_t item_k = 0;          // items finished (hand-over barrier phases)
         // S of an item's first tile of this parity completes s_full[par]
         // (once per item in which the parity has a tile; s_use counts them);
         // S of every later tile t is reported with P V of tile t - 2 on
@@ -480,13 +525,14 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
                 any = true;
                 g_last = gt;
             }
+            // the parity of the item's last tile combines and stores the
+            // item; the other one finished a tile earlier and only hands over
+            // its (m, l, O), then goes on to the next item's first tile (which
+            // is its own: tiles alternate parity across items too)
+            const bool combiner = ((g + (uint32_t)nkt - 1u) & 1u) == (uint32_t)par;
             g += (uint32_t)nkt;
             // every P V of this parity done: read O_par, release it (a parity
-            // without tiles in this item contributes m = -inf, l = 0, O = 0).
-            // After a wait gave up (the kernel is aborting) the warps still go
-            // through the combine's barriers below, with zeros, and leave the
-            // item loop together after it: no warp waits at a named barrier
-            // for one that has left.
+            // without tiles in this item contributes m = -inf, l = 0, O = 0)
             float acc[DH];
 #pragma unroll
             for (int d = 0; d < DH; ++d) acc[d] = 0.f;
@@ -507,56 +553,53 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
             tc_fence_before();
             __syncwarp();
             if (lane == 0) mbar_arrive(o_free);
-            // combine the two parities of each row:
-            // O = (O_0 2^(m_0-m) + O_1 2^(m_1-m)) / (l_0 2^(m_0-m) + l_1 2^(m_1-m))
-            // parity 1's O: float4 d4 of row r at r * DH + 4 (d4 ^ (r % (DH / 4))),
-            // so a warp's row-per-lane accesses hit distinct banks
-            constexpr int kV4 = DH / 4;
-            float4 *mine = reinterpret_cast<float4 *>(sComb + row * DH);
-            if (par == 1) {
+            // Hand-over through shared memory, per TMEM lane quarter q (one
+            // warp of each parity): comb_full[q] completes once per item when
+            // the other parity's 32 rows are written, comb_free[q] once per
+            // item when the combiner has read them (so the next item's
+            // writer may overwrite them).  float4 d4 of row r sits at
+            // r * DH + 4 (d4 ^ (r % (DH / 4))), so a warp's row-per-lane
+            // accesses hit distinct banks.  Every wait is bounded; after one
+            // gave up (the kernel is aborting) the warp leaves the item loop.
+            const uint32_t ph = item_k & 1u;
+            ++item_k;
+            constexpr int kV4 = DH / 4;  // float4 slots of a row
+            float4 *slot = reinterpret_cast<float4 *>(sComb + row * DH);
+            if (!ok) break;
+            if (!combiner) {
+                if (!warp_all(mbar_wait(&comb_free[q], ph ^ 1u, abort_flag, p.err))) break;
                 sML[row] = make_float2(m_ref, l_run);
 #pragma unroll
                 for (int d4 = 0; d4 < kV4; ++d4)
-                    mine[d4 ^ (row & (kV4 - 1))] = make_float4(acc[4 * d4], acc[4 * d4 + 1], acc[4 * d4 + 2], acc[4 * d4 + 3]);
+                    slot[d4 ^ (row & (kV4 - 1))] = make_float4(acc[4 * d4], acc[4 * d4 + 1], acc[4 * d4 + 2], acc[4 * d4 + 3]);
+                mbar_arrive(&comb_full[q]);  // every lane: its own row is released
+                continue;
             }
-            asm volatile("bar.sync 1, %0;" ::"n"(kSoftmaxThreads) : "memory");
-            if (par == 0) {
-                const float2 ml1 = sML[row];
-                const float m1 = ml1.x, l1 = ml1.y;
-                const float m = fmaxf(m_ref, m1);
-                const float a0 = exp2_fast(m_ref - m), a1 = exp2_fast(m1 - m);
-                const float inv = 1.0f / (l_run * a0 + l1 * a1);
-                const int orow = it.q_row0 + row;
-                if (orow < it.store_end) {
-                    uint4 *dst = reinterpret_cast<uint4 *>(p.out + (size_t)orow * p.ldo + it.h * DH);
-#pragma unroll
-                    for (int d = 0; d < DH; d += 8) {
-                        const float4 b0 = mine[(d / 4) ^ (row & (kV4 - 1))], b1 = mine[(d / 4 + 1) ^ (row & (kV4 - 1))];
-                        const float ob[8] = {b0.x, b0.y, b0.z, b0.w, b1.x, b1.y, b1.z, b1.w};
-                        float o[8];
-#pragma unroll
-                        for (int e = 0; e < 8; ++e) o[e] = (acc[d + e] * a0 + ob[e] * a1) * inv;
-                        uint4 u;
-                        u.x = pack_bf16x2(o[0], o[1]);
-                        u.y = pack_bf16x2(o[2], o[3]);
-                        u.z = pack_bf16x2(o[4], o[5]);
-                        u.w = pack_bf16x2(o[6], o[7]);
-                        dst[d / 8] = u;
-                    }
-                }
+            if (!warp_all(mbar_wait(&comb_full[q], ph, abort_flag, p.err))) break;
+            // O = (O_0 2^(m_0-m) + O_1 2^(m_1-m)) / (l_0 2^(m_0-m) + l_1 2^(m_1-m)),
+            // in this order whichever parity combines
+            const float2 other = sML[row];
+            const float m0 = par == 0 ? m_ref : other.x, l0 = par == 0 ? l_run : other.y;
+            const float m1 = par == 0 ? other.x : m_ref, l1 = par == 0 ? other.y : l_run;
+            const float m = fmaxf(m0, m1);
+            const float a0 = exp2_fast(m0 - m), a1 = exp2_fast(m1 - m);
+            const float inv = 1.0f / (l0 * a0 + l1 * a1);
+            const int orow = it.q_row0 + row;
+            if (orow < it.store_end) {
+                uint4 *dst = reinterpret_cast<uint4 *>(p.out + (size_t)orow * p.ldo + it.h * DH);
+                if (par == 0)
+                    combine_row<DH, false>(acc, slot, row, a0, a1, inv, dst);
+                else
+                    combine_row<DH, true>(acc, slot, row, a0, a1, inv, dst);
             }
-            // one snapshot of the abort flag, read by every softmax thread
-            // after the barrier, decides for all whether to go on
-            if (threadIdx.x == 64) *stop_flag = *abort_flag;
-            asm volatile("bar.sync 1, %0;" ::"n"(kSoftmaxThreads) : "memory");
-            if (*stop_flag) break;
+            mbar_arrive(&comb_free[q]);  // every lane: its row was read
         }
     }
     __syncthreads();
     if (*abort_flag) {
-        if (warp == 1 && lane == 0) {
-            mma_commit(drain);
-            wait_bounded(drain, 0, 100000000ull);
+        if (warp == 1) {
+            commit_w(drain);  // the MMAs' issuing lane
+            if (lane == 0) wait_bounded(drain, 0, 100000000ull);
         }
         if (threadIdx.x == 0) spin_ns(200000);
         __syncthreads();
