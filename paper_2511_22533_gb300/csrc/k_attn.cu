@@ -95,48 +95,12 @@ F3DC_DEV Item decode_item(const AttnParams &p, int w)
     return it;
 }
 
-// every lane's outcome, so a warp takes the same branch around its
-// warp-collective TMEM accesses even when a bounded wait gives up in one lane
-F3DC_DEV bool warp_all(bool v) { return __all_sync(0xffffffffu, v); }
-
 F3DC_DEV bool wait_bounded(uint64_t *bar, uint32_t parity, uint64_t ns)
 {
     const uint64_t t0 = globaltimer();
     while (!mbar_try_wait(bar, parity))
         if (globaltimer() - t0 > ns) return false;
     return true;
-}
-
-// tcgen05 issue from a converged warp: every lane runs the issuer's loop and
-// elect.sync picks the issuing lane inside each instruction's asm (the same
-// lane every time: the warp is converged and the member mask full, so the
-// commits track the MMAs of the thread that issued them).  Measured in
-// isolation, this form issues the tile's 12 MMAs in ~525 cycles against
-// ~580 for a loop run by lane 0 alone, and keeps ~945 cycles (lane 0 alone:
-// ~2600) when two warps busy with FMAs share the issuer's SM sub-partition,
-// as the softmax warps do here.
-F3DC_DEV void mma_ss_w(uint32_t d, uint64_t a, uint64_t b, uint32_t id, uint32_t acc)
-{
-    asm volatile(
-        "{\n .reg .pred p, e;\n elect.sync _|e, 0xffffffff;\n"
-        " setp.ne.b32 p, %4, 0;\n @e tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n}\n" ::"r"(d),
-        "l"(a), "l"(b), "r"(id), "r"(acc)
-        : "memory");
-}
-F3DC_DEV void mma_ts_w(uint32_t d, uint32_t a, uint64_t b, uint32_t id, uint32_t acc)
-{
-    asm volatile(
-        "{\n .reg .pred p, e;\n elect.sync _|e, 0xffffffff;\n"
-        " setp.ne.b32 p, %4, 0;\n @e tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], %2, %3, p;\n}\n" ::"r"(d),
-        "r"(a), "l"(b), "r"(id), "r"(acc)
-        : "memory");
-}
-F3DC_DEV void commit_w(uint64_t *bar)
-{
-    asm volatile(
-        "{\n .reg .pred e;\n elect.sync _|e, 0xffffffff;\n"
-        " @e tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];\n}\n" ::"r"(smem_u32(bar))
-        : "memory");
 }
 
 // One output row of the end-of-item combine, in parity order whichever
@@ -311,8 +275,8 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
                 const uint64_t kd = k_desc0 + (gt % kKVStages) * kStageStep;
 #pragma unroll
                 for (int kk = 0; kk < DH / 16; ++kk)
-                    mma_ss_w(tmem + (gt & 1) * 128, q_desc + 2 * kk, kd + 2 * kk, idesc_s, kk > 0);
-                if (commit) commit_w(&s_full[gt & 1]);
+                    mma_bf16_elect(tmem + (gt & 1) * 128, q_desc + 2 * kk, kd + 2 * kk, idesc_s, kk > 0);
+                if (commit) mma_commit_elect(&s_full[gt & 1]);
             };
             // O_e (+)= P_e V for tile gt of parity e = gt % 2, P_e read from
             // TMEM (8 columns per 16 keys); `fresh` overwrites O_e (the item's
@@ -322,9 +286,9 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
                 const uint64_t vd = v_desc0 + (gt % kKVStages) * kStageStep;
 #pragma unroll
                 for (int kk = 0; kk < 8; ++kk)  // keys 16kk..16kk+15
-                    mma_ts_w(tmem + Cfg::kColO + pb * DH, tmem + Cfg::kColP + pb * 64 + kk * 8,
+                    mma_bf16_ts_elect(tmem + Cfg::kColO + pb * DH, tmem + Cfg::kColP + pb * 64 + kk * 8,
                                 vd + kk * kVRowStep, idesc_o, !(fresh && kk == 0));
-                commit_w(&kv_empty[gt % kKVStages]);
+                mma_commit_elect(&kv_empty[gt % kKVStages]);
             };
             auto kv_ready = [&](uint32_t gt) { return warp_all(mbar_test(&kv_full[gt % kKVStages], (gt / kKVStages) & 1)); };
             auto kv_wait = [&](uint32_t gt) {
@@ -369,7 +333,7 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
                     pv_mmas(gt, j < 2);  // its commit also reports S_(gt+2)
                 }
                 if (!ok) break;
-                commit_w(&q_empty[qb]);  // every S of the item issued: its Q buffer may be refilled
+                mma_commit_elect(&q_empty[qb]);  // every S of the item issued: its Q buffer may be refilled
                 for (; j < nkt; ++j) {
                     const uint32_t gt = g + j;
                     if (!p_ready(gt) && !p_wait(gt)) {
@@ -598,7 +562,7 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
     __syncthreads();
     if (*abort_flag) {
         if (warp == 1) {
-            commit_w(drain);  // the MMAs' issuing lane
+            mma_commit_elect(drain);  // the MMAs' issuing lane
             if (lane == 0) wait_bounded(drain, 0, 100000000ull);
         }
         if (threadIdx.x == 0) spin_ns(200000);

@@ -429,7 +429,9 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
         // issuer tests the next stage's `full` barrier before issuing the
         // current stage's MMAs, so the read overlaps them, and takes the
         // bounded wait only when the test found the stage not yet loaded.
-        if (lane == 0) {
+        // The whole warp runs the loop (barrier outcomes as warp votes) and
+        // elect.sync issues.
+        {
             constexpr uint32_t idesc_w = make_idesc_bf16(128, BN, 0, 0);
             constexpr uint32_t idesc_n = make_idesc_bf16(128, BN / 2 < 16 ? 16 : BN / 2, 0, 0);
             const uint32_t idesc = narrow ? idesc_n : idesc_w;
@@ -440,33 +442,35 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
             int s = 0, it = 0;
             uint32_t ph = 0;
             bool ok = true;
-            bool ready = mbar_test(&full[0], 0);
+            bool ready = warp_all(mbar_test(&full[0], 0));
             for (int t = blockIdx.x; t < total && ok; t += gridDim.x, ++it) {
                 const int buf = it & 1;
                 const uint32_t aph = (it >> 1) & 1;
-                if (!mbar_test(&acce[buf], aph ^ 1) && !mbar_wait(&acce[buf], aph ^ 1, abort_flag, p.err)) break;
+                if (!warp_all(mbar_test(&acce[buf], aph ^ 1)) &&
+                    !warp_all(mbar_wait(&acce[buf], aph ^ 1, abort_flag, p.err)))
+                    break;
                 const uint32_t d = tmem + buf * BN;
                 int m0, n0, kb0, kb1;
                 U.decode(t, m0, n0, kb0, kb1, bn);
                 for (int kb = kb0; kb < kb1; ++kb) {
-                    if (!ready && !mbar_wait(&full[s], ph, abort_flag, p.err)) {
+                    if (!ready && !warp_all(mbar_wait(&full[s], ph, abort_flag, p.err))) {
                         ok = false;
                         break;
                     }
                     tc_fence_after();
                     const int s_next = s + 1 == S ? 0 : s + 1;
                     const uint32_t ph_next = s_next == 0 ? ph ^ 1 : ph;
-                    ready = mbar_test(&full[s_next], ph_next);  // read overlaps the MMAs below
+                    ready = warp_all(mbar_test(&full[s_next], ph_next));  // read overlaps the MMAs below
                     const uint64_t ad = a_desc0 + (uint64_t)s * (kAStage >> 4);
                     const uint64_t bd = b_desc0 + (uint64_t)s * (Cfg::kBStage >> 4);
 #pragma unroll
                     for (int k = 0; k < kBK / 16; ++k)
-                        mma_bf16(d, ad + 2 * k, bd + 2 * k, idesc, (kb != kb0) || (k != 0));
-                    mma_commit(&empty[s]);
+                        mma_bf16_elect(d, ad + 2 * k, bd + 2 * k, idesc, (kb != kb0) || (k != 0));
+                    mma_commit_elect(&empty[s]);
                     s = s_next;
                     ph = ph_next;
                 }
-                if (ok) mma_commit(&accf[buf]);
+                if (ok) mma_commit_elect(&accf[buf]);
             }
         }
     } else {
@@ -569,9 +573,9 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
     __syncthreads();
     if (*abort_flag) {
         // drain: wait (bounded) for this CTA's outstanding MMAs and copies
-        if (warp == 1 && lane == 0) {
-            mma_commit(drain);
-            mbar_wait_bounded(drain, 0, 100000000ull);
+        if (warp == 1) {
+            mma_commit_elect(drain);  // the MMAs' issuing lane
+            if (lane == 0) mbar_wait_bounded(drain, 0, 100000000ull);
         }
         if (threadIdx.x == 0) spin_ns(200000);
         __syncthreads();
@@ -705,7 +709,9 @@ __global__ void __launch_bounds__(kPairThreads, 1)
             }
         }
     } else if (warp == 1) {
-        if (lane == 0 && rank == 0) {
+        // the even CTA's warp issues for the pair: the whole warp runs the
+        // loop (barrier outcomes as warp votes) and elect.sync issues
+        if (rank == 0) {
             constexpr uint32_t idesc_w = make_idesc_bf16(256, 256, 0, 0);
             constexpr uint32_t idesc_n = make_idesc_bf16(256, 128, 0, 0);
             const uint32_t idesc = narrow ? idesc_n : idesc_w;
@@ -714,33 +720,35 @@ __global__ void __launch_bounds__(kPairThreads, 1)
             int s = 0, it = 0;
             uint32_t ph = 0;
             bool ok = true;
-            bool ready = mbar_test(&full[0], 0);
+            bool ready = warp_all(mbar_test(&full[0], 0));
             for (int t = cl; t < tiles && ok; t += ncl, ++it) {
                 const int buf = it & 1;
                 const uint32_t aph = (it >> 1) & 1;
-                if (!mbar_test(&acce[buf], aph ^ 1) && !mbar_wait(&acce[buf], aph ^ 1, abort_flag, p.err)) break;
+                if (!warp_all(mbar_test(&acce[buf], aph ^ 1)) &&
+                    !warp_all(mbar_wait(&acce[buf], aph ^ 1, abort_flag, p.err)))
+                    break;
                 const uint32_t d = tmem + buf * 256;
                 for (int kb = 0; kb < kb_n; ++kb) {
-                    if (!ready && !mbar_wait(&full[s], ph, abort_flag, p.err)) {
+                    if (!ready && !warp_all(mbar_wait(&full[s], ph, abort_flag, p.err))) {
                         ok = false;
                         break;
                     }
                     tc_fence_after();
                     const int s_next = s + 1 == S ? 0 : s + 1;
                     const uint32_t ph_next = s_next == 0 ? ph ^ 1 : ph;
-                    ready = mbar_test(&full[s_next], ph_next);
+                    ready = warp_all(mbar_test(&full[s_next], ph_next));
                     const uint64_t ad = a_desc0 + (uint64_t)s * (kPairAStage >> 4);
                     const uint64_t bd = b_desc0 + (uint64_t)s * (kPairBStage >> 4);
 #pragma unroll
                     for (int k = 0; k < kPairBK / 16; ++k) {
                         const uint64_t off = (uint64_t)(k >> 2) * (kPairHalf >> 4) + 2 * (k & 3);
-                        mma_bf16_pair(d, ad + off, bd + off, idesc, (kb != 0) || (k != 0));
+                        mma_bf16_pair_elect(d, ad + off, bd + off, idesc, (kb != 0) || (k != 0));
                     }
-                    mma_commit_pair_mc(&empty[s], 3);
+                    mma_commit_pair_mc_elect(&empty[s], 3);
                     s = s_next;
                     ph = ph_next;
                 }
-                if (ok) mma_commit_pair_mc(&accf[buf], 3);
+                if (ok) mma_commit_pair_mc_elect(&accf[buf], 3);
             }
         }
     } else {
@@ -779,9 +787,9 @@ __global__ void __launch_bounds__(kPairThreads, 1)
     }
     __syncthreads();
     if (*abort_flag) {
-        if (warp == 1 && lane == 0 && rank == 0) {
-            mma_commit_pair(drain);
-            mbar_wait_bounded(drain, 0, 100000000ull);
+        if (warp == 1 && rank == 0) {
+            mma_commit_pair_elect(drain);  // the MMAs' issuing lane
+            if (lane == 0) mbar_wait_bounded(drain, 0, 100000000ull);
         }
         if (threadIdx.x == 0) spin_ns(200000);
         __syncthreads();
