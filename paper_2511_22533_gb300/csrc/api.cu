@@ -493,8 +493,9 @@ cudaError_t run_attention(f3dc_handle *h, int mode, const CUtensorMap &tq, const
     p.ldo = h->W;
     p.scale_log2 = (float)(1.4426950408889634 / std::sqrt((double)h->dh));
     p.err = h->dev_err;
-    int items = h->max_tiles * h->H;
-    int grid = items < h->num_sms ? items : h->num_sms;
+    // work items: (pair of query tiles, head)
+    const int items = (h->max_tiles + 1) / 2 * h->H;
+    const int grid = items < h->num_sms ? items : h->num_sms;
     return launch_attention(&tq, &tkv, &tkv, p, grid, s);
 }
 
@@ -1478,7 +1479,7 @@ f3dc_status f3dc_attention(const void *q, int32_t ldq, const void *k, const void
     int dev = 0, sms = 0;
     CK(cudaGetDevice(&dev));
     CK(cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev));
-    const int items = p.n_tiles * heads;
+    const int items = (p.n_tiles + 1) / 2 * heads;  // (pair of query tiles, head)
     CK(launch_attention(&tq, &tk, &tv, p, items < sms ? items : sms, (cudaStream_t)stream));
     return F3DC_OK;
 }

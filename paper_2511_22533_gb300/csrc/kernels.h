@@ -253,6 +253,8 @@ struct AttnParams {
     int fault_skip_kv;
     uint32_t *err;
 };
+// grid: persistent CTAs (at most one per SM), each taking the work items
+// (pair of 128-query tiles, head) in turn.
 cudaError_t launch_attention(const CUtensorMap *tq, const CUtensorMap *tk, const CUtensorMap *tv,
                              const AttnParams &p, int grid, cudaStream_t s);
 size_t attn_smem_bytes(int dh);
