@@ -21,14 +21,16 @@
 //              each once P_t is written; P read straight from TMEM)
 //   warps 2-5  softmax of tile A, warps 6-9 of tile B: one thread per query
 //              row (TMEM lane = row), all 128 keys of each key tile, online
-//              softmax with the row's running max m and sum l.  Pass 1 takes
-//              the tile's maximum; pass 2 reloads S, releases the S buffer
-//              for the next key tile's MMA as soon as its last load landed,
-//              and writes P = exp2(S scale - m) as bf16 pairs into TMEM P_t
-//              (once P V of the previous key tile has read P_t).  O_t stays
-//              in TMEM for the whole item; the reference max m is only raised
-//              (O_t, l rescaled in place) when a tile's max exceeds it by
-//              more than 2^8.  At the item's end O_t / l is stored as bf16.
+//              softmax with the row's running max m and sum l, in one pass
+//              over the key tile's two halves of 64 keys: each half is
+//              loaded once, its maximum raises the reference max m only when
+//              it exceeds m by more than 2^8 (O_t, l rescaled in place; a
+//              raise in the second half recomputes the first half's P), and
+//              P = exp2(S scale - m) goes to TMEM P_t as bf16 pairs (once
+//              P V of the previous key tile has read P_t).  The S buffer is
+//              released for the next key tile's MMA as soon as its last load
+//              landed.  O_t stays in TMEM for the whole item; at the item's
+//              end O_t / l is stored as bf16.
 // TMEM: S_A S_B (fp32, 128 columns each) | O_A O_B (dh each) | P_A P_B (64).
 // V is the MN-major B operand of the P V MMA straight from its row-major
 // TMA tile.  Keys beyond a sample's count are masked to -inf before the
@@ -325,16 +327,71 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
                     break;
                 }
                 tc_fence_after();
-                // pass 1: the tile's maximum (S stays in TMEM for pass 2)
+                // one pass over the tile's two halves of 64 keys: load, take the
+                // half's maximum, raise the reference max when it grew by more
+                // than 2^8 (warp-uniform), then exponents against it.  A raise
+                // in the second half makes the first half's P stale: its S is
+                // still in TMEM (released only after this check), so it is
+                // recomputed against the new max.
                 const int valid = it.nk - j * 128;  // < 128 only on the last, ragged key tile
-                float mx4[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
+                f32x2 sum0 = {0.f, 0.f}, sum1 = {0.f, 0.f};
+                bool pv_ready = gt == 0;  // P V of the previous key tile done (P_t, O_t free)
+                bool o_live = j > 0;      // O_t holds this item's earlier tiles
+                auto ensure_pv = [&]() {
+                    if (!pv_ready) {
+                        pv_ready = wait(&pv_done[t], (gt - 1) & 1);
+                        if (!pv_ready) ok = false;
+                    }
+                    return pv_ready;
+                };
+                auto rescale = [&](float alpha) {
+                    if (o_live) {
+                        tc_fence_after();
 #pragma unroll
-                for (int hb = 0; hb < 2; ++hb) {  // two halves of 64 keys
+                        for (int d0 = 0; d0 < DH; d0 += 16) {
+                            uint32_t r[16];
+                            tmem_ld16(o_addr + d0, r);
+                            tmem_wait_ld();
+#pragma unroll
+                            for (int d = 0; d < 16; ++d) r[d] = __float_as_uint(__uint_as_float(r[d]) * alpha);
+                            tmem_st16(o_addr + d0, r);
+                        }
+                    }
+                    l_run *= alpha;
+                };
+                // exponents of one half against m_ref, P to TMEM as bf16 pairs
+                auto emit_half = [&](int hb, const float (&sv)[64]) {
+                    const float m_use = m_ref == -INFINITY ? 0.f : m_ref;
+                    const f32x2 sc2 = {p.scale_log2, p.scale_log2}, nm2 = {-m_use, -m_use};
+                    f32x2 s0 = {0.f, 0.f}, s1 = {0.f, 0.f};
+                    uint32_t pw[32];
+#pragma unroll
+                    for (int c = 0; c < 32; c += 2) {
+                        const int k0 = 2 * c;
+                        const f32x2 x0 = ffma2({sv[k0], sv[k0 + 1]}, sc2, nm2);
+                        const f32x2 x1 = ffma2({sv[k0 + 2], sv[k0 + 3]}, sc2, nm2);
+                        const f32x2 e0 = {exp2_fast(x0.x), exp2_fast(x0.y)};
+                        const f32x2 e1 = {exp2_fast(x1.x), exp2_fast(x1.y)};
+                        s0 = fadd2(s0, e0);
+                        s1 = fadd2(s1, e1);
+                        pw[c] = pack_bf16x2(e0.x, e0.y);
+                        pw[c + 1] = pack_bf16x2(e1.x, e1.y);
+                    }
+                    if (!ensure_pv()) return;
+                    tmem_st32(p_addr + 32 * hb, pw);
+                    if (hb == 0) {
+                        sum0 = s0;
+                        sum1 = s1;
+                    } else {
+                        sum0 = fadd2(sum0, s0);
+                        sum1 = fadd2(sum1, s1);
+                    }
+                };
+                auto load_half = [&](int hb, float (&sv)[64]) {
                     uint32_t r0[32], r1[32];
                     tmem_ld32(s_addr + 64 * hb, r0);
                     tmem_ld32(s_addr + 64 * hb + 32, r1);
                     tmem_wait_ld();
-                    float sv[64];
 #pragma unroll
                     for (int c = 0; c < 32; ++c) {
                         sv[c] = __uint_as_float(r0[c]);
@@ -345,82 +402,52 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
                         for (int c = 0; c < 64; ++c)
                             if (64 * hb + c >= valid) sv[c] = -INFINITY;
                     }
+                };
+                auto half_max = [&](const float (&sv)[64]) {
+                    float mx4[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
 #pragma unroll
                     for (int c = 0; c < 64; c += 8) {
 #pragma unroll
                         for (int e = 0; e < 4; ++e) mx4[e] = fmax3(mx4[e], sv[c + e], sv[c + 4 + e]);
                     }
-                }
-                const float mx = fmax3(mx4[0], mx4[1], fmaxf(mx4[2], mx4[3])) * p.scale_log2;
-                const bool raise = __any_sync(0xffffffffu, mx > m_ref + 8.0f);
-                float alpha = 1.f;
-                if (raise) {
+                    return fmax3(mx4[0], mx4[1], fmaxf(mx4[2], mx4[3])) * p.scale_log2;
+                };
+                // raise m_ref to cover mx when it grew by more than 2^8; O_t and
+                // l are rescaled (P V of the previous key tile must be done)
+                auto maybe_raise = [&](float mx) {
+                    if (!__any_sync(0xffffffffu, mx > m_ref + 8.0f)) return false;
                     const float m_new = fmaxf(m_ref, mx);
-                    alpha = exp2_fast(m_ref - m_new);
+                    const float alpha = exp2_fast(m_ref - m_new);
                     m_ref = m_new;
-                }
-                const float m_use = m_ref == -INFINITY ? 0.f : m_ref;
-                // P_t and O_t: P V of the previous key tile must be done
-                if (gt >= 1 && !wait(&pv_done[t], (gt - 1) & 1)) {
-                    ok = false;
-                    break;
-                }
-                if (raise && j > 0) {  // O_t holds this item's earlier tiles: rescale in place
-                    tc_fence_after();
-#pragma unroll
-                    for (int d0 = 0; d0 < DH; d0 += 16) {
-                        uint32_t r[16];
-                        tmem_ld16(o_addr + d0, r);
-                        tmem_wait_ld();
-#pragma unroll
-                        for (int d = 0; d < 16; ++d) r[d] = __float_as_uint(__uint_as_float(r[d]) * alpha);
-                        tmem_st16(o_addr + d0, r);
-                    }
-                    l_run *= alpha;
-                }
-                // pass 2: exponents and row sums; P to TMEM as bf16 pairs.  Once
-                // the second half's S is loaded, S_t is released for the next
-                // key tile's MMA
-                f32x2 sum0 = {0.f, 0.f}, sum1 = {0.f, 0.f};
-                const f32x2 sc2 = {p.scale_log2, p.scale_log2}, nm2 = {-m_use, -m_use};
-#pragma unroll
-                for (int hb = 0; hb < 2; ++hb) {
+                    if (ensure_pv()) rescale(alpha);
+                    return true;
+                };
+                {
                     float sv[64];
-                    {
-                        uint32_t r0[32], r1[32];
-                        tmem_ld32(s_addr + 64 * hb, r0);
-                        tmem_ld32(s_addr + 64 * hb + 32, r1);
-                        tmem_wait_ld();
-#pragma unroll
-                        for (int c = 0; c < 32; ++c) {
-                            sv[c] = __uint_as_float(r0[c]);
-                            sv[32 + c] = __uint_as_float(r1[c]);
-                        }
+                    load_half(0, sv);
+                    maybe_raise(half_max(sv));
+                    if (!ok) break;
+                    emit_half(0, sv);
+                    if (!ok) break;
+                }
+                {
+                    float sv[64];
+                    load_half(1, sv);
+                    const bool raised = maybe_raise(half_max(sv));
+                    if (!ok) break;
+                    if (raised) {
+                        // the first half's P is against the old max: redo it
+                        float sv0[64];
+                        load_half(0, sv0);
+                        emit_half(0, sv0);
+                        if (!ok) break;
                     }
-                    if (hb == 1) {
-                        tc_fence_before();
-                        __syncwarp();
-                        if (lane == 0) mbar_arrive(&s_free[t]);
-                    }
-                    if (valid < 128) {
-#pragma unroll
-                        for (int c = 0; c < 64; ++c)
-                            if (64 * hb + c >= valid) sv[c] = -INFINITY;
-                    }
-                    uint32_t pw[32];
-#pragma unroll
-                    for (int c = 0; c < 32; c += 2) {
-                        const int k0 = 2 * c;
-                        const f32x2 x0 = ffma2({sv[k0], sv[k0 + 1]}, sc2, nm2);
-                        const f32x2 x1 = ffma2({sv[k0 + 2], sv[k0 + 3]}, sc2, nm2);
-                        const f32x2 e0 = {exp2_fast(x0.x), exp2_fast(x0.y)};
-                        const f32x2 e1 = {exp2_fast(x1.x), exp2_fast(x1.y)};
-                        sum0 = fadd2(sum0, e0);
-                        sum1 = fadd2(sum1, e1);
-                        pw[c] = pack_bf16x2(e0.x, e0.y);
-                        pw[c + 1] = pack_bf16x2(e1.x, e1.y);
-                    }
-                    tmem_st32(p_addr + 32 * hb, pw);
+                    // S_t fully read: the next key tile's S may overwrite it
+                    tc_fence_before();
+                    __syncwarp();
+                    if (lane == 0) mbar_arrive(&s_free[t]);
+                    emit_half(1, sv);
+                    if (!ok) break;
                 }
                 tmem_wait_st();
                 l_run += (sum0.x + sum0.y) + (sum1.x + sum1.y);

@@ -49,15 +49,17 @@ def test_attention_rows_beyond_nq_untouched():
 
 def _rescale_case(nq, nk, H, dh, seed):
     """Queries and keys along one direction u per head (entries +-1) so that
-    each row's scores are set per key tile.  The first two tiles (one per
-    parity) hold keys of strength 1; tile j >= 2 holds keys one strength step
-    above the previous tile of its parity -- all its keys, except in the last
-    tile of each parity, which holds a single such key.  A step is worth
-    8.4-9.3 log2 units of scaled score for query strengths in [0.9, 1], just
-    past the kernel's 2^8 margin, so each parity raises its reference max
-    (and rescales O and l in place) at every later tile, while the full tiles
-    before a parity's last one keep a visible share of the softmax weight;
-    the last tile is ragged."""
+    each row's scores are set per key tile.  The first two tiles hold keys of
+    strength 1; tile j >= 2 holds keys one strength step above tile j - 2 --
+    all its keys, except in the last two tiles, which hold a single such key
+    each (at position 37 j within the tile).  A step is worth 8.4-9.3 log2
+    units of scaled score for query strengths in [0.9, 1], just past the
+    kernel's 2^8 margin, so the reference max is raised (and O and l
+    rescaled in place) at every even tile from 2 on, while the full tiles
+    before the last ones keep a visible share of the softmax weight; the
+    last tile is ragged.  With 900 keys the single strong key of tile 6 sits
+    in the tile's second half (position 94), so the raise comes after the
+    first half's P was written and the kernel recomputes it."""
     g = np.random.default_rng(seed)
     W = H * dh
     u = np.where(g.random((H, dh)) < 0.5, -1.0, 1.0)
@@ -77,13 +79,13 @@ def _rescale_case(nq, nk, H, dh, seed):
     return [synth.f32_to_bf16_bits(x.astype(np.float32)) for x in (q, k, v)]
 
 
-@pytest.mark.parametrize("nq,nk,H,dh", [(256, 700, 2, 64), (200, 900, 2, 32), (130, 641, 1, 64)])
+@pytest.mark.parametrize("nq,nk,H,dh", [(256, 700, 2, 64), (200, 900, 2, 32), (256, 900, 2, 64), (130, 641, 1, 64)])
 def test_attention_reference_max_raised_in_late_tiles(orc, nq, nk, H, dh):
     # the kernel keeps a per-row reference max and raises it (rescaling O and
-    # l in TMEM) only when a key tile's max exceeds it by more than 2^8; keys
-    # drawn N(0, 1) never get there, so these cases place the strongest keys
-    # in late tiles of both parities and check the outcome against the
-    # oracle's fp64 softmax attention
+    # l in TMEM) only when a half key tile's max exceeds it by more than 2^8;
+    # keys drawn N(0, 1) never get there, so these cases place the strongest
+    # keys in late tiles (and, with 900 keys, in a tile's second half) and
+    # check the outcome against the oracle's fp64 softmax attention
     W = H * dh
     q, k, v = _rescale_case(nq, nk, H, dh, nq + nk)
     qf, kf, vf = (synth.bf16_bits_to_f32(x).astype(np.float64) for x in (q, k, v))
