@@ -51,7 +51,7 @@ FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustain
 GEMM_TRAFFIC = {"dram_bytes_per_launch": 68.9e6 / 6, "algorithmic_bytes_per_launch": 67.1e6 / 6,
                 "shape": "QKV, attention out, cross Q, cross out, fc1, fc2 at 1229 active rows, width 1024",
                 "profile": "profiles/k_gemm_pair_cached_step_1229rows.md",
-                "k_gemm_cu_sha256": "1c2cbc85b684b77c0b482c531383b424fd7530a096cd28cbff42e463c0121b2d"}
+                "k_gemm_cu_sha256": "d080472e424c0a678d801a1a68e8872efd72620b4b902365757673d2778e0f3e"}
 
 
 def parse():
