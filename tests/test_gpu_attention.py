@@ -1,7 +1,9 @@
 """K5 / K6 parity: the tcgen05 flash attention against the oracle's fp64
 softmax attention (Supp. Sec. F self- and cross-attention) on sampled query
 rows: active-token sequences (ragged, 1229, 4096), the 1374-token condition,
-head dims 32 and 64, a single key and odd tails."""
+head dims 32 and 64, a single key and odd tails.  The kernel's work items
+are pairs of query tiles; an odd tile count (e.g. 2600 queries: 21 tiles)
+leaves the last pair with rows that are computed and never stored."""
 import numpy as np
 import pytest
 import torch
@@ -13,7 +15,7 @@ pytestmark = pytest.mark.gpu
 
 CASES = [(300, 300, 4, 32), (1229, 1229, 16, 64), (4096, 4096, 16, 64), (1229, 1374, 16, 64), (5, 1, 2, 64),
          (130, 129, 2, 32), (128, 256, 1, 64), (700, 77, 4, 32), (256, 256, 1, 64), (128, 384, 1, 64),
-         (1, 200, 1, 32), (128, 129, 1, 64)]
+         (1, 200, 1, 32), (128, 129, 1, 64), (2600, 700, 8, 32)]
 
 
 @pytest.mark.parametrize("nq,nk,H,dh", CASES)
@@ -79,13 +81,15 @@ def _rescale_case(nq, nk, H, dh, seed):
     return [synth.f32_to_bf16_bits(x.astype(np.float32)) for x in (q, k, v)]
 
 
-@pytest.mark.parametrize("nq,nk,H,dh", [(256, 700, 2, 64), (200, 900, 2, 32), (256, 900, 2, 64), (130, 641, 1, 64)])
+@pytest.mark.parametrize("nq,nk,H,dh", [(256, 700, 2, 64), (200, 900, 2, 32), (256, 900, 2, 64), (130, 641, 1, 64),
+                                        (1280, 900, 16, 64)])
 def test_attention_reference_max_raised_in_late_tiles(orc, nq, nk, H, dh):
     # the kernel keeps a per-row reference max and raises it (rescaling O and
     # l in TMEM) only when a half key tile's max exceeds it by more than 2^8;
     # keys drawn N(0, 1) never get there, so these cases place the strongest
     # keys in late tiles (and, with 900 keys, in a tile's second half) and
-    # check the outcome against the oracle's fp64 softmax attention
+    # check the outcome against the oracle's fp64 softmax attention.  The
+    # 1280-query, 16-head case fills 80 CTAs with pairs of query tiles.
     W = H * dh
     q, k, v = _rescale_case(nq, nk, H, dh, nq + nk)
     qf, kf, vf = (synth.bf16_bits_to_f32(x).astype(np.float64) for x in (q, k, v))
