@@ -93,10 +93,10 @@ def test_attention_reference_max_raised_in_late_tiles(orc, nq, nk, H, dh):
     W = H * dh
     q, k, v = _rescale_case(nq, nk, H, dh, nq + nk)
     qf, kf, vf = (synth.bf16_bits_to_f32(x).astype(np.float64) for x in (q, k, v))
-    # the branch is taken: per row and head, every later tile of a parity
-    # beats the previous tile of that parity by more than 8 (log2 units of
-    # scaled score), with a margin for fp32 scores; and the raised-over tiles
-    # still carry a visible share of the softmax weight
+    # the branch is taken: per row and head, every tile from the third on
+    # beats the tile two before it by more than 8 (log2 units of scaled
+    # score), with a margin for fp32 scores; and the raised-over tiles still
+    # carry a visible share of the softmax weight
     sc = np.einsum("rhd,jhd->rhj", qf.reshape(nq, H, dh), kf.reshape(nk, H, dh)) * np.log2(np.e) / np.sqrt(dh)
     nkt = (nk + 127) // 128
     tmax = np.stack([sc[:, :, 128 * j:min(nk, 128 * j + 128)].max(axis=2) for j in range(nkt)], axis=2)

@@ -90,9 +90,11 @@ def test_create_reports_oom_and_frees(n):
 
 def test_attention_wait_runs_out_and_is_reported(orc):
     # the attention kernel's first CTA is told to skip the load of its first
-    # item's last key tile (the earlier tiles go through): the MMA issuer's and the softmax warps' bounded waits on it run
-    # out (1 s), every warp leaves the work loop together, the kernel returns
-    # and the timeout is reported; the next call computes the right result
+    # item's last key tile (the earlier tiles go through): the MMA issuer's
+    # and then the softmax warps' bounded waits run out (1 s, the others
+    # seeing the abort flag), every warp leaves its work loop, the kernel
+    # returns and the timeout is reported; the next call computes the right
+    # result
     nq, nk, H, dh = 256, 512, 2, 64
     W = H * dh
     g = np.random.default_rng(3)
