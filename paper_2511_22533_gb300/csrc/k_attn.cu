@@ -181,6 +181,8 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
         tmem_relinquish();
     }
     if (p.kv_prefetch_rows > 0 && warp == 0 && lane == 0) {
+        // keys / values written long before this launch (the condition's):
+        // pull this CTA's share into L2 while the previous kernel finishes
         const int rb = (p.kv_prefetch_rows + 127) / 128, boxes = rb * p.heads * 2;
         for (int i = blockIdx.x; i < boxes; i += gridDim.x) {
             const int r = i % rb, hk = i / rb, h = hk >> 1;
@@ -191,6 +193,7 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
     __syncthreads();
     tc_fence_after();
     const uint32_t tmem = *tmem_holder;
+    // the previous kernel's outputs (Q / K / V, the row plan) are complete
     griddep_wait();
     const int n_tiles = p.n_tiles_dev ? *p.n_tiles_dev : p.n_tiles;
     const int total = total_items(p, n_tiles);
@@ -207,6 +210,7 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
                 Item it;
                 if (!decode_item(p, w, n_tiles, it)) continue;
                 const uint32_t my_it = item_it++;
+                // Q buffer qb holds items qb, qb + 2, ...: its (my_it / 2)-th use
                 const uint32_t qb = my_it & 1, qph = (my_it >> 1) & 1;
                 if (!mbar_wait(&q_empty[qb], qph ^ 1, abort_flag, p.err)) break;
                 mbar_arrive_expect_tx(&q_full[qb], 2 * Cfg::kTileBytes);
@@ -221,6 +225,10 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
                         ok = false;
                         break;
                     }
+                    // fault injection (tests of the failure path): the last
+                    // key tile of CTA 0's first item is never loaded, so the
+                    // waits on it (and on what follows it) run out while the
+                    // earlier tiles went through, and the kernel aborts
                     if (p.fault_skip_kv && blockIdx.x == 0 && my_it == 0 && j == nkt - 1) continue;
                     mbar_arrive_expect_tx(&kv_full[s], 2 * Cfg::kTileBytes);
                     tma_load_2d(sK + s * Cfg::kTileBytes, &tmk, p.k_col0 + it.h * DH, it.kv_row0 + j * 128,
@@ -232,9 +240,17 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
         }
     } else if (warp == 1) {
         // ------------------------------------------------ MMA issuer
+        // Every lane runs the loop (a converged warp keeps the descriptors
+        // warp-uniform) and takes each barrier outcome as a warp vote;
+        // elect.sync issues.  Key tile g (counted over the CTA's whole run)
+        // sits in K/V stage g % kKVStages; every barrier here completes once
+        // per key tile (or per item), so its phase parity follows from g.
         {
             constexpr uint32_t idesc_s = make_idesc_bf16(128, 128, 0, 0);
             constexpr uint32_t idesc_o = make_idesc_bf16(128, DH, 0, 1);
+            // descriptors of the stage bases; a K step of 16 elements inside a
+            // 128B / 64B swizzle atom advances the start address by 32 bytes,
+            // i.e. the descriptor by 2
             const uint64_t q_desc0 = make_sdesc(smem_u32(sQ), 16, Cfg::kAtom, Cfg::kSwz);
             const uint64_t k_desc0 = make_sdesc(smem_u32(sK), 16, Cfg::kAtom, Cfg::kSwz);
             const uint64_t v_desc0 = make_sdesc(smem_u32(sV), Cfg::kAtom, Cfg::kAtom, Cfg::kSwz);
@@ -249,6 +265,10 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
                 const uint32_t nkt = (uint32_t)((it.nk + 127) / 128);
                 const uint32_t qb = my_it & 1;
                 if (!wait(&q_full[qb], (my_it >> 1) & 1)) break;
+                // step j: S of key tile j (j < nkt), then P V of key tile j - 1
+                // (j >= 1); every item has at least one key tile (a sample
+                // without active tokens owns no query tile, and the entry
+                // points reject nk < 1)
                 for (uint32_t j = 0; j <= nkt && ok; ++j) {
                     if (j < nkt) {
                         // S_A and S_B of key tile gt, each once the softmax
@@ -280,7 +300,8 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
                         const bool fresh = j == 1;
                         const uint64_t vd = v_desc0 + (gp % kKVStages) * kStageStep;
                         for (int t = 0; t < 2; ++t) {
-                            // the item's first P V overwrites O_t: the softmax has read the previous item's
+                            // the item's first P V overwrites O_t: the softmax
+                            // must have read the previous item's
                             if (fresh && !wait(&o_free[t], (my_it & 1) ^ 1)) {
                                 ok = false;
                                 break;
@@ -313,7 +334,11 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
         const uint32_t o_addr = tmem + tl + Cfg::kColO + t * DH;
         const uint32_t p_addr = tmem + tl + Cfg::kColP + t * 64;
         auto wait = [&](uint64_t *bar, uint32_t ph) { return warp_all(mbar_wait(bar, ph, abort_flag, p.err)); };
-        uint32_t g = 0;
+        // S_t of key tile g completes s_full[t] (phase g), the four warps'
+        // arrivals on s_free[t] / p_full[t] complete phase g once S_t is
+        // loaded / P_t written, and P_t V of tile g completes pv_done[t]; a
+        // wait that gives up (the kernel is aborting) ends this warp's loop
+        uint32_t g = 0;  // key tiles of this CTA's earlier items
         for (int w = blockIdx.x; w < total; w += gridDim.x) {
             Item it;
             if (!decode_item(p, w, n_tiles, it)) continue;
