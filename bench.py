@@ -63,11 +63,12 @@ def parse():
     return p.parse_args()
 
 
-def gemm_traffic():
-    """The captured GEMM traffic per launch, or None once k_gemm.cu has changed
-    since the counters were taken."""
+def gemm_traffic(path=None):
+    """The captured GEMM traffic per launch, or None once k_gemm.cu (or the
+    file at `path`) differs from the source the counters were taken on."""
     import hashlib
-    path = os.path.join(ROOT, "paper_2511_22533_gb300", "csrc", "k_gemm.cu")
+    if path is None:
+        path = os.path.join(ROOT, "paper_2511_22533_gb300", "csrc", "k_gemm.cu")
     try:
         with open(path, "rb") as f:
             sha = hashlib.sha256(f.read()).hexdigest()
