@@ -18,7 +18,7 @@ BUILD = os.path.join(HERE, "_build")
 LIB = os.path.join(BUILD, "libf3dc.so")
 INCLUDE = os.path.join(os.path.dirname(HERE), "include")
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
-SOURCES = ["api.cu", "k_select.cu", "k_rows.cu", "k_gemm.cu", "k_attn.cu", "k_decode.cu", "noalloc.cu"]
+SOURCES = ["api.cu", "k_select.cu", "k_rows.cu", "k_gemm.cu", "k_attn.cu", "k_attn_one.cu", "k_decode.cu", "noalloc.cu"]
 
 
 def _nvcc() -> str:

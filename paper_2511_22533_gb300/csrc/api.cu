@@ -295,6 +295,11 @@ struct f3dc_handle {
     float *dec_scratch = nullptr;  // convolutional decoder (cfg.decoder == 1)
     uint32_t *dec_bits = nullptr;
     int cfg_B_now = 0;  // guided step in flight: samples >= cfg_B_now are the unguided copies
+    // f3dc_sample's host copy of every step's quotas ([k * B + b]) while it
+    // runs its steps (null otherwise), and whether the step in flight takes
+    // the one-tile attention kernel (its query-tile count known on the host)
+    const int32_t *hq_steps = nullptr;
+    bool attn_one_now = false;
     // pinned per-step quota slots, two generations so one sampler call can
     // be enqueued while the previous one still copies from its slots
     int32_t *h_quota = nullptr;
@@ -310,6 +315,7 @@ struct f3dc_handle {
     struct SegmentGraph {
         int B, k0, k1, ka;
         float *S;
+        std::vector<uint8_t> attn_one;  // per step k0..k1: the attention kernel captured
         cudaGraphExec_t exec;
         int64_t launches;
     };
@@ -494,9 +500,37 @@ cudaError_t run_attention(f3dc_handle *h, int mode, const CUtensorMap &tq, const
     p.scale_log2 = (float)(1.4426950408889634 / std::sqrt((double)h->dh));
     p.err = h->dev_err;
     // work items: (pair of query tiles, head)
-    const int items = (h->max_tiles + 1) / 2 * h->H;
+    // persistent CTAs, one per work item up to one per SM: (query tile, head)
+    // items for the one-tile kernel, (pair of query tiles, head) otherwise
+    const bool one = h->attn_one_now;
+    const int items = one ? h->max_tiles * h->H : (h->max_tiles + 1) / 2 * h->H;
     const int grid = items < h->num_sms ? items : h->num_sms;
-    return launch_attention(&tq, &tkv, &tkv, p, grid, s);
+    return one ? launch_attention_one(&tq, &tkv, &tkv, p, grid, s) : launch_attention(&tq, &tkv, &tkv, p, grid, s);
+}
+
+// Whether step k's attention takes the one-tile kernel: only when the step's
+// quotas are known on the host (f3dc_sample) and its query tiles (each
+// sample's active rows padded to 128, doubled on a guided step) times the
+// heads fit one item per SM.  Both kernels compute the same attention; this
+// only picks the faster one.
+bool step_attn_one(const f3dc_handle *h, int k, int B, bool guided)
+{
+    if (!h->hq_steps) return false;
+    int64_t tiles = 0;
+    for (int b = 0; b < B; ++b) {
+        int c = h->hq_steps[(size_t)k * B + b];
+        c = c < 0 ? 0 : (c > h->N ? h->N : c);
+        tiles += (h->N - c + kTileRows - 1) / kTileRows;
+    }
+    if (guided) tiles *= 2;
+    return attn_one_tile(tiles, h->H, h->num_sms);
+}
+
+bool step_guided(const f3dc_handle *h, int k)
+{
+    std::vector<float> t(h->T + 1);
+    time_schedule(h->cfg, t.data());
+    return h->cfg.cfg_strength > 0.0 && (double)t[k - 1] >= h->cfg.cfg_t_lo;
 }
 
 // The flow transformer on the packed active rows described by h->plan,
@@ -572,9 +606,13 @@ f3dc_status run_dit(f3dc_handle *h, float t, const float *S, cudaStream_t s, con
 // plan from device memory, so the graph is valid for any quotas).
 f3dc_status run_segment_graph(f3dc_handle *h, int B, float *S, int k0, int k1, int ka, cudaStream_t s)
 {
+    // the attention kernel of each step is part of the captured graph: a
+    // replay whose quotas pick other kernels captures anew
+    std::vector<uint8_t> one((size_t)(k1 - k0 + 1));
+    for (int k = k0; k <= k1; ++k) one[(size_t)(k - k0)] = step_attn_one(h, k, B, step_guided(h, k)) ? 1 : 0;
     f3dc_handle::SegmentGraph *g = nullptr;
     for (auto &e : h->graphs)
-        if (e.B == B && e.S == S && e.k0 == k0 && e.k1 == k1 && e.ka == ka) g = &e;
+        if (e.B == B && e.S == S && e.k0 == k0 && e.k1 == k1 && e.ka == ka && e.attn_one == one) g = &e;
     if (!g) {
         if (h->graphs.size() >= 8) {
             cudaGraphExecDestroy(h->graphs.front().exec);
@@ -599,7 +637,7 @@ f3dc_status run_segment_graph(f3dc_handle *h, int B, float *S, int k0, int k1, i
         e = cudaGraphInstantiate(&exec, graph, 0);
         cudaGraphDestroy(graph);
         CK(e);
-        h->graphs.push_back(f3dc_handle::SegmentGraph{B, k0, k1, ka, S, exec, captured});
+        h->graphs.push_back(f3dc_handle::SegmentGraph{B, k0, k1, ka, S, one, exec, captured});
         g = &h->graphs.back();
     }
     CK(cudaEventRecord(h->ev_in, s));
@@ -1060,9 +1098,11 @@ f3dc_status f3dc_step(f3dc_handle *h, int32_t k, int32_t B, float *S_inout, void
 
     // FlowTransformer on the active tokens at t_k
     h->cfg_B_now = guided ? B : 0;
+    h->attn_one_now = step_attn_one(h, k, B, guided);
     f3dc_status st = run_dit(h, t[k - 1], S_inout, s,
                              h->mod_pre ? h->mod_all + (size_t)(k - 1) * h->mod_rows : nullptr);
     h->cfg_B_now = 0;
+    h->attn_one_now = false;
     if (st != F3DC_OK) return st;
 
     // merge + Euler + history (Algorithm 1 step 3)
@@ -1160,7 +1200,14 @@ static f3dc_status sample_run(f3dc_handle *h, float *S_inout, const void *cond, 
                 if (quota_log) quota_log[(size_t)(k - 1) * B + b] = hq[(size_t)k * B + b];
             }
     };
+    // the steps' quotas stay readable on the host while they run (kernel choice)
+    struct HostQuotas {
+        f3dc_handle *h;
+        HostQuotas(f3dc_handle *hh, const int32_t *q) : h(hh) { h->hq_steps = q; }
+        ~HostQuotas() { h->hq_steps = nullptr; }
+    };
     auto run = [&](int k0, int k1) -> f3dc_status {
+        HostQuotas hq_guard(h, hq);
         CK(cudaMemcpyAsync(h->quota_dev + (size_t)k0 * B, hq + (size_t)k0 * B, (size_t)(k1 - k0 + 1) * B * sizeof(int32_t),
                            cudaMemcpyHostToDevice, s));
         if (h->use_graphs && !h->prof.on) return run_segment_graph(h, B, S_inout, k0, k1, ka, s);
@@ -1479,8 +1526,13 @@ f3dc_status f3dc_attention(const void *q, int32_t ldq, const void *k, const void
     int dev = 0, sms = 0;
     CK(cudaGetDevice(&dev));
     CK(cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev));
-    const int items = (p.n_tiles + 1) / 2 * heads;  // (pair of query tiles, head)
-    CK(launch_attention(&tq, &tk, &tv, p, items < sms ? items : sms, (cudaStream_t)stream));
+    // one-tile items when each gets an SM of its own, pairs of query tiles otherwise
+    if (attn_one_tile(p.n_tiles, heads, sms)) {
+        CK(launch_attention_one(&tq, &tk, &tv, p, p.n_tiles * heads, (cudaStream_t)stream));
+    } else {
+        const int items = (p.n_tiles + 1) / 2 * heads;  // (pair of query tiles, head)
+        CK(launch_attention(&tq, &tk, &tv, p, items < sms ? items : sms, (cudaStream_t)stream));
+    }
     return F3DC_OK;
 }
 

@@ -257,6 +257,12 @@ struct AttnParams {
 // (pair of 128-query tiles, head) in turn.
 cudaError_t launch_attention(const CUtensorMap *tq, const CUtensorMap *tk, const CUtensorMap *tv,
                              const AttnParams &p, int grid, cudaStream_t s);
+// The same attention with one query tile per work item (k_attn_one.cu): the
+// faster kernel when every (query tile, head) item gets a CTA of its own,
+// i.e. tiles * heads <= grid (attn_one_tile).
+cudaError_t launch_attention_one(const CUtensorMap *tq, const CUtensorMap *tk, const CUtensorMap *tv,
+                                 const AttnParams &p, int grid, cudaStream_t s);
+inline bool attn_one_tile(int64_t tiles, int heads, int grid) { return tiles * heads <= grid; }
 size_t attn_smem_bytes(int dh);
 
 // ------------------------------------------------------------ host helpers

@@ -1,9 +1,12 @@
 """K5 / K6 parity: the tcgen05 flash attention against the oracle's fp64
 softmax attention (Supp. Sec. F self- and cross-attention) on sampled query
 rows: active-token sequences (ragged, 1229, 4096), the 1374-token condition,
-head dims 32 and 64, a single key and odd tails.  The kernel's work items
-are pairs of query tiles; an odd tile count (e.g. 2600 queries: 21 tiles)
-leaves the last pair with rows that are computed and never stored."""
+head dims 32 and 64, a single key and odd tails.  f3dc_attention runs the
+one-tile kernel (k_attn_one.cu) when every (query tile, head) item gets an
+SM of its own and the pair kernel (k_attn.cu) otherwise: on a 152-SM GB300
+the cases with more than 152 items (1229 x 16 heads, 4096 x 16, 2600 x 8,
+whose odd tile count leaves the last pair half empty) take the pair kernel,
+the others the one-tile kernel."""
 import numpy as np
 import pytest
 import torch
@@ -89,7 +92,8 @@ def test_attention_reference_max_raised_in_late_tiles(orc, nq, nk, H, dh):
     # keys drawn N(0, 1) never get there, so these cases place the strongest
     # keys in late tiles (and, with 900 keys, in a tile's second half) and
     # check the outcome against the oracle's fp64 softmax attention.  The
-    # 1280-query, 16-head case fills 80 CTAs with pairs of query tiles.
+    # 1280-query, 16-head case (160 items) takes the pair kernel, the others
+    # the one-tile kernel.
     W = H * dh
     q, k, v = _rescale_case(nq, nk, H, dh, nq + nk)
     qf, kf, vf = (synth.bf16_bits_to_f32(x).astype(np.float64) for x in (q, k, v))

@@ -88,14 +88,16 @@ def test_create_reports_oom_and_frees(n):
     _tiny_step_clean()
 
 
-def test_attention_wait_runs_out_and_is_reported(orc):
+@pytest.mark.parametrize("nq,H", [(256, 2), (2600, 8)])
+def test_attention_wait_runs_out_and_is_reported(orc, nq, H):
     # the attention kernel's first CTA is told to skip the load of its first
     # item's last key tile (the earlier tiles go through): the MMA issuer's
     # and then the softmax warps' bounded waits run out (1 s, the others
     # seeing the abort flag), every warp leaves its work loop, the kernel
     # returns and the timeout is reported; the next call computes the right
-    # result
-    nq, nk, H, dh = 256, 512, 2, 64
+    # result.  256 queries x 2 heads run the one-tile kernel, 2600 x 8 (168
+    # tile-head items on 152 SMs) the pair kernel.
+    nk, dh = 512, 64
     W = H * dh
     g = np.random.default_rng(3)
     q = synth.f32_to_bf16_bits(g.standard_normal((nq, W)).astype(np.float32))
