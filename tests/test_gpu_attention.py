@@ -18,7 +18,7 @@ pytestmark = pytest.mark.gpu
 
 CASES = [(300, 300, 4, 32), (1229, 1229, 16, 64), (4096, 4096, 16, 64), (1229, 1374, 16, 64), (5, 1, 2, 64),
          (130, 129, 2, 32), (128, 256, 1, 64), (700, 77, 4, 32), (256, 256, 1, 64), (128, 384, 1, 64),
-         (1, 200, 1, 32), (128, 129, 1, 64), (2600, 700, 8, 32)]
+         (1, 200, 1, 32), (128, 129, 1, 64), (2600, 700, 8, 32), (955, 1374, 16, 64)]
 
 
 @pytest.mark.parametrize("nq,nk,H,dh", CASES)
